@@ -1,0 +1,404 @@
+#!/usr/bin/env python3
+"""Benchmark of the GASLoC replica-update path on GB300.
+
+One step = one outer round of the whole hot path on the workload's replicas,
+already resident in HBM: H local AdamW steps for every worker (K_adamw), the
+round's neighbour table where it is random (K_topo), and the gossip round with
+the outer optimizer and the fused consensus-error reduction (K_gossip).
+
+Prints ONE JSON line (rank 0).  `value` is replica-element updates per second
+over the timed rounds (n_workers * n_params * rounds / time, summed over ranks
+that each run their own replica set: multi-GPU runs are independent replicas).
+`e2e` repeats the measurement through the public C ABI from host buffers:
+upload of the initial replicas, centres and curvature from pinned host memory,
+every round's consensus error read back to the host, and the network average
+read back at the end.  `roofline` is the dominant kernel's algorithmic bytes
+per launch over its CUDA-event duration, against the measured HBM copy peak.
+`cpu_baseline` is the CPU oracle timed on the host cores on a bounded slice.
+
+--impl reference runs the CPU oracle as the reference arm (there is no
+released code for the paper; the oracle written from it is the baseline).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "replica-element updates/sec per gossip round; achieved HBM GB/s vs 8 TB/s"
+UNIT = "replica-element updates/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gasloc", choices=["gasloc", "reference"])
+    ap.add_argument("--workload", default=None)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+def peak_hbm():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel
+    source is unchanged since the capture (else None)."""
+    prof = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
+    src = os.path.join(ROOT, "paper_2606_11081_gb300", "csrc", "%s.cu" % kernel)
+    try:
+        text = open(prof).read()
+        m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+        h = re.search(r"source_sha256:\s*([0-9a-f]+)", text)
+        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if m and h and h.group(1) == cur:
+            return float(m.group(1))
+    except Exception:
+        pass
+    return None
+
+
+class ClockSampler:
+    """Samples nvidia-smi during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                smax.append(float(p[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, p[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def cpu_baseline(w, seconds: float):
+    """Times the CPU oracle (fp32 build) on a slice of the workload's
+    parameter indices: full n_workers, the workload's H, whole rounds."""
+    import oracle
+    oracle.build()
+    orc = oracle.get("f32")
+    from paper_2606_11081_gb300 import workloads as wl
+    hp = wl.hparams_of(w)
+    topo, torus = w.topology, (0, 0)
+    if topo.startswith("torus:"):
+        r, c = topo[6:].split("x")
+        topo, torus = "torus", (int(r), int(c))
+    slice_p = 1 << 20
+    pb = oracle.make_problem(w.n_workers, w.n_params, topo, seed=w.seed, torus=torus,
+                             **{k: (bool(v) if k == "per_worker_h" else v) for k, v in hp.items()})
+    import numpy as np
+    kidx = np.arange(slice_p, dtype=np.int64)
+    st = orc.state(pb, kidx)
+    Hi = orc.draw_local_steps(w.seed, w.n_workers, w.draw_hmax) if w.H < 0 else None
+    rounds = 0
+    t0 = time.perf_counter()
+    while True:
+        st.local_steps(w.H if w.H > 0 else 0, Hi)
+        st.gossip_round()
+        st.consensus_error()
+        rounds += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or rounds >= 1000:
+            break
+    value = w.n_workers * slice_p * rounds / el
+    return {"value": value, "unit": UNIT, "cores": orc.lib.oc_num_threads(), "kind": "oracle",
+            "sample": "%d rounds of the workload on parameter indices [0, %d) with all %d workers "
+                      "(fp32 oracle, OpenMP over elements), %.1f s" % (rounds, slice_p, w.n_workers, el)}
+
+
+def run_reference(args, w):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import numpy as np
+    import oracle
+    from paper_2606_11081_gb300 import workloads as wl
+    oracle.build()
+    orc = oracle.get("f32")
+    hp = wl.hparams_of(w)
+    topo, torus = w.topology, (0, 0)
+    if topo.startswith("torus:"):
+        r, c = topo[6:].split("x")
+        topo, torus = "torus", (int(r), int(c))
+    pb = oracle.make_problem(w.n_workers, w.n_params, topo, seed=w.seed, torus=torus,
+                             **{k: (bool(v) if k == "per_worker_h" else v) for k, v in hp.items()})
+    slice_p = 1 << 18
+    st = orc.state(pb, np.arange(slice_p, dtype=np.int64))
+    Hi = orc.draw_local_steps(w.seed, w.n_workers, w.draw_hmax) if w.H < 0 else None
+
+    def step():
+        st.local_steps(w.H if w.H > 0 else 0, Hi)
+        st.gossip_round()
+        return st.consensus_error()
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    value = w.n_workers * slice_p * args.steps / el
+    sample = ("each step: one round of the workload on parameter indices [0, %d) with all %d "
+              "workers (fp32 oracle, OpenMP over elements)" % (slice_p, w.n_workers))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": workload_config(w, args),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": orc.lib.oc_num_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(w, args):
+    state_gb = w.n_workers * w.n_params * 4 * (6 + (1 if w.hp.get("per_worker_h") else 0)) / 1e9
+    return {"workload": w.name, "n_workers": w.n_workers, "n_params": w.n_params,
+            "topology": w.topology, "H": w.H if w.H > 0 else "H_i~U{1..%d}" % w.draw_hmax,
+            "layout": "tensor-list(%d)" % len(w.numels) if w.numels else "flat",
+            "weights": w.hp.get("weights", "uniform"), "outer": "nesterov(0.7, 0.9)",
+            "seed": w.seed, "parallelism": "replicas x%d" % args.gpus,
+            "l2": "inputs larger than L2 (%.1f GB replica state per GPU, no flush)" % state_gb}
+
+
+def main():
+    args = parse_args()
+    from paper_2606_11081_gb300 import workloads as wl
+    w = wl.WORKLOADS[args.workload or wl.BENCH_WORKLOAD]
+    if args.impl == "reference":
+        return run_reference(args, w)
+
+    import numpy as np
+    import torch
+    import paper_2606_11081_gb300 as g
+    from paper_2606_11081_gb300 import build as gbuild
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        pg = dist
+    if rank == 0 or world == 1:
+        gbuild.build()
+    if pg:
+        pg.barrier()
+
+    hp = g.make_hparams(**wl.hparams_of(w))
+    ctx = g.Context(w.n_workers, w.n_params, w.topology, w.seed, hparams=hp, numels=w.numels,
+                    draw_hmax=w.draw_hmax)
+    H = w.H if w.H > 0 else g.PER_WORKER_STEPS
+    Hi = g.gasloc_get_local_steps(ctx.h, w.n_workers).tolist() if w.H < 0 else None
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        ctx.local_steps(H)
+        ctx.gossip_round()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    clocks = ClockSampler(local)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    l0 = ctx.launches
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(K):
+        ev[k][0].record(stream)
+        ctx.local_steps(H)
+        ev[k][1].record(stream)
+        ctx.gossip_round()
+        ev[k][2].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    launches = ctx.launches - l0
+    ms = t_start.elapsed_time(t_end)
+    local_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(K))
+    gossip_ms = sum(ev[k][1].elapsed_time(ev[k][2]) for k in range(K))
+    if pg:
+        t = torch.tensor([ms], device="cuda")
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms = float(t.item())
+        pg.barrier()
+    ce = ctx.consensus_error()
+
+    # algorithmic bytes
+    N, P = w.n_workers, w.n_params
+    per_h = bool(w.hp.get("per_worker_h"))
+    steps = [H] * N if H > 0 else Hi
+    adamw_launches = max(steps)
+    adamw_bytes = 0
+    for s in range(max(steps)):
+        act = sum(1 for h in steps if h > s)
+        adamw_bytes += (32 * act if per_h else 28 * act + 4) * P
+    gossip_bytes = 20 * N * P
+    peak, peak_kind = peak_hbm()
+    adamw_gbs = adamw_bytes / (local_ms / K / 1e3) / 1e9
+    gossip_gbs = gossip_bytes / (gossip_ms / K / 1e3) / 1e9
+    dom = "adamw" if local_ms >= gossip_ms else "gossip"
+    dom_gbs = adamw_gbs if dom == "adamw" else gossip_gbs
+    dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
+    traffic = kernel_traffic(dom, w.name)
+    value = N * P * K / (ms / 1e3) * world
+
+    e2e = None
+    if not args.no_e2e:
+        ctx.close()
+        torch.cuda.empty_cache()
+        e2e = measure_e2e(g, torch, w, hp, H, K)
+    else:
+        ctx.close()
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+            "warmup": args.warmup, "ms_per_step": ms / K, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": workload_config(w, args),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": dom_gbs, "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": dom_gbs / peak,
+                         "traffic": traffic, "algorithmic_bytes_per_launch": dom_bytes_launch},
+            "kernels": {"adamw": {"gbs": adamw_gbs, "frac": adamw_gbs / peak, "ms_per_round": local_ms / K,
+                                  "bytes_per_round": adamw_bytes, "launches_per_round": adamw_launches},
+                        "gossip": {"gbs": gossip_gbs, "frac": gossip_gbs / peak,
+                                   "ms_per_round": gossip_ms / K, "bytes_per_round": gossip_bytes}},
+            "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clk,
+            "consensus_error": ce,
+        }
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+    return 0
+
+
+def measure_e2e(g, torch, w, hp, H, K):
+    """Same rounds through the public C ABI from host buffers: upload the
+    initial replicas (x_0 broadcast), centres and curvature from pinned memory,
+    read the consensus error back every round, read the average back at the end."""
+    import numpy as np
+    N, P = w.n_workers, w.n_params
+    ctx = g.Context(N, P, w.topology, w.seed, hparams=hp, numels=w.numels, draw_hmax=w.draw_hmax)
+    per_h = bool(w.hp.get("per_worker_h"))
+    nh = N if per_h else 1
+    # host inputs (taken from the device initialisation, untimed)
+    x0 = torch.empty(P, dtype=torch.float32, pin_memory=True)
+    cs = torch.empty((N, P), dtype=torch.float32, pin_memory=True)
+    hs = torch.empty((nh, P), dtype=torch.float32, pin_memory=True)
+    g.gasloc_read(ctx.h, "x", 0, x0.numpy())
+    for i in range(N):
+        g.gasloc_read(ctx.h, "c", i, cs[i].numpy())
+    for i in range(nh):
+        g.gasloc_read(ctx.h, "h", i, hs[i].numpy())
+    out = torch.empty(P, dtype=torch.float32, pin_memory=True)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    g.gasloc_write_ptr(ctx.h, "x", -1, x0.data_ptr())
+    for i in range(N):
+        g.gasloc_write_ptr(ctx.h, "c", i, cs[i].data_ptr())
+    for i in range(nh):
+        g.gasloc_write_ptr(ctx.h, "h", i, hs[i].data_ptr())
+    ces = []
+    for _ in range(K):
+        ctx.local_steps(H)
+        ctx.gossip_round()
+        ces.append(ctx.consensus_error())
+    g.gasloc_average_host(ctx.h, out.numpy())
+    el = time.perf_counter() - t0
+    ctx.close()
+    h2d = (P + N * P + nh * P) * 4
+    d2h = 8 * K + 4 * P
+    return {"value": N * P * K / el, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
+            "d2h_bytes_per_step": d2h / K, "seconds": el,
+            "note": "initial replicas, centres and curvature uploaded once per run (amortised); "
+                    "consensus error read every round; average read at the end"}
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,227 @@
+/*
+ * gasloc.h -- C ABI of libgasloc, the GB300 (sm_103a) replica-update path of
+ * GASLoC ("Unifying Local Communications and Local Updates for LLM
+ * Pretraining", arXiv 2606.11081).
+ *
+ * The library simulates n workers whose fp32 replicas live together in one
+ * GPU's memory as a structure of arrays and runs, per outer round t, the steps
+ * of Algorithm 1:
+ *   1. H_i inner AdamW steps per worker, x_i -> y_i (App. B optimisation
+ *      settings), on the synthetic diagonal quadratic
+ *      f_i(x) = 1/2 sum_k h_k (x_k - c_ik)^2 with gradient noise;
+ *   2. one gossip round: each worker mixes the y_j of its round-t neighbourhood
+ *      N_i (always containing i) with row-stochastic weights w_ij and applies
+ *      the outer optimizer (Nesterov by default, App. B; SGDM, SGD; the
+ *      accelerated-gossip update of Eq. 2; DAdam and Local-DAdam of App. C);
+ *   3. the consensus error (1/n) sum_i ||x_i - xbar||^2 of the new replicas.
+ *
+ * Conventions (all entry points):
+ *  - Every call returns a gasloc_status; on failure gasloc_last_error()
+ *    returns a message (thread-local, valid until the next call on the thread).
+ *  - Device memory is owned by the context.  It is obtained from the allocator
+ *    registered with gasloc_set_allocator() (e.g. a framework's caching
+ *    allocator) or, if none is registered, from cudaMalloc, and released by
+ *    gasloc_destroy().
+ *  - Work is enqueued asynchronously on the context's stream (default: the
+ *    CUDA legacy default stream; see gasloc_set_stream).  Calls documented as
+ *    "synchronising" wait for that stream before returning.
+ *  - Floating-point parameters are fp32 on the device; host-side scalars of a
+ *    step (bias corrections etc.) are computed in double and rounded once.
+ *  - A context is not thread-safe.  Distinct contexts are independent.
+ */
+#ifndef GASLOC_H
+#define GASLOC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gasloc_ctx gasloc_ctx;
+
+typedef enum {
+    GASLOC_OK = 0,
+    GASLOC_EINVAL = -1,   /* an argument is out of range or inconsistent   */
+    GASLOC_ENOMEM = -2,   /* an allocation failed or a size limit was hit  */
+    GASLOC_ECUDA = -3,    /* a CUDA runtime call or a launch failed        */
+    GASLOC_ESTATE = -4,   /* call not valid in the context's current state */
+    GASLOC_EDEVICE = -5,  /* a kernel set the device error flag            */
+    GASLOC_EIO = -6       /* checkpoint file could not be read or written  */
+} gasloc_status;
+
+/* Outer update applied after mixing (Algorithm 1 "Optimizer^out"; Eq. 2; App. C). */
+enum {
+    GASLOC_OUTER_SGD = 0,          /* x -= eta_out * D                       */
+    GASLOC_OUTER_SGDM = 1,         /* b = mu b + D; x -= eta_out * b          */
+    GASLOC_OUTER_NESTEROV = 2,     /* b = mu b + D; x -= eta_out (D + mu b)   */
+    GASLOC_OUTER_EQ2 = 3,          /* Eq. 2 on z = x + eta (y - x)            */
+    GASLOC_OUTER_DADAM = 4,        /* x = sum_j w_ij x_j + (y - x)            */
+    GASLOC_OUTER_LOCAL_DADAM = 5   /* Nesterov step of D = x - sum w x_j at y */
+};
+
+/* Mixing-weight rule applied to the round's graph. */
+enum {
+    GASLOC_W_UNIFORM = 0,          /* w_ij = 1/|N_i|  (Algorithm 1)           */
+    GASLOC_W_METROPOLIS = 1,       /* w_ij = 1/(1+max(d_i,d_j)), w_ii = rest  */
+    GASLOC_W_LAZY = 2              /* w_ii = 1/2, w_ij = 1/(2 d_i): W = I -
+                                      Lambda^(k) of the k-Peer schemes        */
+};
+
+/* Buffers of the replica store (gasloc_buffer / gasloc_read / gasloc_write). */
+enum {
+    GASLOC_BUF_X = 0,   /* outer (anchor) parameters x_i                      */
+    GASLOC_BUF_Y = 1,   /* inner iterate y_i                                  */
+    GASLOC_BUF_M = 2,   /* AdamW first moment                                 */
+    GASLOC_BUF_V = 3,   /* AdamW second moment                                */
+    GASLOC_BUF_B = 4,   /* outer momentum (z_{t-1} in Eq. 2 mode)             */
+    GASLOC_BUF_C = 5,   /* quadratic centre c_i                               */
+    GASLOC_BUF_H = 6    /* curvature h (per worker if per_worker_h)           */
+};
+
+#define GASLOC_MAX_WORKERS 32
+#define GASLOC_PER_WORKER_STEPS (-1)
+
+typedef struct gasloc_hparams {
+    /* inner AdamW (App. B): lr, (beta1, beta2), eps, weight decay */
+    double lr, beta1, beta2, eps, weight_decay;
+    /* sigma of the gradient noise sigma * xi, xi uniform with unit variance */
+    double noise_sigma;
+    /* outer optimizer: eta_out and mu (Nesterov/SGDM/Local-DAdam) */
+    double outer_lr, outer_momentum;
+    /* Eq. 1/2: eta (outer step on g = y - x), alpha (mixing), gamma (momentum) */
+    double eta, alpha, gamma;
+    /* probability that an edge of the base graph is active in a round */
+    double edge_prob;
+    int32_t outer_mode;     /* GASLOC_OUTER_* */
+    int32_t weights;        /* GASLOC_W_*     */
+    int32_t per_worker_h;   /* 1: one curvature vector per worker */
+    int32_t reserved;
+} gasloc_hparams;
+
+/* Device allocator hooks: alloc returns a device pointer (NULL on failure) of
+ * at least `bytes` bytes, 256-byte aligned, usable on `stream`. */
+typedef void *(*gasloc_alloc_fn)(size_t bytes, void *stream, void *user);
+typedef void (*gasloc_free_fn)(void *ptr, void *stream, void *user);
+
+/* Fills *hp with the defaults: AdamW lr 3e-4, betas (0.9, 0.95), eps 1e-8,
+ * weight decay 0.1 (App. B); sigma 0.01; Nesterov with eta_out 0.7, mu 0.9;
+ * eta = alpha = 1, gamma = 0; edge_prob 1; uniform weights; shared h. */
+void gasloc_default_hparams(gasloc_hparams *hp);
+
+/* Creates a context for n_workers (1..32) replicas of n_params (>= 1) fp32
+ * parameters each, communicating over `topology`:
+ *   "none", "ring", "complete", "exp" (peers at +-2^q), "torus:RxC" (R*C = n),
+ *   "matching" (randomized 1-Peer, Sec. 3.2), "2peer" (randomized 2-Peer).
+ * `seed` keys every random draw (initial point, centres, curvature, noise,
+ * permutations, edge activation, H_i).  Nothing is allocated on the device
+ * until gasloc_start().  Errors: EINVAL (n_workers, n_params, topology),
+ * ENOMEM. */
+int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint64_t seed,
+                gasloc_ctx **out);
+
+/* Sets the hyperparameters (copied).  Before gasloc_start any field may
+ * change; afterwards per_worker_h may not (ESTATE).  EINVAL if lr < 0,
+ * beta not in [0,1), eps <= 0, edge_prob not in [0,1], an unknown mode or
+ * weight rule, or eta/alpha/gamma/outer_lr negative. */
+int gasloc_set_hparams(gasloc_ctx *ctx, const gasloc_hparams *hp);
+int gasloc_get_hparams(const gasloc_ctx *ctx, gasloc_hparams *hp);
+
+/* Declares that the n_params of each replica form a list of n_tensors
+ * parameter tensors with the given element counts (sum = n_params), stored as
+ * separate device allocations of shape [n_workers, numel].  Without this call
+ * the replica is one flat tensor.  Element k of the concatenation is the
+ * parameter index used by every generator.  Before gasloc_start only. */
+int gasloc_set_layout(gasloc_ctx *ctx, int32_t n_tensors, const int64_t *numels);
+
+/* Registers device allocator hooks (before gasloc_start only). */
+int gasloc_set_allocator(gasloc_ctx *ctx, gasloc_alloc_fn alloc, gasloc_free_fn free_fn,
+                         void *user);
+
+/* Sets the cudaStream_t all later work is enqueued on. */
+int gasloc_set_stream(gasloc_ctx *ctx, void *cuda_stream);
+
+/* Allocates the replica store and initialises it on the device: identical
+ * x_i = x_0 ~ N(0, 0.02^2) on every worker (Prop. 2 assumes equal initial
+ * replicas), y_i = x_i, centres c_i ~ N(0,1), curvature h ~ U(0.1, 1), and
+ * m = v = b = 0.  Asynchronous.  ENOMEM if an allocation fails. */
+int gasloc_start(gasloc_ctx *ctx);
+
+/* Per-worker local step counts H_i (Sec. 3.2, heterogeneous local steps),
+ * each in [0, 1024]; host array of n_workers entries, copied. */
+int gasloc_set_local_steps(gasloc_ctx *ctx, const int32_t *H_i);
+/* Draws H_i = 1 + floor(u_i * hmax) from the seed (u_i uniform), hmax >= 1. */
+int gasloc_draw_local_steps(gasloc_ctx *ctx, int32_t hmax);
+int gasloc_get_local_steps(const gasloc_ctx *ctx, int32_t *H_i);
+
+/* Inner loop of Algorithm 1: H > 0 gives every worker H AdamW steps;
+ * H = GASLOC_PER_WORKER_STEPS gives worker i its H_i steps.  The first step
+ * of a round starts from x_i; later ones from y_i.  Moments and step counters
+ * persist across rounds.  Asynchronous.  ESTATE before gasloc_start. */
+int gasloc_local_steps(gasloc_ctx *ctx, int32_t H);
+
+/* Outer step of Algorithm 1 for round t: builds the round-t neighbour table
+ * on the device, mixes each worker's sent quantity over N_i in ascending j,
+ * applies the outer update and reduces the consensus error of the new x.
+ * A worker that took no local step this round sends x_i.  Asynchronous. */
+int gasloc_gossip_round(gasloc_ctx *ctx);
+
+/* Consensus error CE = (1/n) sum_i sum_k (x_ik - xbar_k)^2 of the current
+ * replicas (||pi x||^2 / n with pi = I - 11^T/n).  Returns the value the last
+ * gossip round reduced when nothing changed x since, else reduces it now.
+ * Synchronising; EDEVICE if a kernel reported an error since the last check. */
+int gasloc_consensus_error(gasloc_ctx *ctx, double *out);
+/* Same quantity, always reduced now from the current x by the standalone
+ * reduction kernel (ignores the value the last gossip round produced). */
+int gasloc_consensus_error_now(gasloc_ctx *ctx, double *out);
+
+/* Neighbour table of round `round` as the device generates it: host arrays
+ * nbr[n*n] (row i: N_i ascending, deg[i]+1 valid entries), w[n*n] (fp32) and
+ * deg[n] (graph degree, self excluded).  Synchronising. */
+int gasloc_get_topology(gasloc_ctx *ctx, int64_t round, int32_t *nbr, float *w, int32_t *deg);
+
+/* Output of Algorithm 1: xbar = (1/n) sum_i x_i into dst (n_params fp32,
+ * device memory; concatenation order).  Asynchronous. */
+int gasloc_average(gasloc_ctx *ctx, float *dst_device);
+/* Same into host memory (pinned or pageable).  Synchronising. */
+int gasloc_average_host(gasloc_ctx *ctx, float *dst_host);
+
+/* Device pointer of buffer `which` for tensor `tensor`: worker i's slice
+ * starts at *dptr + i * (*worker_stride) floats (worker_stride may be NULL;
+ * for GASLOC_BUF_H with a shared curvature it is 0).  Valid until destroy. */
+int gasloc_buffer(gasloc_ctx *ctx, int32_t which, int32_t tensor, void **dptr,
+                  int64_t *worker_stride);
+
+/* Copies buffer `which` of `worker` (flat, n_params floats) to or from host
+ * memory.  In gasloc_write, worker = -1 writes every worker (x_0 broadcast).
+ * Synchronising. */
+int gasloc_read(gasloc_ctx *ctx, int32_t which, int32_t worker, float *host_dst);
+int gasloc_write(gasloc_ctx *ctx, int32_t which, int32_t worker, const float *host_src);
+
+/* Gathers n elements (global indices idx[], host array) of buffer `which` of
+ * `worker` into host out[].  Synchronising. */
+int gasloc_gather(gasloc_ctx *ctx, int32_t which, int32_t worker, int64_t n,
+                  const int64_t *idx, float *out);
+
+/* Completed gossip rounds and local steps taken by a worker. */
+int gasloc_round(const gasloc_ctx *ctx, int64_t *round);
+int gasloc_steps_taken(const gasloc_ctx *ctx, int32_t worker, int64_t *steps);
+
+/* Checkpoint: every buffer plus counters.  gasloc_load needs a started
+ * context of the same shape, topology and seed.  Synchronising; EIO. */
+int gasloc_save(gasloc_ctx *ctx, const char *path);
+int gasloc_load(gasloc_ctx *ctx, const char *path);
+
+/* Launch counter of the library's kernels on this context (for accounting). */
+int gasloc_launch_count(const gasloc_ctx *ctx, int64_t *count);
+
+const char *gasloc_last_error(void);
+
+/* Releases the context and all its device memory (waits for its stream). */
+void gasloc_destroy(gasloc_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GASLOC_H */

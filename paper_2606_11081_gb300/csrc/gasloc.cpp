@@ -1,0 +1,919 @@
+// gasloc.cpp -- the C ABI of include/gasloc.h: argument checking, the
+// structure-of-arrays replica store, per-step host scalars and kernel launches.
+//
+// Host arithmetic that the device results depend on (bias corrections, decay,
+// the fp32 rounding of hyperparameters) is done in double and rounded once;
+// this file is compiled with -ffp-contract=off so that no a*b+c is fused.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/gasloc.h"
+#include "internal.h"
+
+using namespace gasloc;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+    return fail(GASLOC_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr int64_t kMaxParams = (int64_t(1) << 31) - 1;
+constexpr int64_t kPadFloats = 64;
+constexpr int kTileA = 1024;          // init / adamw / ce / average tiles (4 x 256 threads)
+constexpr int kMaxLocalSteps = 1024;
+
+int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+}  // namespace
+
+struct gasloc_ctx {
+    int32_t n = 0;
+    int64_t P = 0;
+    TopoSpec spec{};
+    uint64_t seed = 0;
+    gasloc_hparams hp{};
+    std::vector<int64_t> numels;
+    gasloc_alloc_fn alloc = nullptr;
+    gasloc_free_fn free_fn = nullptr;
+    void *alloc_user = nullptr;
+    cudaStream_t stream = nullptr;
+    bool started = false;
+    int sms = 0;
+
+    // device store
+    std::vector<TensorDesc> tens_h;
+    std::vector<int64_t> goff;
+    TensorDesc *tens_d = nullptr;
+    Tile *tiles_a = nullptr;
+    int64_t ntiles_a = 0;
+    Tile *tiles_g = nullptr;
+    int64_t ntiles_g = 0;
+    int tile_g = 0, block_g = 0, stages_g = 0;
+    size_t smem_g = 0;
+    int grid_a = 0, grid_g = 0, grid_ce = 0;
+    Topo *topo_d = nullptr, *topo_scratch = nullptr;
+    double *partials = nullptr;
+    unsigned int *ticket = nullptr;
+    double *ce_d = nullptr;
+    int32_t *err_d = nullptr;
+    void *pinned = nullptr;   // [ce double][err int32][Topo]
+    std::vector<std::pair<void *, size_t>> allocs;
+
+    // counters
+    std::vector<int64_t> nsteps;
+    std::vector<double> p1, p2;
+    std::vector<int32_t> Hi;
+    bool has_Hi = false;
+    uint32_t fresh_mask = 0;
+    int64_t round = 0;
+    bool ce_valid = false;
+    bool topo_static = false, topo_ready = false;
+    int64_t launches = 0;
+
+    void *dalloc(size_t bytes) {
+        bytes = static_cast<size_t>(round_up(static_cast<int64_t>(bytes ? bytes : 1), 256));
+        void *p = nullptr;
+        if (alloc) {
+            p = alloc(bytes, stream, alloc_user);
+        } else if (cudaMalloc(&p, bytes) != cudaSuccess) {
+            cudaGetLastError();
+            p = nullptr;
+        }
+        if (p) allocs.emplace_back(p, bytes);
+        return p;
+    }
+    void dfree(void *p) {
+        if (!p) return;
+        for (size_t q = 0; q < allocs.size(); ++q)
+            if (allocs[q].first == p) {
+                allocs.erase(allocs.begin() + static_cast<long>(q));
+                break;
+            }
+        if (free_fn) free_fn(p, stream, alloc_user);
+        else cudaFree(p);
+    }
+    void release_all() {
+        if (started || !allocs.empty()) cudaStreamSynchronize(stream);
+        for (auto &pr : allocs) {
+            if (free_fn) free_fn(pr.first, stream, alloc_user);
+            else cudaFree(pr.first);
+        }
+        allocs.clear();
+        if (pinned) cudaFreeHost(pinned);
+        pinned = nullptr;
+    }
+};
+
+namespace {
+
+double *pin_ce(gasloc_ctx *c) { return reinterpret_cast<double *>(c->pinned); }
+int32_t *pin_err(gasloc_ctx *c) { return reinterpret_cast<int32_t *>(static_cast<char *>(c->pinned) + 8); }
+Topo *pin_topo(gasloc_ctx *c) { return reinterpret_cast<Topo *>(static_cast<char *>(c->pinned) + 64); }
+
+int parse_topology(const char *s, int32_t n, TopoSpec *spec) {
+    if (!s) return fail(GASLOC_EINVAL, "topology is NULL");
+    std::string t(s);
+    spec->rows = spec->cols = 0;
+    if (t == "none") spec->kind = kNone;
+    else if (t == "ring") spec->kind = kRing;
+    else if (t == "complete") spec->kind = kComplete;
+    else if (t == "exp") spec->kind = kExp;
+    else if (t == "matching") spec->kind = kMatching;
+    else if (t == "2peer") spec->kind = kTwoPeer;
+    else if (t.rfind("torus:", 0) == 0) {
+        int r = 0, c = 0;
+        char tail = 0;
+        if (std::sscanf(t.c_str() + 6, "%dx%d%c", &r, &c, &tail) != 2 || r < 1 || c < 1)
+            return fail(GASLOC_EINVAL, "bad torus spec '%s' (want torus:RxC)", s);
+        if (static_cast<int64_t>(r) * c != n)
+            return fail(GASLOC_EINVAL, "torus %dx%d does not have %d nodes", r, c, n);
+        spec->kind = kTorus;
+        spec->rows = r;
+        spec->cols = c;
+    } else {
+        return fail(GASLOC_EINVAL, "unknown topology '%s'", s);
+    }
+    if ((spec->kind == kMatching || spec->kind == kTwoPeer) && n < 2)
+        return fail(GASLOC_EINVAL, "randomized peer schemes need at least 2 workers");
+    return GASLOC_OK;
+}
+
+int check_hparams(const gasloc_hparams *hp) {
+    if (!(hp->lr >= 0.0) || !std::isfinite(hp->lr)) return fail(GASLOC_EINVAL, "lr must be >= 0");
+    if (!(hp->beta1 >= 0.0 && hp->beta1 < 1.0) || !(hp->beta2 >= 0.0 && hp->beta2 < 1.0))
+        return fail(GASLOC_EINVAL, "betas must be in [0, 1)");
+    if (!(hp->eps > 0.0) || !std::isfinite(hp->eps)) return fail(GASLOC_EINVAL, "eps must be > 0");
+    if (!(hp->weight_decay >= 0.0) || !std::isfinite(hp->weight_decay))
+        return fail(GASLOC_EINVAL, "weight decay must be >= 0");
+    if (!(hp->noise_sigma >= 0.0) || !std::isfinite(hp->noise_sigma))
+        return fail(GASLOC_EINVAL, "noise sigma must be >= 0");
+    if (!(hp->edge_prob >= 0.0 && hp->edge_prob <= 1.0)) return fail(GASLOC_EINVAL, "edge_prob must be in [0, 1]");
+    if (!(hp->outer_lr >= 0.0) || !(hp->outer_momentum >= 0.0) || !(hp->eta >= 0.0) || !(hp->alpha >= 0.0) ||
+        !(hp->gamma >= 0.0) || !std::isfinite(hp->outer_lr) || !std::isfinite(hp->outer_momentum) ||
+        !std::isfinite(hp->eta) || !std::isfinite(hp->alpha) || !std::isfinite(hp->gamma))
+        return fail(GASLOC_EINVAL, "outer hyperparameters must be finite and >= 0");
+    if (hp->outer_mode < GASLOC_OUTER_SGD || hp->outer_mode > GASLOC_OUTER_LOCAL_DADAM)
+        return fail(GASLOC_EINVAL, "unknown outer mode %d", hp->outer_mode);
+    if (hp->weights < GASLOC_W_UNIFORM || hp->weights > GASLOC_W_LAZY)
+        return fail(GASLOC_EINVAL, "unknown weight rule %d", hp->weights);
+    if (hp->per_worker_h != 0 && hp->per_worker_h != 1) return fail(GASLOC_EINVAL, "per_worker_h must be 0 or 1");
+    return GASLOC_OK;
+}
+
+void refresh_spec(gasloc_ctx *c) {
+    c->spec.n = c->n;
+    c->spec.seed = c->seed;
+    c->spec.weights = c->hp.weights;
+    const double thr = std::floor(c->hp.edge_prob * 4294967296.0);
+    c->spec.edge_thr = static_cast<uint64_t>(thr);
+    c->topo_static = (c->spec.kind != kMatching && c->spec.kind != kTwoPeer && c->spec.edge_thr >= (1ull << 32));
+    c->topo_ready = false;
+}
+
+int check_started(const gasloc_ctx *c) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (!c->started) return fail(GASLOC_ESTATE, "context not started (call gasloc_start)");
+    return GASLOC_OK;
+}
+
+int sync_and_check(gasloc_ctx *c) {
+    cudaError_t e = cudaMemcpyAsync(pin_err(c), c->err_d, sizeof(int32_t), cudaMemcpyDeviceToHost, c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device error flag");
+    e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    const int32_t err = *pin_err(c);
+    if (err != kDevOk) {
+        cudaMemsetAsync(c->err_d, 0, sizeof(int32_t), c->stream);
+        cudaStreamSynchronize(c->stream);
+        return fail(GASLOC_EDEVICE, "a kernel reported device error %d (%s)", err,
+                    err == kDevWaitTimeout ? "bounded wait timed out" : "index out of range");
+    }
+    return GASLOC_OK;
+}
+
+int launch_checked(gasloc_ctx *c, cudaError_t e, const char *what) {
+    if (e != cudaSuccess) return cuda_fail(e, what);
+    ++c->launches;
+    return GASLOC_OK;
+}
+
+int build_topology(gasloc_ctx *c, int64_t round, Topo *dst) {
+    return launch_checked(c, launch_topo(c->spec, round, dst, c->stream), "topology kernel");
+}
+
+float *buffer_base(const TensorDesc &d, int which, int64_t *stride) {
+    *stride = d.wstride;
+    switch (which) {
+    case GASLOC_BUF_X: return d.x;
+    case GASLOC_BUF_Y: return d.y;
+    case GASLOC_BUF_M: return d.m;
+    case GASLOC_BUF_V: return d.v;
+    case GASLOC_BUF_B: return d.b;
+    case GASLOC_BUF_C: return d.c;
+    case GASLOC_BUF_H: *stride = d.hstride; return d.h;
+    default: return nullptr;
+    }
+}
+
+int check_which_worker(const gasloc_ctx *c, int32_t which, int32_t worker, bool allow_all) {
+    if (which < GASLOC_BUF_X || which > GASLOC_BUF_H) return fail(GASLOC_EINVAL, "unknown buffer %d", which);
+    const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
+    if (worker == -1 && allow_all) return GASLOC_OK;
+    if (worker < 0 || worker >= rows) return fail(GASLOC_EINVAL, "worker %d out of range", worker);
+    return GASLOC_OK;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ API ----
+
+extern "C" {
+
+void gasloc_default_hparams(gasloc_hparams *hp) {
+    if (!hp) return;
+    std::memset(hp, 0, sizeof *hp);
+    hp->lr = 3e-4;
+    hp->beta1 = 0.9;
+    hp->beta2 = 0.95;
+    hp->eps = 1e-8;
+    hp->weight_decay = 0.1;
+    hp->noise_sigma = 0.01;
+    hp->outer_lr = 0.7;
+    hp->outer_momentum = 0.9;
+    hp->eta = 1.0;
+    hp->alpha = 1.0;
+    hp->gamma = 0.0;
+    hp->edge_prob = 1.0;
+    hp->outer_mode = GASLOC_OUTER_NESTEROV;
+    hp->weights = GASLOC_W_UNIFORM;
+    hp->per_worker_h = 0;
+}
+
+const char *gasloc_last_error(void) { return g_err.c_str(); }
+
+int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint64_t seed, gasloc_ctx **out) {
+    if (!out) return fail(GASLOC_EINVAL, "out is NULL");
+    *out = nullptr;
+    if (n_workers < 1 || n_workers > GASLOC_MAX_WORKERS)
+        return fail(GASLOC_EINVAL, "n_workers must be in [1, %d], got %d", GASLOC_MAX_WORKERS, n_workers);
+    if (n_params < 1 || n_params > kMaxParams)
+        return fail(GASLOC_EINVAL, "n_params must be in [1, 2^31-1], got %lld", static_cast<long long>(n_params));
+    TopoSpec spec{};
+    int rc = parse_topology(topology, n_workers, &spec);
+    if (rc) return rc;
+    gasloc_ctx *c = new (std::nothrow) gasloc_ctx();
+    if (!c) return fail(GASLOC_ENOMEM, "out of host memory");
+    c->n = n_workers;
+    c->P = n_params;
+    c->spec = spec;
+    c->seed = seed;
+    gasloc_default_hparams(&c->hp);
+    c->numels.assign(1, n_params);
+    c->nsteps.assign(n_workers, 0);
+    c->p1.assign(n_workers, 1.0);
+    c->p2.assign(n_workers, 1.0);
+    c->Hi.assign(n_workers, 0);
+    refresh_spec(c);
+    *out = c;
+    return GASLOC_OK;
+}
+
+int gasloc_set_hparams(gasloc_ctx *c, const gasloc_hparams *hp) {
+    if (!c || !hp) return fail(GASLOC_EINVAL, "NULL argument");
+    int rc = check_hparams(hp);
+    if (rc) return rc;
+    if (c->started && hp->per_worker_h != c->hp.per_worker_h)
+        return fail(GASLOC_ESTATE, "per_worker_h cannot change after gasloc_start");
+    c->hp = *hp;
+    refresh_spec(c);
+    return GASLOC_OK;
+}
+
+int gasloc_get_hparams(const gasloc_ctx *c, gasloc_hparams *hp) {
+    if (!c || !hp) return fail(GASLOC_EINVAL, "NULL argument");
+    *hp = c->hp;
+    return GASLOC_OK;
+}
+
+int gasloc_set_layout(gasloc_ctx *c, int32_t n_tensors, const int64_t *numels) {
+    if (!c || !numels) return fail(GASLOC_EINVAL, "NULL argument");
+    if (c->started) return fail(GASLOC_ESTATE, "layout cannot change after gasloc_start");
+    if (n_tensors < 1 || n_tensors > (1 << 20)) return fail(GASLOC_EINVAL, "n_tensors out of range");
+    int64_t tot = 0;
+    for (int32_t t = 0; t < n_tensors; ++t) {
+        if (numels[t] < 1) return fail(GASLOC_EINVAL, "tensor %d has %lld elements", t, (long long)numels[t]);
+        tot += numels[t];
+    }
+    if (tot != c->P) return fail(GASLOC_EINVAL, "tensor sizes sum to %lld, not n_params %lld", (long long)tot,
+                                 (long long)c->P);
+    c->numels.assign(numels, numels + n_tensors);
+    return GASLOC_OK;
+}
+
+int gasloc_set_allocator(gasloc_ctx *c, gasloc_alloc_fn a, gasloc_free_fn f, void *user) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (c->started) return fail(GASLOC_ESTATE, "allocator cannot change after gasloc_start");
+    if ((a == nullptr) != (f == nullptr)) return fail(GASLOC_EINVAL, "give both alloc and free, or neither");
+    c->alloc = a;
+    c->free_fn = f;
+    c->alloc_user = user;
+    return GASLOC_OK;
+}
+
+int gasloc_set_stream(gasloc_ctx *c, void *s) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    c->stream = static_cast<cudaStream_t>(s);
+    return GASLOC_OK;
+}
+
+int gasloc_start(gasloc_ctx *c) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (c->started) return fail(GASLOC_ESTATE, "context already started");
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "multiprocessor count");
+
+    const int32_t n = c->n;
+    const int32_t nh = c->hp.per_worker_h ? n : 1;
+    // size check before any allocation
+    int64_t need = 0;
+    for (int64_t ne : c->numels) {
+        const int64_t ws = round_up(ne, kPadFloats);
+        need += (6LL * n + nh) * ws * 4;
+    }
+    size_t fr = 0, tot = 0;
+    if (cudaMemGetInfo(&fr, &tot) == cudaSuccess && static_cast<size_t>(need) > fr)
+        return fail(GASLOC_ENOMEM, "replica store needs %lld bytes, %zu free", (long long)need, fr);
+
+    // gossip launch shape: 16-byte column per thread; stage ~32 KB of sent rows
+    int block = 2048 / n;
+    block = std::max(64, std::min(256, block));
+    int pw = 64;
+    while (pw * 2 <= block) pw *= 2;
+    c->block_g = pw;
+    c->tile_g = 4 * c->block_g;
+    const int rows = c->hp.outer_mode == GASLOC_OUTER_EQ2 ? 2 * n : n;
+    const size_t stage_bytes = static_cast<size_t>(rows) * c->tile_g * 4;
+    int stages = static_cast<int>((110 * 1024 - 8704) / stage_bytes);
+    c->stages_g = std::max(2, std::min(4, stages));
+    // the EQ2 layout bounds the smem attribute for every mode
+    c->smem_g = gasloc::gossip_smem_bytes(n, c->tile_g, c->stages_g, c->hp.outer_mode);
+    const size_t smem_max = gasloc::gossip_smem_bytes(n, c->tile_g, c->stages_g, GASLOC_OUTER_EQ2);
+    e = gossip_set_smem(smem_max);
+    if (e != cudaSuccess) return cuda_fail(e, "gossip shared-memory attribute");
+
+    auto oom = [&](const char *what) {
+        c->release_all();
+        c->tens_h.clear();
+        return fail(GASLOC_ENOMEM, "device allocation failed (%s)", what);
+    };
+
+    // replica store
+    c->tens_h.clear();
+    c->goff.clear();
+    int64_t g = 0;
+    for (size_t t = 0; t < c->numels.size(); ++t) {
+        TensorDesc d{};
+        d.numel = c->numels[t];
+        d.wstride = round_up(d.numel, kPadFloats);
+        d.hstride = c->hp.per_worker_h ? d.wstride : 0;
+        d.goff = g;
+        g += d.numel;
+        float **arrs[6] = {&d.x, &d.y, &d.m, &d.v, &d.b, &d.c};
+        for (float **a : arrs) {
+            *a = static_cast<float *>(c->dalloc(static_cast<size_t>(n) * d.wstride * 4));
+            if (!*a) return oom("replica arrays");
+        }
+        d.h = static_cast<float *>(c->dalloc(static_cast<size_t>(nh) * d.wstride * 4));
+        if (!d.h) return oom("curvature");
+        c->tens_h.push_back(d);
+        c->goff.push_back(d.goff);
+    }
+    for (auto &pr : c->allocs) {
+        e = cudaMemsetAsync(pr.first, 0, pr.second, c->stream);
+        if (e != cudaSuccess) { c->release_all(); return cuda_fail(e, "zero fill"); }
+    }
+
+    // tile tables
+    auto make_tiles = [&](int tile, std::vector<Tile> &v) {
+        v.clear();
+        for (size_t t = 0; t < c->numels.size(); ++t)
+            for (int64_t s = 0; s < c->numels[t]; s += tile)
+                v.push_back(Tile{static_cast<int32_t>(t), static_cast<int32_t>(std::min<int64_t>(tile, c->numels[t] - s)), s});
+    };
+    std::vector<Tile> ta, tg;
+    make_tiles(kTileA, ta);
+    make_tiles(c->tile_g, tg);
+    c->ntiles_a = static_cast<int64_t>(ta.size());
+    c->ntiles_g = static_cast<int64_t>(tg.size());
+
+    c->tens_d = static_cast<TensorDesc *>(c->dalloc(sizeof(TensorDesc) * c->tens_h.size()));
+    c->tiles_a = static_cast<Tile *>(c->dalloc(sizeof(Tile) * ta.size()));
+    c->tiles_g = static_cast<Tile *>(c->dalloc(sizeof(Tile) * tg.size()));
+    c->topo_d = static_cast<Topo *>(c->dalloc(sizeof(Topo)));
+    c->topo_scratch = static_cast<Topo *>(c->dalloc(sizeof(Topo)));
+    const int max_grid = c->sms * 32;
+    c->partials = static_cast<double *>(c->dalloc(sizeof(double) * max_grid));
+    c->ticket = static_cast<unsigned int *>(c->dalloc(sizeof(unsigned int) * 4));
+    c->ce_d = static_cast<double *>(c->dalloc(sizeof(double) * 2));
+    c->err_d = static_cast<int32_t *>(c->dalloc(sizeof(int32_t) * 4));
+    if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
+        !c->ce_d || !c->err_d)
+        return oom("tables");
+    if (cudaMallocHost(&c->pinned, 64 + sizeof(Topo)) != cudaSuccess) {
+        cudaGetLastError();
+        c->pinned = nullptr;
+        return oom("pinned host buffer");
+    }
+    cudaError_t es[6];
+    es[0] = cudaMemcpyAsync(c->tens_d, c->tens_h.data(), sizeof(TensorDesc) * c->tens_h.size(), cudaMemcpyHostToDevice, c->stream);
+    es[1] = cudaMemcpyAsync(c->tiles_a, ta.data(), sizeof(Tile) * ta.size(), cudaMemcpyHostToDevice, c->stream);
+    es[2] = cudaMemcpyAsync(c->tiles_g, tg.data(), sizeof(Tile) * tg.size(), cudaMemcpyHostToDevice, c->stream);
+    es[3] = cudaMemsetAsync(c->ticket, 0, sizeof(unsigned int) * 4, c->stream);
+    es[4] = cudaMemsetAsync(c->err_d, 0, sizeof(int32_t) * 4, c->stream);
+    es[5] = cudaMemsetAsync(c->ce_d, 0, sizeof(double) * 2, c->stream);
+    for (cudaError_t x : es)
+        if (x != cudaSuccess) { c->release_all(); return cuda_fail(x, "table upload"); }
+    // the host vectors are freed on return: make the uploads complete first
+    e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) { c->release_all(); return cuda_fail(e, "table upload"); }
+
+    c->grid_a = c->sms * adamw_blocks_per_sm(256);
+    c->grid_g = std::min(max_grid, c->sms * gossip_blocks_per_sm(c->block_g, c->smem_g));
+    c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256));
+
+    InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed};
+    int rc = launch_checked(c, launch_init(ia, c->sms * 8, c->stream), "init kernel");
+    if (rc) { c->release_all(); return rc; }
+    c->started = true;
+    c->round = 0;
+    c->fresh_mask = 0;
+    c->ce_valid = false;
+    std::fill(c->nsteps.begin(), c->nsteps.end(), 0);
+    std::fill(c->p1.begin(), c->p1.end(), 1.0);
+    std::fill(c->p2.begin(), c->p2.end(), 1.0);
+    refresh_spec(c);
+    return GASLOC_OK;
+}
+
+int gasloc_set_local_steps(gasloc_ctx *c, const int32_t *H) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (!H) {
+        c->has_Hi = false;
+        return GASLOC_OK;
+    }
+    for (int32_t i = 0; i < c->n; ++i)
+        if (H[i] < 0 || H[i] > kMaxLocalSteps) return fail(GASLOC_EINVAL, "H_%d = %d out of [0, %d]", i, H[i], kMaxLocalSteps);
+    c->Hi.assign(H, H + c->n);
+    c->has_Hi = true;
+    return GASLOC_OK;
+}
+
+int gasloc_draw_local_steps(gasloc_ctx *c, int32_t hmax) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (hmax < 1 || hmax > kMaxLocalSteps) return fail(GASLOC_EINVAL, "hmax out of [1, %d]", kMaxLocalSteps);
+    for (int32_t i = 0; i < c->n; ++i) {
+        const uint64_t r = host_hash(c->seed, 7, static_cast<uint64_t>(i), 0) >> 32;
+        c->Hi[i] = 1 + static_cast<int32_t>((r * static_cast<uint64_t>(hmax)) >> 32);
+    }
+    c->has_Hi = true;
+    return GASLOC_OK;
+}
+
+int gasloc_get_local_steps(const gasloc_ctx *c, int32_t *H) {
+    if (!c || !H) return fail(GASLOC_EINVAL, "NULL argument");
+    if (!c->has_Hi) return fail(GASLOC_ESTATE, "no per-worker step counts set");
+    std::copy(c->Hi.begin(), c->Hi.end(), H);
+    return GASLOC_OK;
+}
+
+int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (H == 0) return GASLOC_OK;
+    if (H != GASLOC_PER_WORKER_STEPS && (H < 1 || H > kMaxLocalSteps))
+        return fail(GASLOC_EINVAL, "H must be in [1, %d] or GASLOC_PER_WORKER_STEPS", kMaxLocalSteps);
+    if (H == GASLOC_PER_WORKER_STEPS && !c->has_Hi)
+        return fail(GASLOC_ESTATE, "per-worker steps requested but none set");
+    const gasloc_hparams &hp = c->hp;
+    int32_t hmax = H;
+    if (H < 0) hmax = *std::max_element(c->Hi.begin(), c->Hi.end());
+    AdamwArgs a{};
+    a.tens = c->tens_d;
+    a.tiles = c->tiles_a;
+    a.ntiles = c->ntiles_a;
+    a.per_worker_h = hp.per_worker_h;
+    a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
+    a.beta1 = static_cast<float>(hp.beta1);
+    a.beta2 = static_cast<float>(hp.beta2);
+    a.omb1 = static_cast<float>(1.0 - hp.beta1);
+    a.omb2 = static_cast<float>(1.0 - hp.beta2);
+    a.eps = static_cast<float>(hp.eps);
+    a.sigma = static_cast<float>(hp.noise_sigma);
+    for (int32_t s = 0; s < hmax; ++s) {
+        int na = 0;
+        for (int32_t i = 0; i < c->n; ++i) {
+            if (H < 0 && s >= c->Hi[i]) continue;
+            const int64_t nstep = c->nsteps[i] + 1;
+            const double p1 = c->p1[i] * hp.beta1, p2 = c->p2[i] * hp.beta2;
+            const double bc1 = 1.0 - p1, bc2 = 1.0 - p2;
+            a.worker[na] = i;
+            a.step[na] = static_cast<float>(hp.lr / bc1);
+            a.isb[na] = static_cast<float>(1.0 / std::sqrt(bc2));
+            const uint64_t key = host_hash(c->seed, 4, static_cast<uint64_t>(i), static_cast<uint64_t>(nstep));
+            a.key_lo[na] = static_cast<uint32_t>(key);
+            a.key_hi[na] = static_cast<uint32_t>(key >> 32);
+            ++na;
+        }
+        if (na == 0) continue;
+        a.n_active = na;
+        a.from_x_mask = ~c->fresh_mask;
+        rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, c->stream), "adamw kernel");
+        if (rc) return rc;
+        for (int q = 0; q < na; ++q) {
+            const int i = a.worker[q];
+            c->nsteps[i] += 1;
+            c->p1[i] *= hp.beta1;
+            c->p2[i] *= hp.beta2;
+            c->fresh_mask |= 1u << i;
+        }
+    }
+    return GASLOC_OK;
+}
+
+int gasloc_gossip_round(gasloc_ctx *c) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!c->topo_static || !c->topo_ready) {
+        rc = build_topology(c, c->round, c->topo_d);
+        if (rc) return rc;
+        c->topo_ready = c->topo_static;
+    }
+    const gasloc_hparams &hp = c->hp;
+    GossipArgs a{};
+    a.tens = c->tens_d;
+    a.tiles = c->tiles_g;
+    a.ntiles = c->ntiles_g;
+    a.topo = c->topo_d;
+    a.n_workers = c->n;
+    a.mode = hp.outer_mode;
+    a.fresh_mask = c->fresh_mask;
+    a.first_round = c->round == 0 ? 1 : 0;
+    a.tile = c->tile_g;
+    a.stages = c->stages_g;
+    a.eta_out = static_cast<float>(hp.outer_lr);
+    a.mu = static_cast<float>(hp.outer_momentum);
+    a.eta = static_cast<float>(hp.eta);
+    a.alpha = static_cast<float>(hp.alpha);
+    a.oma = static_cast<float>(1.0 - hp.alpha);
+    a.gamma = static_cast<float>(hp.gamma);
+    a.partials = c->partials;
+    a.ticket = c->ticket;
+    a.ce_out = c->ce_d;
+    a.err = c->err_d;
+    const size_t smem = gasloc::gossip_smem_bytes(c->n, c->tile_g, c->stages_g, hp.outer_mode);
+    int grid = c->grid_g;
+    if (smem > c->smem_g) grid = std::max(1, std::min(grid, c->sms * gossip_blocks_per_sm(c->block_g, smem)));
+    rc = launch_checked(c, launch_gossip(a, grid, c->block_g, smem, c->stream), "gossip kernel");
+    if (rc) return rc;
+    c->round += 1;
+    c->fresh_mask = 0;
+    c->ce_valid = true;
+    return GASLOC_OK;
+}
+
+int gasloc_consensus_error(gasloc_ctx *c, double *out) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!out) return fail(GASLOC_EINVAL, "out is NULL");
+    if (!c->ce_valid) {
+        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->partials, c->ticket, c->ce_d};
+        rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
+        if (rc) return rc;
+        c->ce_valid = true;
+    }
+    cudaError_t e = cudaMemcpyAsync(pin_ce(c), c->ce_d, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the consensus error");
+    rc = sync_and_check(c);
+    if (rc) return rc;
+    *out = *pin_ce(c);
+    return GASLOC_OK;
+}
+
+int gasloc_consensus_error_now(gasloc_ctx *c, double *out) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    c->ce_valid = false;
+    return gasloc_consensus_error(c, out);
+}
+
+int gasloc_get_topology(gasloc_ctx *c, int64_t round, int32_t *nbr, float *w, int32_t *deg) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!nbr || !w || !deg) return fail(GASLOC_EINVAL, "NULL output");
+    if (round < 0) return fail(GASLOC_EINVAL, "round must be >= 0");
+    rc = build_topology(c, round, c->topo_scratch);
+    if (rc) return rc;
+    cudaError_t e = cudaMemcpyAsync(pin_topo(c), c->topo_scratch, sizeof(Topo), cudaMemcpyDeviceToHost, c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the topology");
+    rc = sync_and_check(c);
+    if (rc) return rc;
+    const Topo *t = pin_topo(c);
+    const int32_t n = c->n;
+    for (int32_t i = 0; i < n; ++i) {
+        deg[i] = t->deg[i];
+        for (int32_t q = 0; q < n; ++q) {
+            nbr[i * n + q] = q <= t->deg[i] ? t->nbr[i][q] : -1;
+            w[i * n + q] = q <= t->deg[i] ? t->w[i][q] : 0.0f;
+        }
+    }
+    return GASLOC_OK;
+}
+
+int gasloc_average(gasloc_ctx *c, float *dst) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!dst) return fail(GASLOC_EINVAL, "dst is NULL");
+    return launch_checked(c, launch_average(c->tens_d, c->tiles_a, c->ntiles_a, c->n, dst, c->sms * 8, c->stream),
+                          "average kernel");
+}
+
+int gasloc_average_host(gasloc_ctx *c, float *dst) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!dst) return fail(GASLOC_EINVAL, "dst is NULL");
+    float *tmp = static_cast<float *>(c->dalloc(static_cast<size_t>(c->P) * 4));
+    if (!tmp) return fail(GASLOC_ENOMEM, "device allocation failed (average)");
+    rc = gasloc_average(c, tmp);
+    if (!rc) {
+        cudaError_t e = cudaMemcpyAsync(dst, tmp, static_cast<size_t>(c->P) * 4, cudaMemcpyDeviceToHost, c->stream);
+        if (e != cudaSuccess) rc = cuda_fail(e, "copying the average");
+        else rc = sync_and_check(c);
+    }
+    cudaStreamSynchronize(c->stream);
+    c->dfree(tmp);
+    return rc;
+}
+
+int gasloc_buffer(gasloc_ctx *c, int32_t which, int32_t tensor, void **dptr, int64_t *worker_stride) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!dptr) return fail(GASLOC_EINVAL, "dptr is NULL");
+    if (tensor < 0 || tensor >= static_cast<int32_t>(c->tens_h.size())) return fail(GASLOC_EINVAL, "tensor out of range");
+    int64_t stride = 0;
+    float *p = buffer_base(c->tens_h[tensor], which, &stride);
+    if (!p) return fail(GASLOC_EINVAL, "unknown buffer %d", which);
+    *dptr = p;
+    if (worker_stride) *worker_stride = stride;
+    return GASLOC_OK;
+}
+
+int gasloc_read(gasloc_ctx *c, int32_t which, int32_t worker, float *host) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!host) return fail(GASLOC_EINVAL, "host buffer is NULL");
+    rc = check_which_worker(c, which, worker, false);
+    if (rc) return rc;
+    for (const TensorDesc &d : c->tens_h) {
+        int64_t stride = 0;
+        const float *p = buffer_base(d, which, &stride);
+        cudaError_t e = cudaMemcpyAsync(host + d.goff, p + worker * stride, static_cast<size_t>(d.numel) * 4,
+                                        cudaMemcpyDeviceToHost, c->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
+    }
+    return sync_and_check(c);
+}
+
+int gasloc_write(gasloc_ctx *c, int32_t which, int32_t worker, const float *host) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!host) return fail(GASLOC_EINVAL, "host buffer is NULL");
+    rc = check_which_worker(c, which, worker, true);
+    if (rc) return rc;
+    const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
+    const int32_t w0 = worker < 0 ? 0 : worker, w1 = worker < 0 ? rows : worker + 1;
+    for (const TensorDesc &d : c->tens_h) {
+        int64_t stride = 0;
+        float *p = buffer_base(d, which, &stride);
+        cudaError_t e = cudaMemcpyAsync(p + w0 * stride, host + d.goff, static_cast<size_t>(d.numel) * 4,
+                                        cudaMemcpyHostToDevice, c->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
+        for (int32_t i = w0 + 1; i < w1; ++i) {
+            e = cudaMemcpyAsync(p + i * stride, p + w0 * stride, static_cast<size_t>(d.numel) * 4,
+                                cudaMemcpyDeviceToDevice, c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "device-to-device copy");
+        }
+    }
+    if (which == GASLOC_BUF_X) c->ce_valid = false;
+    return sync_and_check(c);
+}
+
+int gasloc_gather(gasloc_ctx *c, int32_t which, int32_t worker, int64_t n, const int64_t *idx, float *out) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (n < 0 || (n > 0 && (!idx || !out))) return fail(GASLOC_EINVAL, "bad gather arguments");
+    rc = check_which_worker(c, which, worker, false);
+    if (rc) return rc;
+    for (int64_t q = 0; q < n; ++q)
+        if (idx[q] < 0 || idx[q] >= c->P) return fail(GASLOC_EINVAL, "index %lld out of range", (long long)idx[q]);
+    if (n == 0) return GASLOC_OK;
+    int64_t *di = static_cast<int64_t *>(c->dalloc(static_cast<size_t>(n) * 8));
+    float *dout = static_cast<float *>(c->dalloc(static_cast<size_t>(n) * 4));
+    if (!di || !dout) {
+        c->dfree(di);
+        c->dfree(dout);
+        return fail(GASLOC_ENOMEM, "device allocation failed (gather)");
+    }
+    cudaError_t e = cudaMemcpyAsync(di, idx, static_cast<size_t>(n) * 8, cudaMemcpyHostToDevice, c->stream);
+    if (e == cudaSuccess) {
+        rc = launch_checked(c, launch_gather(c->tens_d, static_cast<int32_t>(c->tens_h.size()), which, worker, di, n,
+                                             dout, c->err_d, c->stream),
+                            "gather kernel");
+        if (!rc) {
+            e = cudaMemcpyAsync(out, dout, static_cast<size_t>(n) * 4, cudaMemcpyDeviceToHost, c->stream);
+            rc = e == cudaSuccess ? sync_and_check(c) : cuda_fail(e, "gather copy");
+        }
+    } else {
+        rc = cuda_fail(e, "gather index upload");
+    }
+    cudaStreamSynchronize(c->stream);
+    c->dfree(di);
+    c->dfree(dout);
+    return rc;
+}
+
+int gasloc_round(const gasloc_ctx *c, int64_t *round) {
+    if (!c || !round) return fail(GASLOC_EINVAL, "NULL argument");
+    *round = c->round;
+    return GASLOC_OK;
+}
+
+int gasloc_steps_taken(const gasloc_ctx *c, int32_t worker, int64_t *steps) {
+    if (!c || !steps) return fail(GASLOC_EINVAL, "NULL argument");
+    if (worker < 0 || worker >= c->n) return fail(GASLOC_EINVAL, "worker out of range");
+    *steps = c->nsteps[worker];
+    return GASLOC_OK;
+}
+
+int gasloc_launch_count(const gasloc_ctx *c, int64_t *count) {
+    if (!c || !count) return fail(GASLOC_EINVAL, "NULL argument");
+    *count = c->launches;
+    return GASLOC_OK;
+}
+
+// Checkpoint file: header, counters, then every buffer's valid elements
+// (tensor-major, then buffer, then worker).
+namespace {
+struct CkptHeader {
+    char magic[8];
+    int32_t version, n;
+    int64_t P, n_tensors;
+    uint64_t seed;
+    int32_t kind, rows, cols, per_worker_h;
+    int64_t round;
+    uint32_t fresh_mask;
+    int32_t has_Hi;
+};
+}  // namespace
+
+int gasloc_save(gasloc_ctx *c, const char *path) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!path) return fail(GASLOC_EINVAL, "path is NULL");
+    rc = sync_and_check(c);
+    if (rc) return rc;
+    FILE *f = std::fopen(path, "wb");
+    if (!f) return fail(GASLOC_EIO, "cannot open '%s' for writing", path);
+    CkptHeader h{};
+    std::memcpy(h.magic, "GASLOCK1", 8);
+    h.version = 1;
+    h.n = c->n;
+    h.P = c->P;
+    h.n_tensors = static_cast<int64_t>(c->numels.size());
+    h.seed = c->seed;
+    h.kind = c->spec.kind;
+    h.rows = c->spec.rows;
+    h.cols = c->spec.cols;
+    h.per_worker_h = c->hp.per_worker_h;
+    h.round = c->round;
+    h.fresh_mask = c->fresh_mask;
+    h.has_Hi = c->has_Hi ? 1 : 0;
+    bool ok = std::fwrite(&h, sizeof h, 1, f) == 1;
+    ok = ok && std::fwrite(c->numels.data(), 8, c->numels.size(), f) == c->numels.size();
+    ok = ok && std::fwrite(&c->hp, sizeof c->hp, 1, f) == 1;
+    ok = ok && std::fwrite(c->nsteps.data(), 8, c->n, f) == static_cast<size_t>(c->n);
+    ok = ok && std::fwrite(c->Hi.data(), 4, c->n, f) == static_cast<size_t>(c->n);
+    std::vector<float> buf;
+    for (const TensorDesc &d : c->tens_h) {
+        buf.resize(static_cast<size_t>(d.numel));
+        for (int which = GASLOC_BUF_X; ok && which <= GASLOC_BUF_H; ++which) {
+            const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
+            int64_t stride = 0;
+            const float *p = buffer_base(d, which, &stride);
+            for (int32_t i = 0; ok && i < rows; ++i) {
+                if (cudaMemcpy(buf.data(), p + i * stride, buf.size() * 4, cudaMemcpyDeviceToHost) != cudaSuccess) {
+                    std::fclose(f);
+                    return fail(GASLOC_ECUDA, "checkpoint copy failed");
+                }
+                ok = std::fwrite(buf.data(), 4, buf.size(), f) == buf.size();
+            }
+        }
+    }
+    ok = (std::fclose(f) == 0) && ok;
+    if (!ok) return fail(GASLOC_EIO, "short write to '%s'", path);
+    return GASLOC_OK;
+}
+
+int gasloc_load(gasloc_ctx *c, const char *path) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!path) return fail(GASLOC_EINVAL, "path is NULL");
+    FILE *f = std::fopen(path, "rb");
+    if (!f) return fail(GASLOC_EIO, "cannot open '%s'", path);
+    CkptHeader h{};
+    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK1", 8) == 0 && h.version == 1;
+    if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "'%s' is not a checkpoint", path); }
+    if (h.n != c->n || h.P != c->P || h.n_tensors != static_cast<int64_t>(c->numels.size()) || h.seed != c->seed ||
+        h.kind != c->spec.kind || h.rows != c->spec.rows || h.cols != c->spec.cols ||
+        h.per_worker_h != c->hp.per_worker_h) {
+        std::fclose(f);
+        return fail(GASLOC_EINVAL, "checkpoint does not match this context");
+    }
+    std::vector<int64_t> numels(static_cast<size_t>(h.n_tensors));
+    gasloc_hparams hp{};
+    std::vector<int64_t> nsteps(c->n);
+    std::vector<int32_t> Hi(c->n);
+    ok = std::fread(numels.data(), 8, numels.size(), f) == numels.size() && numels == c->numels &&
+         std::fread(&hp, sizeof hp, 1, f) == 1 &&
+         std::fread(nsteps.data(), 8, nsteps.size(), f) == nsteps.size() &&
+         std::fread(Hi.data(), 4, Hi.size(), f) == Hi.size();
+    if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "truncated checkpoint header"); }
+    rc = sync_and_check(c);
+    if (rc) { std::fclose(f); return rc; }
+    std::vector<float> buf;
+    for (const TensorDesc &d : c->tens_h) {
+        buf.resize(static_cast<size_t>(d.numel));
+        for (int which = GASLOC_BUF_X; ok && which <= GASLOC_BUF_H; ++which) {
+            const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
+            int64_t stride = 0;
+            float *p = buffer_base(d, which, &stride);
+            for (int32_t i = 0; ok && i < rows; ++i) {
+                ok = std::fread(buf.data(), 4, buf.size(), f) == buf.size();
+                if (ok && cudaMemcpy(p + i * stride, buf.data(), buf.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+                    std::fclose(f);
+                    return fail(GASLOC_ECUDA, "checkpoint upload failed");
+                }
+            }
+        }
+    }
+    std::fclose(f);
+    if (!ok) return fail(GASLOC_EIO, "truncated checkpoint data");
+    rc = check_hparams(&hp);
+    if (rc) return rc;
+    c->hp = hp;
+    c->round = h.round;
+    c->fresh_mask = h.fresh_mask;
+    c->has_Hi = h.has_Hi != 0;
+    c->Hi = Hi;
+    c->nsteps = nsteps;
+    for (int32_t i = 0; i < c->n; ++i) {
+        double a = 1.0, b = 1.0;
+        for (int64_t s = 0; s < nsteps[i]; ++s) { a *= hp.beta1; b *= hp.beta2; }
+        c->p1[i] = a;
+        c->p2[i] = b;
+    }
+    c->ce_valid = false;
+    refresh_spec(c);
+    return GASLOC_OK;
+}
+
+void gasloc_destroy(gasloc_ctx *c) {
+    if (!c) return;
+    c->release_all();
+    delete c;
+}
+
+}  // extern "C"

@@ -1,0 +1,127 @@
+// internal.h -- structures shared by the C-ABI layer (gasloc.cpp) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace gasloc {
+
+constexpr int kMaxWorkers = 32;
+
+// One parameter tensor of the replica store.  Every array is one allocation
+// of shape [n_workers][wstride] fp32 (h: [1 or n_workers][wstride]);
+// wstride = numel rounded up to 64 floats so each worker slice is 256-byte
+// aligned.  Padding is zero-filled at start and never written afterwards.
+struct TensorDesc {
+    float *x, *y, *m, *v, *b, *c, *h;
+    int64_t numel;     // valid elements per worker
+    int64_t wstride;   // floats between consecutive workers
+    int64_t hstride;   // floats between workers in h (0 when shared)
+    int64_t goff;      // global index of element 0 (concatenation order)
+};
+
+// A contiguous run of at most `tile` elements of one tensor.  start is a
+// multiple of 4, so every tile begins on a 16-byte boundary.
+struct Tile {
+    int32_t tensor;
+    int32_t len;
+    int64_t start;
+};
+
+// Round-t neighbour table (row i: N_i ascending, deg[i] + 1 entries).
+struct Topo {
+    int32_t nbr[kMaxWorkers][kMaxWorkers];
+    float w[kMaxWorkers][kMaxWorkers];
+    int32_t deg[kMaxWorkers];
+};
+
+enum TopoKind : int32_t { kNone = 0, kRing = 1, kComplete = 2, kExp = 3, kTorus = 4,
+                          kMatching = 5, kTwoPeer = 6 };
+
+struct TopoSpec {
+    int32_t kind, n, rows, cols, weights;
+    int32_t pad;
+    uint64_t seed;
+    uint64_t edge_thr;   // edge kept iff hi32(hash) < edge_thr (2^32 = always)
+};
+
+// Device error codes (first one wins, written with atomicCAS).
+enum DevError : int32_t { kDevOk = 0, kDevWaitTimeout = 1, kDevBadIndex = 2 };
+
+// ---------------------------------------------------------------- kernels --
+
+struct InitArgs {
+    const TensorDesc *tens;
+    const Tile *tiles;
+    int64_t ntiles;
+    int32_t n_workers;
+    int32_t per_worker_h;
+    uint64_t seed;
+};
+
+struct AdamwArgs {
+    const TensorDesc *tens;
+    const Tile *tiles;
+    int64_t ntiles;
+    int32_t n_active;
+    int32_t per_worker_h;
+    uint32_t from_x_mask;                 // bit i: worker i starts from x
+    int32_t worker[kMaxWorkers];
+    float step[kMaxWorkers];              // lr / (1 - beta1^n)
+    float isb[kMaxWorkers];               // 1 / sqrt(1 - beta2^n)
+    uint32_t key_lo[kMaxWorkers], key_hi[kMaxWorkers];   // noise key of the step
+    float decay, beta1, beta2, omb1, omb2, eps, sigma;
+};
+
+struct GossipArgs {
+    const TensorDesc *tens;
+    const Tile *tiles;
+    int64_t ntiles;
+    const Topo *topo;
+    int32_t n_workers;
+    int32_t mode;          // GASLOC_OUTER_*
+    uint32_t fresh_mask;   // bit j: worker j took a local step this round
+    int32_t first_round;   // Eq. 2: no momentum term at t = 0
+    int32_t tile;          // elements per tile (4 * blockDim)
+    int32_t stages;
+    float eta_out, mu, eta, alpha, oma, gamma;
+    double *partials;      // [gridDim] per-CTA consensus-error partials
+    unsigned int *ticket;  // last-CTA-done counter (returns to 0)
+    double *ce_out;        // consensus error of the new x
+    int32_t *err;
+};
+
+struct CeArgs {
+    const TensorDesc *tens;
+    const Tile *tiles;
+    int64_t ntiles;
+    int32_t n_workers;
+    double *partials;
+    unsigned int *ticket;
+    double *ce_out;
+};
+
+// Launchers (return cudaGetLastError()).
+cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s);
+cudaError_t launch_topo(const TopoSpec &spec, int64_t round, Topo *out, cudaStream_t s);
+cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s);
+cudaError_t launch_gossip(const GossipArgs &a, int grid, int block, size_t smem, cudaStream_t s);
+cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s);
+cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
+                           int32_t n_workers, float *dst, int grid, cudaStream_t s);
+cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
+                          const int64_t *idx, int64_t n, float *out, int32_t *err,
+                          cudaStream_t s);
+
+// Occupancy-derived persistent grid sizes.
+int adamw_blocks_per_sm(int block);
+int gossip_blocks_per_sm(int block, size_t smem);
+int ce_blocks_per_sm(int block);
+cudaError_t gossip_set_smem(size_t smem);
+size_t gossip_smem_bytes(int n, int tile, int stages, int mode);
+
+// Host-side copy of the counter-based hash (same definition as the device).
+uint64_t host_hash(uint64_t seed, uint64_t tag, uint64_t a, uint64_t b);
+
+}  // namespace gasloc

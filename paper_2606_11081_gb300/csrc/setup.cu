@@ -1,0 +1,256 @@
+// setup.cu -- one-time and cold-path kernels: replica initialisation, the
+// per-round neighbour-table generator, the network average (output of
+// Algorithm 1) and an index gather used for sampled checks.
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "rng.cuh"
+
+namespace gasloc {
+
+namespace {
+
+// Standard-normal stand-in: Irwin-Hall sum of four 24-bit uniforms,
+// (s - 2^25) * fl32(sqrt3 * 2^-24): one rounding in the integer conversion,
+// one in the product.
+__device__ __forceinline__ float normal_std(uint64_t seed, uint64_t tag, uint64_t i, uint64_t k) {
+    int32_t s = 0;
+#pragma unroll
+    for (uint64_t j = 0; j < 4; ++j) s += static_cast<int32_t>(top24(hash4(seed, tag, i, 4 * k + j)));
+    const float scale = static_cast<float>(1.7320508075688772 * 5.9604644775390625e-08);
+    return __fmul_rn(__int2float_rn(s - (1 << 25)), scale);
+}
+
+// h ~ U(0.1, 1): fma(0.9, r * 2^-24, 0.1).
+__device__ __forceinline__ float curvature(uint64_t seed, uint64_t i, uint64_t k) {
+    const float u = __fmul_rn(__uint2float_rn(top24(hash4(seed, kTagCurv, i, k))), 0x1p-24f);
+    return __fmaf_rn(static_cast<float>(0.9), u, static_cast<float>(0.1));
+}
+
+__global__ void init_kernel(const InitArgs a) {
+    const float x0std = static_cast<float>(0.02);
+    for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
+        const Tile tl = a.tiles[ti];
+        const TensorDesc d = a.tens[tl.tensor];
+        for (int e = threadIdx.x; e < tl.len; e += blockDim.x) {
+            const int64_t off = tl.start + e;
+            const uint64_t k = static_cast<uint64_t>(d.goff + off);
+            const float x0 = __fmul_rn(x0std, normal_std(a.seed, kTagX0, 0, k));
+            for (int i = 0; i < a.n_workers; ++i) {
+                const int64_t o = i * d.wstride + off;
+                d.x[o] = x0;
+                d.y[o] = x0;
+                d.c[o] = normal_std(a.seed, kTagCentre, static_cast<uint64_t>(i), k);
+            }
+            const int nh = a.per_worker_h ? a.n_workers : 1;
+            for (int i = 0; i < nh; ++i)
+                d.h[i * d.hstride + off] = curvature(a.seed, static_cast<uint64_t>(i), k);
+        }
+    }
+}
+
+// Neighbour table of round t, one warp.  Lane 0 draws the permutation
+// (Fisher-Yates, Lemire multiply-shift); edges are bitmasks; each lane then
+// applies edge activation to the edges it owns and builds its own row.
+__global__ void topo_kernel(const TopoSpec spec, const int64_t round, Topo *out) {
+    __shared__ uint32_t adj[kMaxWorkers];
+    __shared__ int32_t perm[kMaxWorkers];
+    __shared__ int32_t deg[kMaxWorkers];
+    const int n = spec.n;
+    const int lane = threadIdx.x;
+    if (lane < kMaxWorkers) adj[lane] = 0u;
+    __syncwarp();
+    if (lane == 0) {
+        auto edge = [&](int a, int b) {
+            if (a != b) { adj[a] |= 1u << b; adj[b] |= 1u << a; }
+        };
+        switch (spec.kind) {
+        case kRing:
+            for (int i = 0; i < n; ++i) edge(i, (i + 1) % n);
+            break;
+        case kComplete:
+            for (int i = 0; i < n; ++i)
+                for (int j = i + 1; j < n; ++j) edge(i, j);
+            break;
+        case kExp:
+            for (int i = 0; i < n; ++i)
+                for (int s = 1; s < n; s *= 2) edge(i, (i + s) % n);
+            break;
+        case kTorus:
+            for (int r = 0; r < spec.rows; ++r)
+                for (int c = 0; c < spec.cols; ++c) {
+                    edge(r * spec.cols + c, ((r + 1) % spec.rows) * spec.cols + c);
+                    edge(r * spec.cols + c, r * spec.cols + (c + 1) % spec.cols);
+                }
+            break;
+        case kMatching:
+        case kTwoPeer: {
+            for (int q = 0; q < n; ++q) perm[q] = q;
+            for (int q = n - 1; q >= 1; --q) {
+                const uint64_t r = hash4(spec.seed, kTagPerm, static_cast<uint64_t>(round),
+                                         static_cast<uint64_t>(q)) >> 32;
+                const int j = static_cast<int>((r * static_cast<uint64_t>(q + 1)) >> 32);
+                const int t = perm[q];
+                perm[q] = perm[j];
+                perm[j] = t;
+            }
+            if (spec.kind == kMatching) {
+                for (int p = 0; p + 1 < n; p += 2) edge(perm[p], perm[p + 1]);
+            } else {
+                for (int q = 0; q < n; ++q) edge(perm[q], perm[(q + 1) % n]);
+            }
+            break;
+        }
+        default:
+            break;
+        }
+    }
+    __syncwarp();
+    // edge activation: lane a decides the edges {a < b}
+    uint32_t drop = 0u;
+    if (spec.edge_thr < (1ull << 32) && lane < n) {
+        const uint32_t mine = adj[lane];
+        for (int b = lane + 1; b < n; ++b) {
+            if (!((mine >> b) & 1u)) continue;
+            const uint64_t r = hash4(spec.seed, kTagEdge, static_cast<uint64_t>(round),
+                                     static_cast<uint64_t>(lane) * n + b) >> 32;
+            if (!(r < spec.edge_thr)) drop |= 1u << b;
+        }
+    }
+    __syncwarp();
+    // apply the drops symmetrically: gather every lane's drop mask
+    uint32_t row = lane < n ? adj[lane] : 0u;
+    for (int a = 0; a < n; ++a) {
+        const uint32_t da = __shfl_sync(0xffffffffu, drop, a);
+        if (lane < n) {
+            if (lane == a) row &= ~da;
+            else if ((da >> lane) & 1u) row &= ~(1u << a);
+        }
+    }
+    if (lane < n) deg[lane] = __popc(row);
+    __syncwarp();
+    if (lane < n) {
+        const int di = deg[lane];
+        int q = 0;
+        double rest = 0.0;
+        for (int j = 0; j < n; ++j) {
+            if (j != lane && !((row >> j) & 1u)) continue;
+            double w;
+            if (spec.weights == 0) {            // uniform
+                w = 1.0 / static_cast<double>(di + 1);
+            } else if (spec.weights == 1) {     // Metropolis
+                if (j == lane) {
+                    w = 0.0;                     // filled below
+                } else {
+                    const int dm = di > deg[j] ? di : deg[j];
+                    w = 1.0 / static_cast<double>(1 + dm);
+                }
+            } else {                             // lazy
+                w = di == 0 ? 1.0 : (j == lane ? 0.5 : 0.5 / static_cast<double>(di));
+            }
+            out->nbr[lane][q] = j;
+            out->w[lane][q] = __double2float_rn(w);
+            ++q;
+        }
+        if (spec.weights == 1) {
+            // self weight = 1 - sum of the others, summed in ascending j
+            int qs = 0;
+            for (int j = 0; j < n; ++j) {
+                if (j == lane) continue;
+                if (!((row >> j) & 1u)) continue;
+                const int dm = di > deg[j] ? di : deg[j];
+                rest += 1.0 / static_cast<double>(1 + dm);
+            }
+            for (int q2 = 0; q2 <= di; ++q2)
+                if (out->nbr[lane][q2] == lane) qs = q2;
+            out->w[lane][qs] = __double2float_rn(1.0 - rest);
+        }
+        for (; q < kMaxWorkers; ++q) {
+            out->nbr[lane][q] = lane;
+            out->w[lane][q] = 0.0f;
+        }
+        out->deg[lane] = di;
+    }
+}
+
+// xbar = (1/n) sum_i x_i: fp32 sum in ascending i, times fl32(1/n).
+__global__ void average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
+                               float *dst) {
+    const float inv_n = static_cast<float>(1.0 / n);
+    for (int64_t ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
+        const Tile tl = tiles[ti];
+        const TensorDesc d = tens[tl.tensor];
+        for (int e = threadIdx.x; e < tl.len; e += blockDim.x) {
+            const int64_t off = tl.start + e;
+            float s = 0.0f;
+            for (int i = 0; i < n; ++i) s = __fadd_rn(s, d.x[i * d.wstride + off]);
+            dst[d.goff + off] = __fmul_rn(s, inv_n);
+        }
+    }
+}
+
+__global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
+                              const int64_t *idx, int64_t n, float *out, int32_t *err) {
+    const int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+    if (q >= n) return;
+    const int64_t k = idx[q];
+    // binary search for the tensor holding global index k
+    int lo = 0, hi = ntens - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) / 2;
+        if (tens[mid].goff <= k) lo = mid; else hi = mid - 1;
+    }
+    const TensorDesc d = tens[lo];
+    const int64_t off = k - d.goff;
+    if (k < 0 || off < 0 || off >= d.numel) {
+        atomicCAS(err, kDevOk, kDevBadIndex);
+        out[q] = 0.0f;
+        return;
+    }
+    const float *base;
+    int64_t stride = d.wstride;
+    switch (which) {
+    case 0: base = d.x; break;
+    case 1: base = d.y; break;
+    case 2: base = d.m; break;
+    case 3: base = d.v; break;
+    case 4: base = d.b; break;
+    case 5: base = d.c; break;
+    default: base = d.h; stride = d.hstride; break;
+    }
+    out[q] = base[worker * stride + off];
+}
+
+}  // namespace
+
+cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s) {
+    init_kernel<<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_topo(const TopoSpec &spec, int64_t round, Topo *out, cudaStream_t s) {
+    topo_kernel<<<1, 32, 0, s>>>(spec, round, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
+                           float *dst, int grid, cudaStream_t s) {
+    average_kernel<<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
+                          const int64_t *idx, int64_t n, float *out, int32_t *err, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t grid = (n + 255) / 256;
+    gather_kernel<<<static_cast<unsigned>(grid), 256, 0, s>>>(tens, ntens, which, worker, idx, n,
+                                                               out, err);
+    return cudaGetLastError();
+}
+
+uint64_t host_hash(uint64_t seed, uint64_t tag, uint64_t a, uint64_t b) {
+    return hash4(seed, tag, a, b);
+}
+
+}  // namespace gasloc

@@ -1,0 +1,245 @@
+"""GPU path vs the oracle, element by element, through the C ABI.
+
+Integer work (neighbour tables, degrees, step counts) must be bit-exact.
+fp32 state must lie within |gpu - oracle| <= 1e-5 (1 + |oracle|) (the parity
+bound); because both sides follow the same one-rounding-per-operation
+sequence in fp32, the runs here are also expected to agree bit for bit, and
+that is asserted too so that any drift in the operation order shows up.
+The consensus error is a reduction whose summation order differs between the
+two sides: relative 1e-5.
+"""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2606_11081_gb300 as g
+from paper_2606_11081_gb300 import build as gbuild
+from paper_2606_11081_gb300 import workloads as wl
+
+from _pairs import TOL, make_pair, oracle_problem, within_tol
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    gbuild.build()
+    oracle.build()
+    yield
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def assert_state_equal(ctx, st, which=("x", "y", "m", "v", "b"), exact=True):
+    for w in which:
+        a = ctx.read_all(w)
+        b = st.get_all(w)
+        ok = within_tol(a, b)
+        assert ok.all(), "%s: %d mismatches, max |d| = %g" % (w, (~ok).sum(), np.abs(a - b).max())
+        if exact:
+            assert np.array_equal(a, b.astype(np.float32)), \
+                "%s: not bit-identical (%d differ, max |d| %g)" % (w, (a != b.astype(np.float32)).sum(),
+                                                                   np.abs(a - b).max())
+
+
+# ---------------------------------------------------------------- init ----
+
+@pytest.mark.parametrize("N,P,per_h", [(4, 4099, False), (3, 1, False), (5, 2050, True), (1, 7, False)])
+def test_init_bit_exact(N, P, per_h):
+    ctx, st = make_pair(N, P, "ring" if N > 1 else "none", seed=12345, hp=dict(per_worker_h=per_h))
+    with ctx:
+        for w in ("x", "y", "c", "h"):
+            np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)
+        for w in ("m", "v", "b"):
+            assert not ctx.read_all(w).any()
+        # identical initial replicas: zero consensus error
+        assert ctx.consensus_error() == 0.0
+
+
+# ------------------------------------------------------------ topology ----
+
+TOPO_CASES = [
+    (4, "ring", {}), (8, "exp", {}), (32, "exp", {}), (8, "torus:2x4", {"weights": "metropolis"}),
+    (6, "complete", {}), (3, "none", {}), (16, "matching", {}), (5, "matching", {}),
+    (8, "2peer", {"weights": "lazy"}), (7, "2peer", {"weights": "uniform"}),
+    (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
+    (12, "exp", {"weights": "uniform", "edge_prob": 0.3}),
+    (9, "ring", {"weights": "lazy", "edge_prob": 0.8}),
+]
+
+
+@pytest.mark.parametrize("N,topo,kw", TOPO_CASES)
+def test_topology_bit_exact(N, topo, kw):
+    ctx, st = make_pair(N, 8, topo, seed=99, hp=kw)
+    with ctx:
+        orc = oracle.get("f64")
+        pb = oracle_problem(N, 8, topo, 99, dict(wl.COMMON_HP, **kw))
+        for t in list(range(40)) + [1000, 123456789]:
+            nbr, w, deg = ctx.topology(t)
+            onbr, ow, odeg = orc.topology(pb, t)
+            np.testing.assert_array_equal(deg, odeg)
+            for i in range(N):
+                k = deg[i] + 1
+                np.testing.assert_array_equal(nbr[i, :k], onbr[i, :k])
+                np.testing.assert_array_equal(w[i, :k], ow[i, :k].astype(np.float32))
+
+
+# --------------------------------------------------------- local steps ----
+
+def test_local_steps_bit_exact():
+    ctx, st = make_pair(4, 4099, "ring", seed=7, hp=dict(lr=1e-3, noise_sigma=0.05))
+    with ctx:
+        ctx.local_steps(3)
+        st.local_steps(3)
+        assert_state_equal(ctx, st, ("y", "m", "v"))
+        for i in range(4):
+            assert ctx.steps_taken(i) == st.steps_taken(i) == 3
+
+
+def test_heterogeneous_steps_per_worker_h():
+    Hi = np.array([0, 1, 3, 2, 5], np.int32)
+    ctx, st = make_pair(5, 3001, "exp", seed=8, hp=dict(per_worker_h=True, lr=1e-3), Hi=Hi)
+    with ctx:
+        for _ in range(3):
+            ctx.local_steps(g.PER_WORKER_STEPS)
+            st.local_steps(0, Hi)
+            ctx.gossip_round()
+            st.gossip_round()
+        assert_state_equal(ctx, st)
+        for i in range(5):
+            assert ctx.steps_taken(i) == 3 * Hi[i]
+
+
+# --------------------------------------------------------- trajectories ---
+
+MODES = ["nesterov", "sgdm", "sgd", "eq2", "dadam", "local_dadam"]
+GRAPHS = [(8, "exp", {}), (16, "matching", {}), (8, "torus:2x4", {"weights": "metropolis"}),
+          (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}), (6, "2peer", {"weights": "lazy"})]
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("N,topo,kw", GRAPHS)
+def test_trajectory_parity(mode, N, topo, kw):
+    P, R, H = 2 * 1024 + 3, 5, 2
+    hp = dict(kw, outer=mode, lr=2e-3, eta=0.9, alpha=0.8, gamma=0.3, outer_lr=0.7,
+              outer_momentum=0.9, noise_sigma=0.02)
+    ctx, st = make_pair(N, P, topo, seed=1000 + N, hp=hp)
+    with ctx:
+        for r in range(R):
+            ctx.local_steps(H)
+            st.local_steps(H)
+            ctx.gossip_round()
+            st.gossip_round()
+            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+        assert_state_equal(ctx, st, ("x", "b", "m", "v"))
+
+
+@pytest.mark.parametrize("N,P,topo", [(1, 5, "none"), (4, 1, "ring"), (4, 3, "complete"),
+                                      (2, 1023, "matching"), (5, 1029, "matching"),
+                                      (3, 20000, "complete")])
+def test_edge_case_shapes(N, P, topo):
+    ctx, st = make_pair(N, P, topo, seed=5, hp=dict(lr=5e-3))
+    with ctx:
+        for _ in range(4):
+            ctx.local_steps(2)
+            st.local_steps(2)
+            ctx.gossip_round()
+            st.gossip_round()
+        assert_state_equal(ctx, st, ("x", "b"))
+        assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+
+
+def test_ring_n4_p1m_full_size():
+    # The 4-worker ring workload at its full size: 1,048,576 parameters, 50 rounds
+    w = wl.WORKLOADS["ring_n4_p1m"]
+    ctx, st = make_pair(w.n_workers, w.n_params, w.topology, w.seed, wl.hparams_of(w))
+    with ctx:
+        for r in range(w.rounds):
+            ctx.local_steps(w.H)
+            st.local_steps(w.H)
+            ctx.gossip_round()
+            st.gossip_round()
+            if r % 10 == 9:
+                assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)
+        assert_state_equal(ctx, st, ("x", "b", "m", "v"))
+        np.testing.assert_allclose(ctx.average_host(), st.average(), rtol=2e-6, atol=1e-7)
+
+
+# --------------------------------------------------------- CE / average ---
+
+def test_consensus_error_closed_form_and_paths():
+    N, P = 7, 5003
+    ctx, _ = make_pair(N, P, "ring", seed=3)
+    with ctx:
+        for i in range(N):
+            ctx.write("x", i, np.full(P, float(i), np.float32))
+        # per-element fp32 shifted sums: relative error below ~N * 2^-22
+        assert ctx.consensus_error() == pytest.approx(P * (N * N - 1) / 12, rel=5e-6)
+        ctx.local_steps(1)
+        ctx.gossip_round()
+        fused = ctx.consensus_error()
+        assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-12)
+
+
+# ------------------------------------------------------ layout / resume ---
+
+def test_tensor_list_equals_flat():
+    numels = [1000, 3, 4097, 64, 1, 2048, 5]
+    P = sum(numels)
+    hp = dict(weights="metropolis", lr=2e-3)
+    a, _ = make_pair(8, P, "torus:2x4", seed=11, hp=hp)
+    b, _ = make_pair(8, P, "torus:2x4", seed=11, hp=hp, numels=numels)
+    with a, b:
+        for _ in range(4):
+            for c in (a, b):
+                c.local_steps(3)
+                c.gossip_round()
+        # per-element terms are identical; the fp32 sums of a 16-byte column
+        # group different elements where a tensor boundary is not 4-aligned
+        assert a.consensus_error() == pytest.approx(b.consensus_error(), rel=1e-6)
+        for w in ("x", "y", "m", "v", "b", "c", "h"):
+            np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
+        # the per-tensor buffers are separate allocations with the real sizes
+        v = b.view("x", 2, numels[2])
+        assert tuple(v.shape) == (8, numels[2])
+        np.testing.assert_array_equal(v.cpu().numpy(), b.read_all("x")[:, 1003:1003 + 4097])
+
+
+def test_resume_is_exact(tmp_path):
+    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True)
+    a, _ = make_pair(6, 3000, "exp", seed=21, hp=hp, Hi=[1, 2, 3, 1, 2, 3])
+    with a:
+        for _ in range(3):
+            a.local_steps(g.PER_WORKER_STEPS)
+            a.gossip_round()
+        path = str(tmp_path / "ckpt.bin")
+        a.save(path)
+        for _ in range(3):
+            a.local_steps(g.PER_WORKER_STEPS)
+            a.gossip_round()
+        xa = a.read_all("x")
+        ce_a = a.consensus_error()
+    b, _ = make_pair(6, 3000, "exp", seed=21, hp=hp, Hi=[1, 1, 1, 1, 1, 1])
+    with b:
+        b.load(path)
+        assert b.round == 3
+        for _ in range(3):
+            b.local_steps(g.PER_WORKER_STEPS)
+            b.gossip_round()
+        np.testing.assert_array_equal(b.read_all("x"), xa)
+        assert b.consensus_error() == ce_a
+
+
+def test_gather_rejects_bad_index():
+    ctx, _ = make_pair(2, 100, "ring", seed=1)
+    with ctx:
+        with pytest.raises(g.GaslocError) as e:
+            ctx.gather("x", 0, np.array([5, 100]))
+        assert e.value.code == g.EINVAL
+        np.testing.assert_array_equal(ctx.gather("x", 1, np.array([0, 99, 42])),
+                                      ctx.read("x", 1)[[0, 99, 42]])
