@@ -176,6 +176,30 @@ int gasloc_consensus_error(gasloc_ctx *ctx, double *out);
  * reduction kernel (ignores the value the last gossip round produced). */
 int gasloc_consensus_error_now(gasloc_ctx *ctx, double *out);
 
+/* Consensus error of caller-owned replicas, for callers that cannot allocate
+ * device memory at the point they need it: a framework that owns all device
+ * memory through its own pool (a side cudaMalloc could fail or fragment it),
+ * a latency-critical loop where cudaMalloc/cudaFree would synchronise the
+ * device, or a plug-in that is handed pre-allocated buffers only.  The paper
+ * has no counterpart; this is a service of the library.
+ *   x: device pointer, n_workers rows of worker_stride floats each (row i is
+ *      replica i; the caller owns all n_workers * worker_stride floats),
+ *      16-byte aligned, worker_stride a multiple of 4 and >= n_params.
+ *   ce_out_device: device pointer to one double that receives
+ *      (1/n) sum_i ||x_i - xbar||^2 (same arithmetic as gasloc_consensus_error).
+ *   cuda_stream: the stream the work is enqueued on (asynchronous).
+ * Nothing is allocated: the reduction's scratch is a fixed 512 KiB + 256 B
+ * array compiled into the library, held by every GPU that loads it until the
+ * process exits.  n_params above 536,870,912 is rejected (GASLOC_ENOMEM).
+ * The first call on a device looks up that array's device address (and the
+ * launch shape) for the current device; make that first call before any
+ * stream capture.  Every call reuses the same array (its completion counter is
+ * cleared at the start of each call): calls whose work overlaps on the GPU
+ * race, so serialise them (one stream, or events).  Errors: EINVAL (null or
+ * misaligned pointers, bad sizes), ENOMEM (size limit), ECUDA. */
+int gasloc_consensus_error_noalloc(const float *x, int32_t n_workers, int64_t n_params,
+                                   int64_t worker_stride, double *ce_out_device, void *cuda_stream);
+
 /* Neighbour table of round `round` as the device generates it: host arrays
  * nbr[n*n] (row i: N_i ascending, deg[i]+1 valid entries), w[n*n] (fp32) and
  * deg[n] (graph degree, self excluded).  Synchronising. */

@@ -69,6 +69,7 @@ SIGNATURES = {
     "gasloc_gossip_round": (ctypes.c_int, [_P]),
     "gasloc_consensus_error": (ctypes.c_int, [_P, _DP]),
     "gasloc_consensus_error_now": (ctypes.c_int, [_P, _DP]),
+    "gasloc_consensus_error_noalloc": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P]),
     "gasloc_get_topology": (ctypes.c_int, [_P, _I64, _I32P, _FP, _I32P]),
     "gasloc_average": (ctypes.c_int, [_P, _P]),
     "gasloc_average_host": (ctypes.c_int, [_P, _FP]),
@@ -196,6 +197,15 @@ def gasloc_consensus_error_now(ctx) -> float:
     out = ctypes.c_double()
     _check(_lib.gasloc_consensus_error_now(ctx, ctypes.byref(out)))
     return out.value
+
+
+def gasloc_consensus_error_noalloc(x_ptr: int, n_workers: int, n_params: int, worker_stride: int,
+                                   ce_out_ptr: int, stream_handle: int = 0) -> None:
+    """Consensus error of caller-owned replicas into a caller-owned device
+    double, without any device allocation (asynchronous on the stream)."""
+    _check(load_library().gasloc_consensus_error_noalloc(
+        ctypes.c_void_p(x_ptr), n_workers, n_params, worker_stride, ctypes.c_void_p(ce_out_ptr),
+        ctypes.c_void_p(stream_handle)))
 
 
 def gasloc_get_topology(ctx, round_: int, n_workers: int):

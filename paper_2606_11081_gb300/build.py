@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 ROOT = os.path.dirname(HERE)
 LIB = os.path.join(HERE, "libgasloc.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["gasloc.cpp", "setup.cu", "adamw.cu", "gossip.cu", "ce.cu"]
+SOURCES = ["gasloc.cpp", "setup.cu", "adamw.cu", "gossip.cu", "ce.cu", "ce_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -47,6 +47,8 @@ int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
 }  // namespace
 
+void gasloc::set_last_error(const char *msg) { g_err = msg; }
+
 struct gasloc_ctx {
     int32_t n = 0;
     int64_t P = 0;

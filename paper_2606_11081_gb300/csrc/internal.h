@@ -121,6 +121,9 @@ int ce_blocks_per_sm(int block);
 cudaError_t gossip_set_smem(size_t smem);
 size_t gossip_smem_bytes(int n, int tile, int stages, int mode);
 
+// Sets the thread-local message returned by gasloc_last_error().
+void set_last_error(const char *msg);
+
 // Host-side copy of the counter-based hash (same definition as the device).
 uint64_t host_hash(uint64_t seed, uint64_t tag, uint64_t a, uint64_t b);
 
