@@ -239,7 +239,7 @@ def workload_config(w, args):
 def main():
     args = parse_args()
     from paper_2606_11081_gb300 import workloads as wl
-    w = wl.WORKLOADS[args.workload or wl.BENCH_WORKLOAD]
+    w = wl.ALL_WORKLOADS[args.workload or wl.BENCH_WORKLOAD]
     if args.impl == "reference":
         return run_reference(args, w)
 

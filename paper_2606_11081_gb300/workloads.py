@@ -90,6 +90,20 @@ WORKLOADS = {
         draw_hmax=8),
 }
 
+# A reduced copy of the benchmark workload for profiler captures: 16 Mi
+# parameters (3.2 GB of replica state, well above the 129 MB L2).
+PROFILE_WORKLOADS = {
+    "exp_n8_p16m": Workload(
+        "exp_n8_p16m", 8, 1 << 24, "exp", 1, 10,
+        hp=dict(weights="uniform", noise_sigma=0.01)),
+    "exp_n32_p4m_hetero": Workload(
+        "exp_n32_p4m_hetero", 32, 1 << 22, "exp", -1, 10,
+        hp=dict(weights="metropolis", noise_sigma=0.01, edge_prob=0.5, per_worker_h=True),
+        draw_hmax=8),
+}
+
+ALL_WORKLOADS = dict(WORKLOADS, **PROFILE_WORKLOADS)
+
 # AdamW settings shared by every workload (App. B: weight decay 0.1,
 # betas (0.9, 0.95)); constant lr 3e-4; Nesterov outer step 0.7 / 0.9.
 COMMON_HP = dict(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1,
