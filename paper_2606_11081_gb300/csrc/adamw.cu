@@ -6,8 +6,8 @@
 // writes y, m, v -- 28 bytes -- plus 4 bytes of shared curvature h per element
 // (h is per worker in the heterogeneous workload: 32 bytes per worker-element).
 // One thread owns one 16-byte column of a tile and walks the active workers U
-// at a time, issuing all 4U loads before any arithmetic so that 16-byte
-// requests stay in flight.  The synthetic gradient g = h (y - c) + sigma xi
+// at a time (U = 4, or 3 with per-worker h), issuing all of their 16-byte loads
+// before any arithmetic so that 15-16 requests per thread stay in flight.  The synthetic gradient g = h (y - c) + sigma xi
 // is formed in registers; xi comes from a 32-bit counter hash of the element
 // index and the step key, so the gradient costs no memory traffic.
 //
@@ -59,7 +59,7 @@ __device__ __forceinline__ float noise_xi(uint32_t k, uint32_t klo, uint32_t khi
 }
 
 template <int U, bool PER_WORKER_H>
-__global__ void __launch_bounds__(kBlock) adamw_kernel(const AdamwArgs a) {
+__global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     const Consts kc{a.decay, a.beta1, a.beta2, a.omb1, a.omb2, a.eps, a.sigma};
     int32_t cur = -1;
     TensorDesc d{};
@@ -132,18 +132,19 @@ __global__ void __launch_bounds__(kBlock) adamw_kernel(const AdamwArgs a) {
 
 }  // namespace
 
-int adamw_blocks_per_sm(int block) {
+int adamw_blocks_per_sm(int block, bool per_worker_h) {
     int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<4, false>, block, 0) !=
-        cudaSuccess)
-        return 1;
+    const cudaError_t e =
+        per_worker_h ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<3, true>, block, 0)
+                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<4, false>, block, 0);
+    if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
 }
 
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s) {
     (void)block;
     if (a.per_worker_h)
-        adamw_kernel<4, true><<<grid, kBlock, 0, s>>>(a);
+        adamw_kernel<3, true><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
     else
         adamw_kernel<4, false><<<grid, kBlock, 0, s>>>(a);
     return cudaGetLastError();

@@ -71,9 +71,9 @@ struct gasloc_ctx {
     int64_t ntiles_a = 0;
     Tile *tiles_g = nullptr;
     int64_t ntiles_g = 0;
-    int tile_g = 0, block_g = 0, stages_g = 0;
-    size_t smem_g = 0;
-    int grid_a = 0, grid_g = 0, grid_ce = 0;
+    int tile_g = 0;
+    int grid_a = 0, grid_ce = 0;
+    int grid_gm[6] = {0, 0, 0, 0, 0, 0};   // gossip grid per outer mode
     Topo *topo_d = nullptr, *topo_scratch = nullptr;
     double *partials = nullptr;
     unsigned int *ticket = nullptr;
@@ -370,21 +370,12 @@ int gasloc_start(gasloc_ctx *c) {
     if (cudaMemGetInfo(&fr, &tot) == cudaSuccess && static_cast<size_t>(need) > fr)
         return fail(GASLOC_ENOMEM, "replica store needs %lld bytes, %zu free", (long long)need, fr);
 
-    // gossip launch shape: 16-byte column per thread; stage ~32 KB of sent rows
-    int block = 2048 / n;
-    block = std::max(64, std::min(256, block));
-    int pw = 64;
-    while (pw * 2 <= block) pw *= 2;
-    c->block_g = pw;
-    c->tile_g = 4 * c->block_g;
-    const int rows = c->hp.outer_mode == GASLOC_OUTER_EQ2 ? 2 * n : n;
-    const size_t stage_bytes = static_cast<size_t>(rows) * c->tile_g * 4;
-    int stages = static_cast<int>((110 * 1024 - 8704) / stage_bytes);
-    c->stages_g = std::max(2, std::min(4, stages));
-    // the EQ2 layout bounds the smem attribute for every mode
-    c->smem_g = gasloc::gossip_smem_bytes(n, c->tile_g, c->stages_g, c->hp.outer_mode);
-    const size_t smem_max = gasloc::gossip_smem_bytes(n, c->tile_g, c->stages_g, GASLOC_OUTER_EQ2);
-    e = gossip_set_smem(smem_max);
+    // gossip launch shape (the tile depends on n only; stages and shared
+    // memory on the mode's staged rows): size the attribute for the largest
+    size_t smem_attr = 0;
+    for (int m = 0; m < 6; ++m) smem_attr = std::max(smem_attr, gossip_shape(n, m).smem);
+    c->tile_g = gossip_shape(n, GASLOC_OUTER_NESTEROV).tile;
+    e = gossip_set_smem(smem_attr);
     if (e != cudaSuccess) return cuda_fail(e, "gossip shared-memory attribute");
 
     auto oom = [&](const char *what) {
@@ -463,8 +454,11 @@ int gasloc_start(gasloc_ctx *c) {
     e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) { c->release_all(); return cuda_fail(e, "table upload"); }
 
-    c->grid_a = c->sms * adamw_blocks_per_sm(256);
-    c->grid_g = std::min(max_grid, c->sms * gossip_blocks_per_sm(c->block_g, c->smem_g));
+    c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0);
+    for (int m = 0; m < 6; ++m) {
+        const GossipShape sm = gossip_shape(n, m);
+        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, sm.smem));
+    }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256));
 
     InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed};
@@ -584,8 +578,10 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     a.mode = hp.outer_mode;
     a.fresh_mask = c->fresh_mask;
     a.first_round = c->round == 0 ? 1 : 0;
-    a.tile = c->tile_g;
-    a.stages = c->stages_g;
+    const GossipShape gs = gossip_shape(c->n, hp.outer_mode);
+    a.tile = gs.tile;
+    a.groups = gs.groups;
+    a.stages = gs.stages;
     a.eta_out = static_cast<float>(hp.outer_lr);
     a.mu = static_cast<float>(hp.outer_momentum);
     a.eta = static_cast<float>(hp.eta);
@@ -596,10 +592,7 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     a.ticket = c->ticket;
     a.ce_out = c->ce_d;
     a.err = c->err_d;
-    const size_t smem = gasloc::gossip_smem_bytes(c->n, c->tile_g, c->stages_g, hp.outer_mode);
-    int grid = c->grid_g;
-    if (smem > c->smem_g) grid = std::max(1, std::min(grid, c->sms * gossip_blocks_per_sm(c->block_g, smem)));
-    rc = launch_checked(c, launch_gossip(a, grid, c->block_g, smem, c->stream), "gossip kernel");
+    rc = launch_checked(c, launch_gossip(a, c->grid_gm[hp.outer_mode], gs.smem, c->stream), "gossip kernel");
     if (rc) return rc;
     c->round += 1;
     c->fresh_mask = 0;

@@ -2,27 +2,39 @@
 // DAdam / Local-DAdam) for all workers, fused with the outer optimizer and the
 // consensus-error reduction of the new replicas.
 //
-// Data movement.  A persistent CTA walks its tiles in a static round-robin.
-// For each tile, one thread issues one 1-D bulk copy (TMA engine) per worker of
-// that worker's sent slice (y_j, or x_j if it took no local step) into a
-// shared-memory stage; S stages are in flight.  Every neighbour slice is
-// therefore read from HBM exactly once per tile, however many workers mix it.
-// The worker's own x_i and outer momentum b_i are streamed with 16-byte loads
-// and stores.  GASLoC moves 20 bytes per worker-element: y (4, staged),
-// x and b (8 read, 8 written).
+// Pipeline (one CTA per SM, persistent, static round-robin over tiles):
+//  * one producer warp (lane j handles worker j) moves ALL data with the
+//    TMA engine: for each tile it issues one 1-D bulk copy per staged row --
+//    every worker's sent slice (y_j, or x_j if the worker took no local step)
+//    plus the worker's own rows the update needs (x_i, b_i) -- into an
+//    S-stage shared-memory ring whose "full" mbarrier counts the bytes, and
+//    after the consumers release a stage ("empty" mbarrier) it writes the
+//    updated rows back with bulk stores before refilling the stage;
+//  * 256 consumer threads never touch global memory in the loop: thread
+//    (g, c) owns 16-byte column c of the tile for workers g, g+G, ...
+//    (G = 1, 2, 4 for n <= 8, 16, 32), reads the neighbours' rows from shared
+//    memory, applies the outer update in place and accumulates the column's
+//    consensus-error terms.
+// Every neighbour slice is read from HBM once per round however many workers
+// mix it: GASLoC/Nesterov moves 20 bytes per worker-element (y 4, x 4 + 4,
+// b 4 + 4).  No block-wide barrier is taken inside the loop (a consumer-only
+// named barrier per tile combines the consensus-error terms when G > 1).
 //
-// Compute.  Thread t owns the 16-byte column t of the tile for every worker:
-//   acc_i = sum_{j in N_i, ascending} fma(w_ij, s_j, acc)
-// then the outer update, then the column's consensus-error contribution
-//   e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n,  s = new x_0k,
-// which equals sum_i (x_ik - xbar_k)^2 and needs no second pass.  Per-thread
-// sums go to double, then warp shuffles, then one partial per CTA; the last
-// CTA to finish (atomic ticket, no waiting) adds the partials in CTA order.
+// Arithmetic per element, one rounding per operation (the oracle's order):
+//   acc_i = sum_{j in N_i ascending} fma(w_ij, s_j, acc)
+//   Nesterov: D = x - acc; b = fma(mu, b, D); x = fma(-eta_out, fma(mu, b, D), x)
+//   (SGD, SGDM, Eq. 2, DAdam, Local-DAdam: see outer_update).
+// Consensus error: per element e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
+// S2 = sum_i (x_i - s)^2, s = worker 0's new x (G = 1) or its sent value
+// (G > 1; a shift every group can read); fp32 per element, fp64 across elements,
+// one partial per CTA, the last CTA (atomic ticket, nothing waits) adds the
+// partials in CTA order.
 //
-// Waiting.  Every wait on a stage barrier is bounded (2 s of wall time).  On
-// a timeout the CTA records kDevWaitTimeout, waits (bounded) for its copies
-// still in flight, contributes a NaN partial so that the ticket protocol
-// completes, and returns.
+// Waiting: every mbarrier wait is bounded (2 s).  A consumer that times out
+// records kDevWaitTimeout and the CTA stops computing but keeps arriving on
+// its barriers; the producer stops issuing, waits (bounded) for copies it has
+// in flight and for its stores, and the CTA returns a NaN partial so that the
+// ticket protocol completes.
 #include <cuda_runtime.h>
 
 #include "internal.h"
@@ -34,28 +46,28 @@ namespace {
 
 constexpr int kOutSgd = 0, kOutSgdm = 1, kOutNesterov = 2, kOutEq2 = 3, kOutDadam = 4,
               kOutLocalDadam = 5;
+constexpr int kConsumers = 256;                      // 8 warps
+constexpr int kThreads = kConsumers + 32;            // + producer warp
 constexpr int kMaxStages = 4;
-constexpr size_t kOffBars = sizeof(Topo);                       // 8320
-constexpr size_t kOffRed = kOffBars + 8 * 8;                     // 8384
-constexpr size_t kOffFlag = kOffRed + 32 * 8;                    // 8640
-constexpr size_t kOffStages = 8704;                              // 128-byte aligned
-static_assert(kOffFlag + 16 <= kOffStages, "smem layout");
+constexpr size_t kOffFull = sizeof(Topo);            // 8320
+constexpr size_t kOffEmpty = kOffFull + 8 * kMaxStages;
+constexpr size_t kOffRed = kOffEmpty + 8 * kMaxStages;
+constexpr size_t kOffFlags = kOffRed + 8 * (kThreads / 32);
+constexpr size_t kOffCe = 8704;                      // 2 x [G][cols] x (S1, S2) float4
+constexpr size_t kCeBytes = 2 * kConsumers * 32;
+constexpr size_t kOffStages = kOffCe + kCeBytes;     // 25088, 128-byte aligned
+static_assert(kOffFlags + 16 <= kOffCe, "smem layout");
 static_assert(kOffStages % 128 == 0, "stage alignment");
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
+// Rows staged per worker: kind 0 = the mixed quantity, kind 1 = own x (own y
+// for the DAdam modes), kind 2 = own b.
 template <int MODE>
-struct ModeTraits {
-    static constexpr bool kStageX = MODE == kOutEq2;                        // extra x rows
+struct ModeRows {
+    static constexpr int kRows = (MODE == kOutSgd || MODE == kOutDadam) ? 2 : 3;
     static constexpr bool kMixX = MODE == kOutDadam || MODE == kOutLocalDadam;
-    static constexpr bool kLoadX = MODE == kOutSgd || MODE == kOutSgdm || MODE == kOutNesterov;
-    static constexpr bool kLoadB = MODE != kOutSgd && MODE != kOutDadam;
-    static constexpr bool kWriteB = kLoadB;
-    static constexpr bool kLoadY = kMixX;                                    // own y_i
+    static constexpr bool kHasB = kRows == 3;
 };
-
-__device__ __forceinline__ float lane_of(const float4 &v, int l) {
-    return l == 0 ? v.x : (l == 1 ? v.y : (l == 2 ? v.z : v.w));
-}
 
 template <int MODE>
 __device__ __forceinline__ float outer_update(float acc, float x, float y, float &b, float z,
@@ -91,210 +103,305 @@ __device__ __forceinline__ float outer_update(float acc, float x, float y, float
     }
 }
 
+__device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
+__device__ __forceinline__ float lane_of(const float4 &v, int l) {
+    return l == 0 ? v.x : (l == 1 ? v.y : (l == 2 ? v.z : v.w));
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ void bulk_s2g(void *dst_gmem, const void *src_smem, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst_gmem),
+                 "r"(ptx::smem_addr(src_smem)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Named barrier 1 over the 256 consumer threads (the producer warp never
+// takes it).  The non-aligned form: threads of a warp may arrive separately.
+__device__ __forceinline__ void consumer_barrier() {
+    asm volatile("barrier.sync 1, %0;" ::"r"(kConsumers) : "memory");
+}
+
 template <int MODE>
-__global__ void __launch_bounds__(256) gossip_kernel(const GossipArgs a) {
-    using T = ModeTraits<MODE>;
+__global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a) {
+    using R = ModeRows<MODE>;
     extern __shared__ __align__(128) unsigned char smem[];
     Topo *tp = reinterpret_cast<Topo *>(smem);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBars);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + kOffFull);
+    uint64_t *empty = reinterpret_cast<uint64_t *>(smem + kOffEmpty);
     double *red = reinterpret_cast<double *>(smem + kOffRed);
-    int *flag = reinterpret_cast<int *>(smem + kOffFlag);
+    volatile int *flags = reinterpret_cast<volatile int *>(smem + kOffFlags);   // [0] abort, [1] last
+    float4 *cebuf = reinterpret_cast<float4 *>(smem + kOffCe);
     float *stages = reinterpret_cast<float *>(smem + kOffStages);
 
     const int n = a.n_workers;
     const int TILE = a.tile;
+    const int G = a.groups;
+    const int cols = TILE / 4;
     const int S = a.stages;
-    const int rows = T::kStageX ? 2 * n : n;
-    const size_t stage_floats = static_cast<size_t>(rows) * TILE;
+    const size_t stage_floats = static_cast<size_t>(R::kRows) * n * TILE;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     {   // neighbour table -> shared memory
         const int *src = reinterpret_cast<const int *>(a.topo);
         int *dst = reinterpret_cast<int *>(tp);
-        for (int q = threadIdx.x; q < static_cast<int>(sizeof(Topo) / 4); q += blockDim.x)
-            dst[q] = src[q];
+        for (int q = threadIdx.x; q < static_cast<int>(sizeof(Topo) / 4); q += blockDim.x) dst[q] = src[q];
     }
     if (threadIdx.x == 0) {
-        for (int s = 0; s < S; ++s) ptx::mbar_init(&bars[s], 1);
+        for (int s = 0; s < S; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], kConsumers / 32);
+        }
         ptx::fence_mbar_init();
-        *flag = 0;
+        flags[0] = 0;
+        flags[1] = 0;
     }
     __syncthreads();
 
     const int64_t first = blockIdx.x, gstride = gridDim.x;
     const int64_t my_n = a.ntiles > first ? (a.ntiles - first + gstride - 1) / gstride : 0;
-
-    // Producer (thread 0): bulk-copy the sent rows of local tile `it`.
-    auto issue = [&](int64_t it) {
-        const Tile tl = a.tiles[first + it * gstride];
-        const TensorDesc &d = a.tens[tl.tensor];
-        const uint32_t bytes = static_cast<uint32_t>(((tl.len + 3) & ~3) * 4);
-        uint64_t *bar = &bars[it % S];
-        float *st = stages + (it % S) * stage_floats;
-        ptx::mbar_arrive_expect_tx(bar, bytes * static_cast<uint32_t>(rows));
-        for (int j = 0; j < n; ++j) {
-            const float *base;
-            if (T::kMixX) base = d.x;
-            else base = ((a.fresh_mask >> j) & 1u) ? d.y : d.x;
-            ptx::bulk_g2s(st + static_cast<size_t>(j) * TILE, base + j * d.wstride + tl.start, bytes,
-                          bar);
-        }
-        if (T::kStageX)
-            for (int j = 0; j < n; ++j)
-                ptx::bulk_g2s(st + static_cast<size_t>(n + j) * TILE, d.x + j * d.wstride + tl.start,
-                              bytes, bar);
-    };
-    if (threadIdx.x == 0)
-        for (int64_t it = 0; it < my_n && it < S; ++it) issue(it);
-
-    const float inv_n = static_cast<float>(1.0 / n);
     double ce_acc = 0.0;
-    int32_t cur = -1;
-    TensorDesc d{};
-    bool aborted = false;
-    int64_t it = 0;
-    for (; it < my_n; ++it) {
-        const int stage = static_cast<int>(it % S);
-        const uint32_t parity = static_cast<uint32_t>((it / S) & 1);
-        const bool ok = ptx::mbar_wait_bounded(&bars[stage], parity, kWaitLimitNs);
-        if (__syncthreads_or(!ok)) {
-            aborted = true;
-            break;
-        }
-        const Tile tl = a.tiles[first + it * gstride];
-        if (tl.tensor != cur) {
-            d = a.tens[tl.tensor];
-            cur = tl.tensor;
-        }
-        const int e0 = 4 * threadIdx.x;
-        float *st = stages + stage * stage_floats;
-        if (e0 < tl.len) {
-            const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-            const int64_t off = tl.start + e0;
-            if (T::kStageX) {
-                // z_j = fma(eta, y_j - x_j, x_j), in place over the sent rows
-                for (int j = 0; j < n; ++j) {
-                    float4 *yr = reinterpret_cast<float4 *>(st + static_cast<size_t>(j) * TILE + e0);
-                    const float4 xr =
-                        *reinterpret_cast<const float4 *>(st + static_cast<size_t>(n + j) * TILE + e0);
-                    float4 z = *yr;
-                    z.x = __fmaf_rn(a.eta, __fsub_rn(z.x, xr.x), xr.x);
-                    z.y = __fmaf_rn(a.eta, __fsub_rn(z.y, xr.y), xr.y);
-                    z.z = __fmaf_rn(a.eta, __fsub_rn(z.z, xr.z), xr.z);
-                    z.w = __fmaf_rn(a.eta, __fsub_rn(z.w, xr.w), xr.w);
-                    *yr = z;
-                }
+
+    if (warp == kConsumers / 32) {
+        // ------------------------------------------------------ producer ---
+        // The whole warp moves the data, lane j the rows of worker j: waits
+        // and abort decisions are warp-uniform (__all_sync / __any_sync).
+        auto row = [&](float *st, int kind, int j) { return st + (static_cast<size_t>(kind) * n + j) * TILE; };
+        auto store_tile = [&](int64_t j) {   // this lane's rows of tile j
+            const Tile tl = a.tiles[first + j * gstride];
+            const TensorDesc &d = a.tens[tl.tensor];
+            const uint32_t bytes = static_cast<uint32_t>(((tl.len + 3) & ~3) * 4);
+            float *st = stages + (j % S) * stage_floats;
+            for (int i = lane; i < n; i += 32) {
+                bulk_s2g(d.x + i * d.wstride + tl.start, row(st, 1, i), bytes);
+                if (R::kHasB) bulk_s2g(d.b + i * d.wstride + tl.start, row(st, 2, i), bytes);
             }
-            float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f}, sh[4] = {0.f, 0.f, 0.f, 0.f};
-            constexpr int U = 4;
-            for (int i0 = 0; i0 < n; i0 += U) {
-                float4 X[U], B[U], Y[U];
-#pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    const int i = i0 + u;
-                    if (i < n) {
-                        const int64_t o = i * d.wstride + off;
-                        if (T::kLoadX) X[u] = ptx::ld_stream(d.x + o);
-                        if (T::kLoadB) B[u] = ptx::ld_stream(d.b + o);
-                        if (T::kLoadY && ((a.fresh_mask >> i) & 1u)) Y[u] = ptx::ld_stream(d.y + o);
-                    }
+            bulk_commit();
+        };
+        auto wait_all_lanes = [&](uint64_t *bar, int64_t j) {
+            const bool ok = ptx::mbar_wait_bounded(bar, static_cast<uint32_t>((j / S) & 1), kWaitLimitNs);
+            return __all_sync(0xffffffffu, ok);
+        };
+        int64_t issued = 0;
+        bool aborted = false;
+        for (int64_t it = 0; it < my_n; ++it) {
+            const int s = static_cast<int>(it % S);
+            if (it >= S) {
+                const int64_t j = it - S;
+                if (!wait_all_lanes(&empty[s], j)) {
+                    aborted = true;
+                    break;
                 }
-#pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    const int i = i0 + u;
-                    if (i >= n) continue;
-                    // mix over N_i in ascending j
+                store_tile(j);
+                bulk_wait_read_all();   // this lane's stores have read the stage
+                __syncwarp();
+            }
+            if (__any_sync(0xffffffffu, flags[0] != 0)) {
+                aborted = true;
+                break;
+            }
+            const Tile tl = a.tiles[first + it * gstride];
+            const TensorDesc &d = a.tens[tl.tensor];
+            const uint32_t bytes = static_cast<uint32_t>(((tl.len + 3) & ~3) * 4);
+            float *st = stages + s * stage_floats;
+            if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], bytes * static_cast<uint32_t>(R::kRows * n));
+            __syncwarp();
+            for (int j = lane; j < n; j += 32) {
+                const int64_t o = j * d.wstride + tl.start;
+                const bool fresh = (a.fresh_mask >> j) & 1u;
+                const float *mixed = R::kMixX ? d.x : (fresh ? d.y : d.x);
+                ptx::bulk_g2s(row(st, 0, j), mixed + o, bytes, &full[s]);
+                const float *own = R::kMixX ? (fresh ? d.y : d.x) : d.x;
+                ptx::bulk_g2s(row(st, 1, j), own + o, bytes, &full[s]);
+                if (R::kHasB) ptx::bulk_g2s(row(st, 2, j), d.b + o, bytes, &full[s]);
+            }
+            issued = it + 1;
+        }
+        if (!aborted) {
+            for (int64_t j = my_n - S > 0 ? my_n - S : 0; j < my_n; ++j) {
+                if (!wait_all_lanes(&empty[j % S], j)) {
+                    aborted = true;
+                    break;
+                }
+                store_tile(j);
+            }
+        }
+        if (aborted) {
+            if (lane == 0) {
+                flags[0] = 1;
+                atomicCAS(a.err, kDevOk, kDevWaitTimeout);
+            }
+            // copies still in flight land before the CTA leaves (bounded)
+            for (int64_t j = issued - S > 0 ? issued - S : 0; j < issued; ++j)
+                ptx::mbar_wait_bounded(&full[j % S], static_cast<uint32_t>((j / S) & 1), kWaitLimitNs);
+        }
+        bulk_wait_all();   // this lane's stores complete before the CTA leaves
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------ consumers ---
+        const int g = threadIdx.x / cols;
+        const int col = threadIdx.x % cols;
+        const int e0 = 4 * col;
+        const float inv_n = static_cast<float>(1.0 / n);
+        for (int64_t it = 0; it < my_n; ++it) {
+            const int s = static_cast<int>(it % S);
+            bool ok = !flags[0];
+            if (ok && !ptx::mbar_wait_bounded(&full[s], static_cast<uint32_t>((it / S) & 1), kWaitLimitNs)) {
+                ok = false;
+                flags[0] = 1;
+                atomicCAS(a.err, kDevOk, kDevWaitTimeout);
+            }
+            const int tlen = a.tiles[first + it * gstride].len;
+            float *st = stages + s * stage_floats;
+            float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f};
+            const bool active = ok && e0 < tlen;
+            const int nvalid = tlen - e0 < 4 ? tlen - e0 : 4;
+            float4 xr[8], br[8];                      // Eq. 2 results, written after a barrier
+            if (active) {
+                // shift of the consensus-error sums: worker 0's new x when one
+                // thread sees every worker of the column (G = 1), else worker
+                // 0's sent value, which every group can read
+                const float4 shift = ld4(st + e0);
+                float sh[4] = {shift.x, shift.y, shift.z, shift.w};
+                int nr = 0;
+                for (int i = g; i < n; i += G) {
                     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
                     const int dg = tp->deg[i];
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
                         const float w = tp->w[i][q];
-                        const float4 sj =
-                            *reinterpret_cast<const float4 *>(st + static_cast<size_t>(j) * TILE + e0);
+                        float4 sj = ld4(st + static_cast<size_t>(j) * TILE + e0);
+                        if (MODE == kOutEq2) {
+                            const float4 xj = ld4(st + (static_cast<size_t>(n) + j) * TILE + e0);
+                            sj.x = __fmaf_rn(a.eta, __fsub_rn(sj.x, xj.x), xj.x);
+                            sj.y = __fmaf_rn(a.eta, __fsub_rn(sj.y, xj.y), xj.y);
+                            sj.z = __fmaf_rn(a.eta, __fsub_rn(sj.z, xj.z), xj.z);
+                            sj.w = __fmaf_rn(a.eta, __fsub_rn(sj.w, xj.w), xj.w);
+                        }
                         acc.x = __fmaf_rn(w, sj.x, acc.x);
                         acc.y = __fmaf_rn(w, sj.y, acc.y);
                         acc.z = __fmaf_rn(w, sj.z, acc.z);
                         acc.w = __fmaf_rn(w, sj.w, acc.w);
                     }
-                    float4 xo;
-                    if (T::kLoadX) {
-                        xo = X[u];
-                    } else if (T::kStageX) {
-                        xo = *reinterpret_cast<const float4 *>(st + static_cast<size_t>(n + i) * TILE + e0);
-                    } else {   // DAdam modes: the staged (mixed) rows are x
-                        xo = *reinterpret_cast<const float4 *>(st + static_cast<size_t>(i) * TILE + e0);
-                    }
-                    float4 yo = xo;
-                    if (T::kLoadY && ((a.fresh_mask >> i) & 1u)) yo = Y[u];
-                    float4 zo = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (T::kStageX)
-                        zo = *reinterpret_cast<const float4 *>(st + static_cast<size_t>(i) * TILE + e0);
-                    float4 bo = T::kLoadB ? B[u] : make_float4(0.f, 0.f, 0.f, 0.f);
-                    float4 zp = bo;
-                    if (T::kStageX && a.first_round) zp = zo;
-                    float4 xn;
-                    xn.x = outer_update<MODE>(acc.x, xo.x, yo.x, bo.x, zo.x, zp.x, a);
-                    xn.y = outer_update<MODE>(acc.y, xo.y, yo.y, bo.y, zo.y, zp.y, a);
-                    xn.z = outer_update<MODE>(acc.z, xo.z, yo.z, bo.z, zo.z, zp.z, a);
-                    xn.w = outer_update<MODE>(acc.w, xo.w, yo.w, bo.w, zo.w, zp.w, a);
-                    const int64_t o = i * d.wstride + off;
-                    if (nvalid == 4) {
-                        ptx::st_stream(d.x + o, xn);
-                        if (T::kWriteB) ptx::st_stream(d.b + o, bo);
+                    float *p0 = st + static_cast<size_t>(i) * TILE + e0;            // mixed row i
+                    float *p1 = st + (static_cast<size_t>(n) + i) * TILE + e0;      // own x (or y)
+                    float *p2 = st + (static_cast<size_t>(2 * n) + i) * TILE + e0;  // own b
+                    float4 xo, yo, zo = make_float4(0.f, 0.f, 0.f, 0.f), bo = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (R::kMixX) {
+                        xo = ld4(p0);
+                        yo = ld4(p1);
                     } else {
-                        for (int l = 0; l < nvalid; ++l) {
-                            d.x[o + l] = lane_of(xn, l);
-                            if (T::kWriteB) d.b[o + l] = lane_of(bo, l);
-                        }
+                        xo = ld4(p1);
+                        yo = xo;
                     }
-                    // consensus-error column sums, shifted by worker 0's new value
-                    const float xa[4] = {xn.x, xn.y, xn.z, xn.w};
+                    if (R::kHasB) bo = ld4(p2);
+                    if (MODE == kOutEq2) {
+                        const float4 y0 = ld4(p0);
+                        zo.x = __fmaf_rn(a.eta, __fsub_rn(y0.x, xo.x), xo.x);
+                        zo.y = __fmaf_rn(a.eta, __fsub_rn(y0.y, xo.y), xo.y);
+                        zo.z = __fmaf_rn(a.eta, __fsub_rn(y0.z, xo.z), xo.z);
+                        zo.w = __fmaf_rn(a.eta, __fsub_rn(y0.w, xo.w), xo.w);
+                    }
+                    const float4 zp = (MODE == kOutEq2 && a.first_round) ? zo : bo;
+                    const float xa[4] = {xo.x, xo.y, xo.z, xo.w}, ya[4] = {yo.x, yo.y, yo.z, yo.w};
+                    const float za[4] = {zo.x, zo.y, zo.z, zo.w}, zpa[4] = {zp.x, zp.y, zp.z, zp.w};
+                    const float aa[4] = {acc.x, acc.y, acc.z, acc.w};
+                    float ba[4] = {bo.x, bo.y, bo.z, bo.w};
+                    float xn[4];
 #pragma unroll
                     for (int l = 0; l < 4; ++l) {
-                        if (i == 0) sh[l] = xa[l];
-                        const float dv = __fsub_rn(xa[l], sh[l]);
-                        s1[l] = __fadd_rn(s1[l], dv);
-                        s2[l] = __fmaf_rn(dv, dv, s2[l]);
+                        if (l < nvalid) {
+                            xn[l] = outer_update<MODE>(aa[l], xa[l], ya[l], ba[l], za[l], zpa[l], a);
+                            if (G == 1 && i == 0) sh[l] = xn[l];
+                            const float dv = __fsub_rn(xn[l], sh[l]);
+                            s1[l] = __fadd_rn(s1[l], dv);
+                            s2[l] = __fmaf_rn(dv, dv, s2[l]);
+                        } else {   // padding keeps its value
+                            xn[l] = R::kMixX ? ya[l] : xa[l];
+                        }
+                    }
+                    const float4 xn4 = make_float4(xn[0], xn[1], xn[2], xn[3]);
+                    const float4 bn4 = make_float4(ba[0], ba[1], ba[2], ba[3]);
+                    if (MODE == kOutEq2) {
+                        xr[nr] = xn4;
+                        br[nr] = bn4;
+                        ++nr;
+                    } else {
+                        st4(p1, xn4);   // own row: read by this thread only
+                        if (R::kHasB) st4(p2, bn4);
                     }
                 }
             }
-            float e = 0.f;
+            if (MODE == kOutEq2) {
+                // Other threads read x_j to form z_j, so the new rows are written
+                // only after every consumer has finished reading.  One barrier
+                // site, reached by every consumer thread on every tile.
+                consumer_barrier();
+                if (active) {
+                    int r = 0;
+                    for (int i = g; i < n; i += G, ++r) {
+                        st4(st + (static_cast<size_t>(n) + i) * TILE + e0, xr[r]);
+                        st4(st + (static_cast<size_t>(2 * n) + i) * TILE + e0, br[r]);
+                    }
+                }
+            }
+            // consensus-error terms of the column
+            if (G == 1) {
+                if (active) {
+                    float e = 0.f;
 #pragma unroll
-            for (int l = 0; l < 4; ++l)
-                if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
-            ce_acc += static_cast<double>(e);
-        }
-        __syncthreads();   // every thread is done with this stage
-        if (threadIdx.x == 0 && it + S < my_n) {
-            ptx::fence_proxy_async_smem();
-            issue(it + S);
+                    for (int l = 0; l < 4; ++l)
+                        if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
+                    ce_acc += static_cast<double>(e);
+                }
+            } else {
+                float4 *buf = cebuf + (it & 1) * (2 * kConsumers);
+                buf[2 * threadIdx.x] = make_float4(s1[0], s1[1], s1[2], s1[3]);
+                buf[2 * threadIdx.x + 1] = make_float4(s2[0], s2[1], s2[2], s2[3]);
+                consumer_barrier();
+                if (g == 0 && active) {
+                    float t1[4] = {s1[0], s1[1], s1[2], s1[3]}, t2[4] = {s2[0], s2[1], s2[2], s2[3]};
+                    for (int gg = 1; gg < G; ++gg) {
+                        const float4 u1 = buf[2 * (gg * cols + col)], u2 = buf[2 * (gg * cols + col) + 1];
+                        t1[0] = __fadd_rn(t1[0], u1.x); t1[1] = __fadd_rn(t1[1], u1.y);
+                        t1[2] = __fadd_rn(t1[2], u1.z); t1[3] = __fadd_rn(t1[3], u1.w);
+                        t2[0] = __fadd_rn(t2[0], u2.x); t2[1] = __fadd_rn(t2[1], u2.y);
+                        t2[2] = __fadd_rn(t2[2], u2.z); t2[3] = __fadd_rn(t2[3], u2.w);
+                    }
+                    float e = 0.f;
+#pragma unroll
+                    for (int l = 0; l < 4; ++l)
+                        if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(t1[l], inv_n), t1[l], t2[l]));
+                    ce_acc += static_cast<double>(e);
+                }
+            }
+            ptx::fence_proxy_async_smem();   // outputs visible to the bulk stores
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
         }
     }
 
-    if (aborted) {
-        if (threadIdx.x == 0) {
-            atomicCAS(a.err, kDevOk, kDevWaitTimeout);
-            // drain the copies this CTA still has in flight (bounded)
-            for (int64_t j = it; j < my_n && j < it + S; ++j)
-                ptx::mbar_wait_bounded(&bars[j % S], static_cast<uint32_t>((j / S) & 1), kWaitLimitNs);
-        }
-        ce_acc = __longlong_as_double(0x7ff8000000000000ll);   // NaN partial
-    }
-
+    if (flags[0]) ce_acc = __longlong_as_double(0x7ff8000000000000ll);   // NaN partial
     // block reduction: warp shuffles, then warps in order
     for (int o = 16; o > 0; o >>= 1) ce_acc += __shfl_down_sync(0xffffffffu, ce_acc, o);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (lane == 0) red[warp] = ce_acc;
     __syncthreads();
     if (threadIdx.x == 0) {
         double s = 0.0;
-        for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
+        for (int w = 0; w < kThreads / 32; ++w) s += red[w];
         a.partials[blockIdx.x] = s;
         __threadfence();
         const unsigned t = atomicAdd(a.ticket, 1u);
-        *flag = (t == gridDim.x - 1) ? 1 : 0;
+        flags[1] = (t == gridDim.x - 1) ? 1 : 0;
     }
     __syncthreads();
-    if (*flag && warp == 0) {
+    if (flags[1] && warp == 0) {
         __threadfence();
         double s = 0.0;
         for (unsigned b = lane; b < gridDim.x; b += 32) s += __ldcg(a.partials + b);
@@ -322,11 +429,21 @@ void *mode_kernel(int mode) {
     }
 }
 
+int mode_rows(int mode) { return (mode == kOutSgd || mode == kOutDadam) ? 2 : 3; }
+
 }  // namespace
 
-size_t gossip_smem_bytes(int n, int tile, int stages, int mode) {
-    const int rows = mode == kOutEq2 ? 2 * n : n;
-    return kOffStages + static_cast<size_t>(stages) * rows * tile * sizeof(float);
+GossipShape gossip_shape(int n, int mode) {
+    GossipShape sh{};
+    sh.groups = n <= 8 ? 1 : (n <= 16 ? 2 : 4);
+    sh.tile = 4 * (kConsumers / sh.groups);
+    sh.block = kThreads;
+    const size_t stage = static_cast<size_t>(mode_rows(mode)) * n * sh.tile * sizeof(float);
+    const size_t budget = 232448 - kOffStages;
+    int st = static_cast<int>(budget / stage);
+    sh.stages = st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
+    sh.smem = kOffStages + sh.stages * stage;
+    return sh;
 }
 
 cudaError_t gossip_set_smem(size_t smem) {
@@ -338,23 +455,24 @@ cudaError_t gossip_set_smem(size_t smem) {
     return cudaSuccess;
 }
 
-int gossip_blocks_per_sm(int block, size_t smem) {
+int gossip_blocks_per_sm(int mode, size_t smem) {
     int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, gossip_kernel<kOutNesterov>, block, smem) !=
-        cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, reinterpret_cast<const void *>(mode_kernel(mode)),
+                                                      kThreads, smem) != cudaSuccess)
         return 1;
     return nb > 0 ? nb : 1;
 }
 
-cudaError_t launch_gossip(const GossipArgs &a, int grid, int block, size_t smem, cudaStream_t s) {
-    if (a.stages < 1 || a.stages > kMaxStages) return cudaErrorInvalidValue;
+cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
+    if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups))
+        return cudaErrorInvalidValue;
     switch (a.mode) {
-    case kOutSgd: gossip_kernel<kOutSgd><<<grid, block, smem, s>>>(a); break;
-    case kOutSgdm: gossip_kernel<kOutSgdm><<<grid, block, smem, s>>>(a); break;
-    case kOutNesterov: gossip_kernel<kOutNesterov><<<grid, block, smem, s>>>(a); break;
-    case kOutEq2: gossip_kernel<kOutEq2><<<grid, block, smem, s>>>(a); break;
-    case kOutDadam: gossip_kernel<kOutDadam><<<grid, block, smem, s>>>(a); break;
-    default: gossip_kernel<kOutLocalDadam><<<grid, block, smem, s>>>(a); break;
+    case kOutSgd: gossip_kernel<kOutSgd><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutSgdm: gossip_kernel<kOutSgdm><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutNesterov: gossip_kernel<kOutNesterov><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutEq2: gossip_kernel<kOutEq2><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutDadam: gossip_kernel<kOutDadam><<<grid, kThreads, smem, s>>>(a); break;
+    default: gossip_kernel<kOutLocalDadam><<<grid, kThreads, smem, s>>>(a); break;
     }
     return cudaGetLastError();
 }

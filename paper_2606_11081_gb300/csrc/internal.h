@@ -83,7 +83,8 @@ struct GossipArgs {
     int32_t mode;          // GASLOC_OUTER_*
     uint32_t fresh_mask;   // bit j: worker j took a local step this round
     int32_t first_round;   // Eq. 2: no momentum term at t = 0
-    int32_t tile;          // elements per tile (4 * blockDim)
+    int32_t tile;          // elements per tile (4 x 256 / groups)
+    int32_t groups;        // consumer threads per 16-byte column
     int32_t stages;
     float eta_out, mu, eta, alpha, oma, gamma;
     double *partials;      // [gridDim] per-CTA consensus-error partials
@@ -106,7 +107,14 @@ struct CeArgs {
 cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s);
 cudaError_t launch_topo(const TopoSpec &spec, int64_t round, Topo *out, cudaStream_t s);
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s);
-cudaError_t launch_gossip(const GossipArgs &a, int grid, int block, size_t smem, cudaStream_t s);
+cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream_t s);
+
+// Launch shape of the gossip kernel for n workers and an outer mode.
+struct GossipShape {
+    int groups, tile, block, stages;
+    size_t smem;
+};
+GossipShape gossip_shape(int n, int mode);
 cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s);
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
                            int32_t n_workers, float *dst, int grid, cudaStream_t s);
@@ -115,11 +123,10 @@ cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, 
                           cudaStream_t s);
 
 // Occupancy-derived persistent grid sizes.
-int adamw_blocks_per_sm(int block);
-int gossip_blocks_per_sm(int block, size_t smem);
+int adamw_blocks_per_sm(int block, bool per_worker_h);
+int gossip_blocks_per_sm(int mode, size_t smem);
 int ce_blocks_per_sm(int block);
 cudaError_t gossip_set_smem(size_t smem);
-size_t gossip_smem_bytes(int n, int tile, int stages, int mode);
 
 // Sets the thread-local message returned by gasloc_last_error().
 void set_last_error(const char *msg);

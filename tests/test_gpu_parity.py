@@ -183,7 +183,9 @@ def test_consensus_error_closed_form_and_paths():
         ctx.local_steps(1)
         ctx.gossip_round()
         fused = ctx.consensus_error()
-        assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-12)
+        # the fused and the standalone reductions shift each column by different
+        # replicas (sent value vs new x of worker 0): equal to fp32 rounding
+        assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-6)
 
 
 # ------------------------------------------------------ layout / resume ---
