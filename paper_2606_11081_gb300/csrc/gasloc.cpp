@@ -4,6 +4,7 @@
 // Host arithmetic that the device results depend on (bias corrections, decay,
 // the fp32 rounding of hyperparameters) is done in double and rounded once;
 // this file is compiled with -ffp-contract=off so that no a*b+c is fused.
+#include <cuda.h>   // tensor-map types only; the encoder is fetched through the runtime
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -45,6 +46,40 @@ constexpr int kMaxLocalSteps = 1024;
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+        else
+            cudaGetLastError();
+    }
+    return fn;
+}
+
+// 2-D map over one array of one tensor: [n workers][numel] fp32 with a row
+// pitch of wstride floats, boxes of [n x 256]; out-of-range elements read as
+// zero and are not written.
+bool make_map(CUtensorMap *m, float *base, int64_t numel, int64_t wstride, int32_t n) {
+    EncodeTiledFn enc = encode_tiled();
+    if (!enc) return false;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(numel), static_cast<cuuint64_t>(n)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(wstride) * 4};
+    const cuuint32_t box[2] = {256, static_cast<cuuint32_t>(n)};
+    const cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 void gasloc::set_last_error(const char *msg) { g_err = msg; }
@@ -75,6 +110,7 @@ struct gasloc_ctx {
     int grid_a = 0, grid_ce = 0;
     int grid_gm[6] = {0, 0, 0, 0, 0, 0};   // gossip grid per outer mode
     Topo *topo_d = nullptr, *topo_scratch = nullptr;
+    void *maps_d = nullptr;   // [tensor][x, y, b] CUtensorMap
     double *partials = nullptr;
     unsigned int *ticket = nullptr;
     double *ce_d = nullptr;
@@ -426,6 +462,17 @@ int gasloc_start(gasloc_ctx *c) {
     c->tens_d = static_cast<TensorDesc *>(c->dalloc(sizeof(TensorDesc) * c->tens_h.size()));
     c->tiles_a = static_cast<Tile *>(c->dalloc(sizeof(Tile) * ta.size()));
     c->tiles_g = static_cast<Tile *>(c->dalloc(sizeof(Tile) * tg.size()));
+    std::vector<CUtensorMap> maps(c->tens_h.size() * 3);
+    for (size_t t = 0; t < c->tens_h.size(); ++t) {
+        const TensorDesc &d = c->tens_h[t];
+        float *arrs[3] = {d.x, d.y, d.b};
+        for (int k = 0; k < 3; ++k)
+            if (!make_map(&maps[t * 3 + k], arrs[k], d.numel, d.wstride, n)) {
+                c->release_all();
+                return fail(GASLOC_ECUDA, "cuTensorMapEncodeTiled failed for tensor %zu", t);
+            }
+    }
+    c->maps_d = c->dalloc(sizeof(CUtensorMap) * maps.size());
     c->topo_d = static_cast<Topo *>(c->dalloc(sizeof(Topo)));
     c->topo_scratch = static_cast<Topo *>(c->dalloc(sizeof(Topo)));
     const int max_grid = c->sms * 32;
@@ -433,7 +480,7 @@ int gasloc_start(gasloc_ctx *c) {
     c->ticket = static_cast<unsigned int *>(c->dalloc(sizeof(unsigned int) * 4));
     c->ce_d = static_cast<double *>(c->dalloc(sizeof(double) * 2));
     c->err_d = static_cast<int32_t *>(c->dalloc(sizeof(int32_t) * 4));
-    if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
+    if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->maps_d || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
         !c->ce_d || !c->err_d)
         return oom("tables");
     if (cudaMallocHost(&c->pinned, 64 + sizeof(Topo)) != cudaSuccess) {
@@ -441,7 +488,9 @@ int gasloc_start(gasloc_ctx *c) {
         c->pinned = nullptr;
         return oom("pinned host buffer");
     }
-    cudaError_t es[6];
+    cudaError_t es[7];
+    es[6] = cudaMemcpyAsync(c->maps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice,
+                            c->stream);
     es[0] = cudaMemcpyAsync(c->tens_d, c->tens_h.data(), sizeof(TensorDesc) * c->tens_h.size(), cudaMemcpyHostToDevice, c->stream);
     es[1] = cudaMemcpyAsync(c->tiles_a, ta.data(), sizeof(Tile) * ta.size(), cudaMemcpyHostToDevice, c->stream);
     es[2] = cudaMemcpyAsync(c->tiles_g, tg.data(), sizeof(Tile) * tg.size(), cudaMemcpyHostToDevice, c->stream);
@@ -574,6 +623,7 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     a.tiles = c->tiles_g;
     a.ntiles = c->ntiles_g;
     a.topo = c->topo_d;
+    a.maps = c->maps_d;
     a.n_workers = c->n;
     a.mode = hp.outer_mode;
     a.fresh_mask = c->fresh_mask;

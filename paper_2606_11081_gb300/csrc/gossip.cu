@@ -59,6 +59,7 @@ constexpr size_t kOffStages = kOffCe + kCeBytes;     // 25088, 128-byte aligned
 static_assert(kOffFlags + 16 <= kOffCe, "smem layout");
 static_assert(kOffStages % 128 == 0, "stage alignment");
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr int kBox = 256;                            // elements per TMA box row
 
 // Rows staged per worker: kind 0 = the mixed quantity, kind 1 = own x (own y
 // for the DAdam modes), kind 2 = own b.
@@ -105,23 +106,34 @@ __device__ __forceinline__ float outer_update(float acc, float x, float y, float
 
 __device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
 __device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
-__device__ __forceinline__ float lane_of(const float4 &v, int l) {
-    return l == 0 ? v.x : (l == 1 ? v.y : (l == 2 ? v.z : v.w));
-}
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
-}
-__device__ __forceinline__ void bulk_s2g(void *dst_gmem, const void *src_smem, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst_gmem),
-                 "r"(ptx::smem_addr(src_smem)), "r"(bytes)
-                 : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read_all() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// 2-D tensor copies through a tensor map in global memory: coordinates are
+// {element, worker}; the element coordinate is a multiple of 4 (16 bytes).
+__device__ __forceinline__ void tma_load_2d(void *dst_smem, const void *tmap, int32_t c0, int32_t c1,
+                                            uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            ptx::smem_addr(dst_smem)),
+        "l"(tmap), "r"(c0), "r"(c1), "r"(ptx::smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void tma_store_2d(const void *tmap, int32_t c0, int32_t c1, const void *src_smem) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(tmap), "r"(c0),
+                 "r"(c1), "r"(ptx::smem_addr(src_smem))
+                 : "memory");
+}
+__device__ __forceinline__ void tmap_acquire(const void *tmap) {
+    asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(tmap) : "memory");
+}
+
 // Named barrier 1 over the 256 consumer threads (the producer warp never
 // takes it).  The non-aligned form: threads of a warp may arrive separately.
 __device__ __forceinline__ void consumer_barrier() {
@@ -146,6 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
     const int cols = TILE / 4;
     const int S = a.stages;
     const size_t stage_floats = static_cast<size_t>(R::kRows) * n * TILE;
+    const int NQ = TILE / kBox;   // sub-boxes per tile: kind k, sub-box q, worker j at ((k NQ + q) n + j) kBox
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     {   // neighbour table -> shared memory
@@ -170,17 +183,44 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
 
     if (warp == kConsumers / 32) {
         // ------------------------------------------------------ producer ---
-        // The whole warp moves the data, lane j the rows of worker j: waits
-        // and abort decisions are warp-uniform (__all_sync / __any_sync).
-        auto row = [&](float *st, int kind, int j) { return st + (static_cast<size_t>(kind) * n + j) * TILE; };
-        auto store_tile = [&](int64_t j) {   // this lane's rows of tile j
+        // The whole warp moves the data.  Each array of a tile is loaded as
+        // ceil(len / 256) 2-D boxes of [n workers x 256 elements] through the
+        // tensor maps (one TMA operation for all workers; elements beyond the
+        // tensor read as zero) and stored back the same way (writes beyond
+        // the tensor are dropped).  Rows whose source differs between workers
+        // (some workers took no local step this round) go as one 1-D bulk
+        // copy per worker and sub-box instead.  Waits and abort decisions are
+        // warp-uniform.
+        const uint32_t all_mask = n >= 32 ? 0xffffffffu : ((1u << n) - 1u);
+        const bool all_fresh = (a.fresh_mask & all_mask) == all_mask;
+        const bool none_fresh = (a.fresh_mask & all_mask) == 0u;
+        const bool uniform = all_fresh || none_fresh;
+        const int kvar = R::kMixX ? 1 : 0;   // the kind whose source depends on freshness
+        auto blk = [&](float *st, int k, int q) { return st + static_cast<size_t>(k * NQ + q) * n * kBox; };
+        auto tmap = [&](int tensor, int arr) {   // arr: 0 x, 1 y, 2 b
+            return static_cast<const unsigned char *>(a.maps) + (static_cast<size_t>(tensor) * 3 + arr) * 128;
+        };
+        auto arr_of = [&](int k) {   // array a box of kind k is loaded from (uniform case)
+            if (k == 2) return 2;
+            if (k == kvar) return all_fresh ? 1 : 0;
+            return 0;
+        };
+        int32_t fenced = -1;
+        auto fence_maps = [&](int tensor) {   // maps written before launch: order them for the TMA proxy
+            if (tensor == fenced) return;
+            for (int arr = 0; arr < 3; ++arr) tmap_acquire(tmap(tensor, arr));
+            fenced = tensor;
+        };
+        auto store_tile = [&](int64_t j) {   // box stores of tile j, spread over lanes
             const Tile tl = a.tiles[first + j * gstride];
-            const TensorDesc &d = a.tens[tl.tensor];
-            const uint32_t bytes = static_cast<uint32_t>(((tl.len + 3) & ~3) * 4);
+            const int nq = (tl.len + kBox - 1) / kBox;
             float *st = stages + (j % S) * stage_floats;
-            for (int i = lane; i < n; i += 32) {
-                bulk_s2g(d.x + i * d.wstride + tl.start, row(st, 1, i), bytes);
-                if (R::kHasB) bulk_s2g(d.b + i * d.wstride + tl.start, row(st, 2, i), bytes);
+            const int nops = (R::kHasB ? 2 : 1) * nq;
+            fence_maps(tl.tensor);
+            for (int o = lane; o < nops; o += 32) {
+                const int k = 1 + o / nq, q = o % nq;
+                const int arr = k == 1 ? 0 : 2;
+                tma_store_2d(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * kBox), 0, blk(st, k, q));
             }
             bulk_commit();
         };
@@ -208,18 +248,35 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
             }
             const Tile tl = a.tiles[first + it * gstride];
             const TensorDesc &d = a.tens[tl.tensor];
-            const uint32_t bytes = static_cast<uint32_t>(((tl.len + 3) & ~3) * 4);
+            const int nq = (tl.len + kBox - 1) / kBox;
+            const int lenr = (tl.len + 3) & ~3;
             float *st = stages + s * stage_floats;
-            if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], bytes * static_cast<uint32_t>(R::kRows * n));
+            fence_maps(tl.tensor);
+            // bytes this stage will receive
+            uint32_t tx = 0;
+            for (int k = 0; k < R::kRows; ++k) {
+                if (k == kvar && !uniform) tx += static_cast<uint32_t>(n) * static_cast<uint32_t>(lenr) * 4u;
+                else tx += static_cast<uint32_t>(nq) * static_cast<uint32_t>(n * kBox * 4);
+            }
+            if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], tx);
             __syncwarp();
-            for (int j = lane; j < n; j += 32) {
-                const int64_t o = j * d.wstride + tl.start;
-                const bool fresh = (a.fresh_mask >> j) & 1u;
-                const float *mixed = R::kMixX ? d.x : (fresh ? d.y : d.x);
-                ptx::bulk_g2s(row(st, 0, j), mixed + o, bytes, &full[s]);
-                const float *own = R::kMixX ? (fresh ? d.y : d.x) : d.x;
-                ptx::bulk_g2s(row(st, 1, j), own + o, bytes, &full[s]);
-                if (R::kHasB) ptx::bulk_g2s(row(st, 2, j), d.b + o, bytes, &full[s]);
+            const int nbox = R::kRows * nq;
+            for (int o = lane; o < nbox; o += 32) {
+                const int k = o / nq, q = o % nq;
+                if (k == kvar && !uniform) continue;
+                tma_load_2d(blk(st, k, q), tmap(tl.tensor, arr_of(k)), static_cast<int32_t>(tl.start + q * kBox), 0,
+                            &full[s]);
+            }
+            if (!uniform) {   // per-worker source: y if the worker is fresh, else x
+                for (int j = lane; j < n; j += 32) {
+                    const bool fresh = (a.fresh_mask >> j) & 1u;
+                    const float *src = (fresh ? d.y : d.x) + j * d.wstride + tl.start;
+                    for (int q = 0; q < nq; ++q) {
+                        const int w = lenr - q * kBox < kBox ? lenr - q * kBox : kBox;
+                        ptx::bulk_g2s(blk(st, kvar, q) + static_cast<size_t>(j) * kBox, src + q * kBox,
+                                      static_cast<uint32_t>(w) * 4u, &full[s]);
+                    }
+                }
             }
             issued = it + 1;
         }
@@ -248,6 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
         const int g = threadIdx.x / cols;
         const int col = threadIdx.x % cols;
         const int e0 = 4 * col;
+        const int qb = e0 / kBox, rb = e0 % kBox;   // sub-box of the column, offset in it
         const float inv_n = static_cast<float>(1.0 / n);
         for (int64_t it = 0; it < my_n; ++it) {
             const int s = static_cast<int>(it % S);
@@ -259,6 +317,10 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
             }
             const int tlen = a.tiles[first + it * gstride].len;
             float *st = stages + s * stage_floats;
+            // row of worker j, kind k, at this thread's column
+            auto cp = [&](int k, int j) {
+                return st + (static_cast<size_t>(k) * NQ + qb) * n * kBox + static_cast<size_t>(j) * kBox + rb;
+            };
             float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f};
             const bool active = ok && e0 < tlen;
             const int nvalid = tlen - e0 < 4 ? tlen - e0 : 4;
@@ -267,7 +329,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                 // shift of the consensus-error sums: worker 0's new x when one
                 // thread sees every worker of the column (G = 1), else worker
                 // 0's sent value, which every group can read
-                const float4 shift = ld4(st + e0);
+                const float4 shift = ld4(cp(0, 0));
                 float sh[4] = {shift.x, shift.y, shift.z, shift.w};
                 int nr = 0;
                 for (int i = g; i < n; i += G) {
@@ -276,9 +338,9 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
                         const float w = tp->w[i][q];
-                        float4 sj = ld4(st + static_cast<size_t>(j) * TILE + e0);
+                        float4 sj = ld4(cp(0, j));
                         if (MODE == kOutEq2) {
-                            const float4 xj = ld4(st + (static_cast<size_t>(n) + j) * TILE + e0);
+                            const float4 xj = ld4(cp(1, j));
                             sj.x = __fmaf_rn(a.eta, __fsub_rn(sj.x, xj.x), xj.x);
                             sj.y = __fmaf_rn(a.eta, __fsub_rn(sj.y, xj.y), xj.y);
                             sj.z = __fmaf_rn(a.eta, __fsub_rn(sj.z, xj.z), xj.z);
@@ -289,9 +351,9 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                         acc.z = __fmaf_rn(w, sj.z, acc.z);
                         acc.w = __fmaf_rn(w, sj.w, acc.w);
                     }
-                    float *p0 = st + static_cast<size_t>(i) * TILE + e0;            // mixed row i
-                    float *p1 = st + (static_cast<size_t>(n) + i) * TILE + e0;      // own x (or y)
-                    float *p2 = st + (static_cast<size_t>(2 * n) + i) * TILE + e0;  // own b
+                    float *p0 = cp(0, i);   // mixed row i
+                    float *p1 = cp(1, i);   // own x (own y in the DAdam modes)
+                    float *p2 = cp(2, i);   // own b
                     float4 xo, yo, zo = make_float4(0.f, 0.f, 0.f, 0.f), bo = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (R::kMixX) {
                         xo = ld4(p0);
@@ -346,8 +408,8 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                 if (active) {
                     int r = 0;
                     for (int i = g; i < n; i += G, ++r) {
-                        st4(st + (static_cast<size_t>(n) + i) * TILE + e0, xr[r]);
-                        st4(st + (static_cast<size_t>(2 * n) + i) * TILE + e0, br[r]);
+                        st4(cp(1, i), xr[r]);
+                        st4(cp(2, i), br[r]);
                     }
                 }
             }
@@ -464,7 +526,8 @@ int gossip_blocks_per_sm(int mode, size_t smem) {
 }
 
 cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
-    if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups))
+    if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups) ||
+        a.tile % kBox != 0 || a.maps == nullptr)
         return cudaErrorInvalidValue;
     switch (a.mode) {
     case kOutSgd: gossip_kernel<kOutSgd><<<grid, kThreads, smem, s>>>(a); break;

@@ -79,6 +79,7 @@ struct GossipArgs {
     const Tile *tiles;
     int64_t ntiles;
     const Topo *topo;
+    const void *maps;      // per tensor: 2-D tensor maps of x, y, b (128 bytes each)
     int32_t n_workers;
     int32_t mode;          // GASLOC_OUTER_*
     uint32_t fresh_mask;   // bit j: worker j took a local step this round
