@@ -139,6 +139,21 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def aggregate(ms_local: float, units_local: float, dist_mod=None, device=None):
+    """Whole-job timing for independent replicas (one per GPU): the job's time
+    is the slowest rank's timed region and its throughput is the units all
+    ranks processed over that time.  Returns (ms_max, units_per_second)."""
+    if dist_mod is None:
+        return ms_local, units_local / (ms_local / 1e3)
+    import torch
+    t_max = torch.tensor([ms_local], dtype=torch.float64, device=device)
+    t_sum = torch.tensor([units_local], dtype=torch.float64, device=device)
+    dist_mod.all_reduce(t_max, op=dist_mod.ReduceOp.MAX)
+    dist_mod.all_reduce(t_sum, op=dist_mod.ReduceOp.SUM)
+    ms = float(t_max.item())
+    return ms, float(t_sum.item()) / (ms / 1e3)
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -297,10 +312,9 @@ def main():
     ms = t_start.elapsed_time(t_end)
     local_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(K))
     gossip_ms = sum(ev[k][1].elapsed_time(ev[k][2]) for k in range(K))
+    units = float(w.n_workers) * w.n_params * K
+    ms, value = aggregate(ms, units, pg, torch.device("cuda", local) if pg else None)
     if pg:
-        t = torch.tensor([ms], device="cuda")
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms = float(t.item())
         pg.barrier()
     ce = ctx.consensus_error()
 
@@ -321,7 +335,6 @@ def main():
     dom_gbs = adamw_gbs if dom == "adamw" else gossip_gbs
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
     traffic = kernel_traffic(dom, w.name)
-    value = N * P * K / (ms / 1e3) * world
 
     e2e = None
     if not args.no_e2e:
@@ -384,18 +397,22 @@ def measure_e2e(g, torch, w, hp, H, K):
         g.gasloc_write_ptr(ctx.h, "c", i, cs[i].data_ptr())
     for i in range(nh):
         g.gasloc_write_ptr(ctx.h, "h", i, hs[i].data_ptr())
+    t1 = time.perf_counter()
     ces = []
     for _ in range(K):
         ctx.local_steps(H)
         ctx.gossip_round()
         ces.append(ctx.consensus_error())
+    t2 = time.perf_counter()
     g.gasloc_average_host(ctx.h, out.numpy())
     el = time.perf_counter() - t0
+    t3 = el - (t2 - t0)
     ctx.close()
     h2d = (P + N * P + nh * P) * 4
     d2h = 8 * K + 4 * P
     return {"value": N * P * K / el, "unit": UNIT, "h2d_bytes_per_step": h2d / K,
             "d2h_bytes_per_step": d2h / K, "seconds": el,
+            "upload_s": t1 - t0, "rounds_s": t2 - t1, "download_s": t3,
             "note": "initial replicas, centres and curvature uploaded once per run (amortised); "
                     "consensus error read every round; average read at the end"}
 

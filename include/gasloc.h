@@ -237,6 +237,17 @@ int gasloc_steps_taken(const gasloc_ctx *ctx, int32_t worker, int64_t *steps);
 int gasloc_save(gasloc_ctx *ctx, const char *path);
 int gasloc_load(gasloc_ctx *ctx, const char *path);
 
+/* Failure detection self-test.  Every wait the pipeline kernels make on an
+ * mbarrier is bounded: on expiry the kernel records a device error, finishes
+ * its in-flight copies and returns, and the next synchronising call reports
+ * GASLOC_EDEVICE and clears the flag.  This call runs that exact wait routine
+ * on a barrier nothing completes, with a limit of limit_ns (1 ns .. 2 s), so
+ * the expected result is GASLOC_EDEVICE; the context stays usable afterwards.
+ * (The paper argues that sparse exchanges tolerate failures that are skipped,
+ * Sec. 3.2 "Fault tolerance"; detecting a stalled exchange is this library's
+ * side of that.)  Synchronising. */
+int gasloc_selftest_bounded_wait(gasloc_ctx *ctx, int64_t limit_ns);
+
 /* Launch counter of the library's kernels on this context (for accounting). */
 int gasloc_launch_count(const gasloc_ctx *ctx, int64_t *count);
 

@@ -82,6 +82,7 @@ SIGNATURES = {
     "gasloc_save": (ctypes.c_int, [_P, ctypes.c_char_p]),
     "gasloc_load": (ctypes.c_int, [_P, ctypes.c_char_p]),
     "gasloc_launch_count": (ctypes.c_int, [_P, _I64P]),
+    "gasloc_selftest_bounded_wait": (ctypes.c_int, [_P, _I64]),
     "gasloc_last_error": (ctypes.c_char_p, []),
     "gasloc_destroy": (None, [_P]),
 }
@@ -279,6 +280,12 @@ def gasloc_launch_count(ctx) -> int:
     r = ctypes.c_int64()
     _check(_lib.gasloc_launch_count(ctx, ctypes.byref(r)))
     return r.value
+
+
+def gasloc_selftest_bounded_wait(ctx, limit_ns: int) -> int:
+    """Runs the bounded-wait self-test; returns the status code (EDEVICE is
+    the expected outcome: the wait expired and was reported)."""
+    return _lib.gasloc_selftest_bounded_wait(ctx, limit_ns)
 
 
 def gasloc_last_error() -> str:

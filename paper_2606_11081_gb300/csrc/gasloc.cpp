@@ -823,6 +823,16 @@ int gasloc_steps_taken(const gasloc_ctx *c, int32_t worker, int64_t *steps) {
     return GASLOC_OK;
 }
 
+int gasloc_selftest_bounded_wait(gasloc_ctx *c, int64_t limit_ns) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (limit_ns < 1 || limit_ns > 2000000000LL) return fail(GASLOC_EINVAL, "limit_ns must be in [1, 2e9]");
+    rc = launch_checked(c, launch_wait_selftest(static_cast<uint64_t>(limit_ns), c->err_d, c->stream),
+                        "bounded-wait self-test kernel");
+    if (rc) return rc;
+    return sync_and_check(c);
+}
+
 int gasloc_launch_count(const gasloc_ctx *c, int64_t *count) {
     if (!c || !count) return fail(GASLOC_EINVAL, "NULL argument");
     *count = c->launches;

@@ -123,6 +123,8 @@ cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, 
                           const int64_t *idx, int64_t n, float *out, int32_t *err,
                           cudaStream_t s);
 
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s);
+
 // Occupancy-derived persistent grid sizes.
 int adamw_blocks_per_sm(int block, bool per_worker_h);
 int gossip_blocks_per_sm(int mode, size_t smem);

@@ -222,7 +222,26 @@ __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t whi
     out[q] = base[worker * stride + off];
 }
 
+// A wait on an mbarrier that nothing ever completes, through the bounded-wait
+// routine the pipeline kernels use: it must give up after limit_ns, record
+// kDevWaitTimeout and return.
+__global__ void wait_selftest_kernel(uint64_t limit_ns, int32_t *err) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(&bar, 1);
+        ptx::fence_mbar_init();
+    }
+    __syncthreads();
+    const bool ok = ptx::mbar_wait_bounded(&bar, 0, limit_ns);
+    if (!ok && threadIdx.x == 0) atomicCAS(err, kDevOk, kDevWaitTimeout);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s) {
+    wait_selftest_kernel<<<1, 32, 0, s>>>(limit_ns, err);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s) {
     init_kernel<<<grid, 256, 0, s>>>(a);
