@@ -82,3 +82,37 @@ def test_workload_full_size_sampled(name):
         ctx.close()
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
+
+
+def test_maximum_replica_size():
+    # n_params at its limit (2^31 - 1): worker offsets exceed 2^32 floats and
+    # element coordinates reach the top of int32; checked on the last tiles.
+    import torch
+    P, N = 2 ** 31 - 1, 2
+    free, _ = torch.cuda.mem_get_info()
+    need = (6 * N + 1) * (P + 64) * 4
+    if free < need + (8 << 30):
+        pytest.skip("not enough device memory for the maximum size")
+    kidx = np.array([0, 1, 1023, 1024, 2 ** 30, 2 ** 31 - 1025, 2 ** 31 - 1024, 2 ** 31 - 257,
+                     2 ** 31 - 256, 2 ** 31 - 5, 2 ** 31 - 4, 2 ** 31 - 3, 2 ** 31 - 2], np.int64)
+    from _pairs import make_pair
+    ctx, st = make_pair(N, P, "ring", seed=91, hp=dict(lr=1e-3), kidx=kidx)
+    try:
+        for _ in range(2):
+            ctx.local_steps(2)
+            ctx.gossip_round()
+            st.local_steps(2)
+            st.gossip_round()
+        for which in ("x", "b", "m", "v", "y"):
+            for i in range(N):
+                a = ctx.gather(which, i, kidx)
+                b = st.get(which, i).astype(np.float32)
+                np.testing.assert_array_equal(a, b, err_msg="%s[%d]" % (which, i))
+        # a 2-node ring is the complete graph: both replicas receive the same mix
+        # from identical starting points, so they stay equal (exact consensus)
+        assert ctx.consensus_error() == 0.0
+        assert np.array_equal(ctx.gather("x", 0, kidx), ctx.gather("x", 1, kidx))
+    finally:
+        ctx.close()
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
