@@ -155,8 +155,8 @@ int gasloc_set_local_steps(gasloc_ctx *ctx, const int32_t *H_i);
 int gasloc_draw_local_steps(gasloc_ctx *ctx, int32_t hmax);
 int gasloc_get_local_steps(const gasloc_ctx *ctx, int32_t *H_i);
 
-/* Inner loop of Algorithm 1: H > 0 gives every worker H AdamW steps;
- * H = GASLOC_PER_WORKER_STEPS gives worker i its H_i steps.  The first step
+/* Inner loop of Algorithm 1: H > 0 gives every worker H AdamW steps (H = 0:
+ * none); H = GASLOC_PER_WORKER_STEPS gives worker i its H_i steps.  The first step
  * of a round starts from x_i; later ones from y_i.  Moments and step counters
  * persist across rounds.  Asynchronous.  ESTATE before gasloc_start. */
 int gasloc_local_steps(gasloc_ctx *ctx, int32_t H);
@@ -166,6 +166,18 @@ int gasloc_local_steps(gasloc_ctx *ctx, int32_t H);
  * applies the outer update and reduces the consensus error of the new x.
  * A worker that took no local step this round sends x_i.  Asynchronous. */
 int gasloc_gossip_round(gasloc_ctx *ctx);
+
+/* Runs `rounds` complete outer rounds -- H local steps (H > 0, or
+ * GASLOC_PER_WORKER_STEPS for each worker's H_i, or 0) followed by a gossip
+ * round -- exactly as that many gasloc_local_steps + gasloc_gossip_round
+ * calls would, but replayed from a CUDA graph of one round that is captured
+ * on the first call and reused until the hyperparameters, H or the H_i
+ * change.  Every per-step scalar is derived on the device from device-resident
+ * step counters, so the replayed rounds need no host work.  Must start at a
+ * round boundary (ESTATE otherwise).  If ce_trace_host is not NULL it
+ * receives the consensus error of each round (rounds <= 4096) and the call
+ * synchronises; otherwise it is asynchronous. */
+int gasloc_run(gasloc_ctx *ctx, int32_t rounds, int32_t H, double *ce_trace_host);
 
 /* Consensus error CE = (1/n) sum_i sum_k (x_ik - xbar_k)^2 of the current
  * replicas (||pi x||^2 / n with pi = I - 11^T/n).  Returns the value the last

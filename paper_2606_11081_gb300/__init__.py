@@ -67,6 +67,7 @@ SIGNATURES = {
     "gasloc_get_local_steps": (ctypes.c_int, [_P, _I32P]),
     "gasloc_local_steps": (ctypes.c_int, [_P, _I32]),
     "gasloc_gossip_round": (ctypes.c_int, [_P]),
+    "gasloc_run": (ctypes.c_int, [_P, _I32, _I32, _DP]),
     "gasloc_consensus_error": (ctypes.c_int, [_P, _DP]),
     "gasloc_consensus_error_now": (ctypes.c_int, [_P, _DP]),
     "gasloc_consensus_error_noalloc": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P]),
@@ -186,6 +187,17 @@ def gasloc_local_steps(ctx, H: int) -> None:
 
 def gasloc_gossip_round(ctx) -> None:
     _check(_lib.gasloc_gossip_round(ctx))
+
+
+def gasloc_run(ctx, rounds: int, H: int, trace: bool = False):
+    """`rounds` complete rounds replayed from a CUDA graph; returns the
+    per-round consensus errors when trace is set (synchronising)."""
+    if trace:
+        out = np.zeros(rounds, np.float64)
+        _check(_lib.gasloc_run(ctx, rounds, H, _arr(out, _DP)))
+        return out
+    _check(_lib.gasloc_run(ctx, rounds, H, None))
+    return None
 
 
 def gasloc_consensus_error(ctx) -> float:
@@ -378,6 +390,9 @@ class Context:
 
     def gossip_round(self) -> None:
         gasloc_gossip_round(self.h)
+
+    def run(self, rounds: int, H: int, trace: bool = False):
+        return gasloc_run(self.h, rounds, H, trace)
 
     def consensus_error(self) -> float:
         return gasloc_consensus_error(self.h)

@@ -61,6 +61,11 @@ __device__ __forceinline__ float noise_xi(uint32_t k, uint32_t klo, uint32_t khi
 template <int U, bool PER_WORKER_H>
 __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     const Consts kc{a.decay, a.beta1, a.beta2, a.omb1, a.omb2, a.eps, a.sigma};
+    // this step's per-worker scalars (written by the prep kernel) -> shared
+    __shared__ StepTable tab;
+    for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += blockDim.x)
+        reinterpret_cast<uint32_t *>(&tab)[q] = reinterpret_cast<const uint32_t *>(a.table)[q];
+    __syncthreads();
     int32_t cur = -1;
     TensorDesc d{};
     for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
@@ -96,9 +101,9 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
             for (int u = 0; u < U; ++u) {
                 if (a0 + u < a.n_active) {
                     const int i = a.worker[a0 + u];
-                    const float step = a.step[a0 + u];
-                    const float isb = a.isb[a0 + u];
-                    const uint32_t klo = a.key_lo[a0 + u], khi = a.key_hi[a0 + u];
+                    const float step = tab.step[i];
+                    const float isb = tab.isb[i];
+                    const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
                     const float4 h4 = PER_WORKER_H ? Hh[u] : hs;
                     float4 yo, mo, vo;
                     yo.x = adamw_lane(Y[u].x, M[u].x, V[u].x, C[u].x, h4.x, noise_xi(k0 + 0, klo, khi),

@@ -43,6 +43,7 @@ constexpr int64_t kMaxParams = (int64_t(1) << 31) - 1;
 constexpr int64_t kPadFloats = 64;
 constexpr int kTileA = 1024;          // init / adamw / ce / average tiles (4 x 256 threads)
 constexpr int kMaxLocalSteps = 1024;
+constexpr int kCeRing = 4096;
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -113,14 +114,21 @@ struct gasloc_ctx {
     void *maps_d = nullptr;   // [tensor][x, y, b] CUtensorMap
     double *partials = nullptr;
     unsigned int *ticket = nullptr;
-    double *ce_d = nullptr;
+    double *ce_d = nullptr;          // [0] standalone reduction result
+    double *ce_ring = nullptr;       // consensus error of round t at [t % kCeRing]
+    DevState *state_d = nullptr;     // device-resident step counters
+    StepTable *table_d = nullptr;    // scalars of the current local step
+    cudaStream_t cap_stream = nullptr;
+    cudaGraphExec_t graph = nullptr; // one round, captured by gasloc_run
+    int32_t graph_H = 0;
+    uint64_t graph_gen = 0, gen = 1; // configuration generation the graph was built for
+    int64_t graph_launches = 0;      // kernels per replayed round
     int32_t *err_d = nullptr;
     void *pinned = nullptr;   // [ce double][err int32][Topo]
     std::vector<std::pair<void *, size_t>> allocs;
 
     // counters
     std::vector<int64_t> nsteps;
-    std::vector<double> p1, p2;
     std::vector<int32_t> Hi;
     bool has_Hi = false;
     uint32_t fresh_mask = 0;
@@ -153,6 +161,10 @@ struct gasloc_ctx {
     }
     void release_all() {
         if (started || !allocs.empty()) cudaStreamSynchronize(stream);
+        if (graph) cudaGraphExecDestroy(graph);
+        graph = nullptr;
+        if (cap_stream) cudaStreamDestroy(cap_stream);
+        cap_stream = nullptr;
         for (auto &pr : allocs) {
             if (free_fn) free_fn(pr.first, stream, alloc_user);
             else cudaFree(pr.first);
@@ -256,8 +268,8 @@ int launch_checked(gasloc_ctx *c, cudaError_t e, const char *what) {
     return GASLOC_OK;
 }
 
-int build_topology(gasloc_ctx *c, int64_t round, Topo *dst) {
-    return launch_checked(c, launch_topo(c->spec, round, dst, c->stream), "topology kernel");
+int build_topology(gasloc_ctx *c, int64_t round, const int64_t *round_ptr, Topo *dst, cudaStream_t s) {
+    return launch_checked(c, launch_topo(c->spec, round, round_ptr, dst, s), "topology kernel");
 }
 
 float *buffer_base(const TensorDesc &d, int which, int64_t *stride) {
@@ -329,8 +341,6 @@ int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint6
     gasloc_default_hparams(&c->hp);
     c->numels.assign(1, n_params);
     c->nsteps.assign(n_workers, 0);
-    c->p1.assign(n_workers, 1.0);
-    c->p2.assign(n_workers, 1.0);
     c->Hi.assign(n_workers, 0);
     refresh_spec(c);
     *out = c;
@@ -344,6 +354,7 @@ int gasloc_set_hparams(gasloc_ctx *c, const gasloc_hparams *hp) {
     if (c->started && hp->per_worker_h != c->hp.per_worker_h)
         return fail(GASLOC_ESTATE, "per_worker_h cannot change after gasloc_start");
     c->hp = *hp;
+    c->gen += 1;
     refresh_spec(c);
     return GASLOC_OK;
 }
@@ -479,16 +490,22 @@ int gasloc_start(gasloc_ctx *c) {
     c->partials = static_cast<double *>(c->dalloc(sizeof(double) * max_grid));
     c->ticket = static_cast<unsigned int *>(c->dalloc(sizeof(unsigned int) * 4));
     c->ce_d = static_cast<double *>(c->dalloc(sizeof(double) * 2));
+    c->ce_ring = static_cast<double *>(c->dalloc(sizeof(double) * kCeRing));
+    c->state_d = static_cast<DevState *>(c->dalloc(sizeof(DevState)));
+    c->table_d = static_cast<StepTable *>(c->dalloc(sizeof(StepTable)));
     c->err_d = static_cast<int32_t *>(c->dalloc(sizeof(int32_t) * 4));
     if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->maps_d || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
-        !c->ce_d || !c->err_d)
+        !c->ce_d || !c->err_d || !c->ce_ring || !c->state_d || !c->table_d)
         return oom("tables");
     if (cudaMallocHost(&c->pinned, 64 + sizeof(Topo)) != cudaSuccess) {
         cudaGetLastError();
         c->pinned = nullptr;
         return oom("pinned host buffer");
     }
-    cudaError_t es[7];
+    DevState st0{};
+    for (int i = 0; i < kMaxWorkers; ++i) st0.p1[i] = st0.p2[i] = 1.0;
+    cudaError_t es[8];
+    es[7] = cudaMemcpyAsync(c->state_d, &st0, sizeof st0, cudaMemcpyHostToDevice, c->stream);
     es[6] = cudaMemcpyAsync(c->maps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice,
                             c->stream);
     es[0] = cudaMemcpyAsync(c->tens_d, c->tens_h.data(), sizeof(TensorDesc) * c->tens_h.size(), cudaMemcpyHostToDevice, c->stream);
@@ -518,8 +535,6 @@ int gasloc_start(gasloc_ctx *c) {
     c->fresh_mask = 0;
     c->ce_valid = false;
     std::fill(c->nsteps.begin(), c->nsteps.end(), 0);
-    std::fill(c->p1.begin(), c->p1.end(), 1.0);
-    std::fill(c->p2.begin(), c->p2.end(), 1.0);
     refresh_spec(c);
     return GASLOC_OK;
 }
@@ -534,6 +549,7 @@ int gasloc_set_local_steps(gasloc_ctx *c, const int32_t *H) {
         if (H[i] < 0 || H[i] > kMaxLocalSteps) return fail(GASLOC_EINVAL, "H_%d = %d out of [0, %d]", i, H[i], kMaxLocalSteps);
     c->Hi.assign(H, H + c->n);
     c->has_Hi = true;
+    c->gen += 1;
     return GASLOC_OK;
 }
 
@@ -545,6 +561,7 @@ int gasloc_draw_local_steps(gasloc_ctx *c, int32_t hmax) {
         c->Hi[i] = 1 + static_cast<int32_t>((r * static_cast<uint64_t>(hmax)) >> 32);
     }
     c->has_Hi = true;
+    c->gen += 1;
     return GASLOC_OK;
 }
 
@@ -555,14 +572,14 @@ int gasloc_get_local_steps(const gasloc_ctx *c, int32_t *H) {
     return GASLOC_OK;
 }
 
-int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
-    int rc = check_started(c);
-    if (rc) return rc;
-    if (H == 0) return GASLOC_OK;
-    if (H != GASLOC_PER_WORKER_STEPS && (H < 1 || H > kMaxLocalSteps))
-        return fail(GASLOC_EINVAL, "H must be in [1, %d] or GASLOC_PER_WORKER_STEPS", kMaxLocalSteps);
-    if (H == GASLOC_PER_WORKER_STEPS && !c->has_Hi)
-        return fail(GASLOC_ESTATE, "per-worker steps requested but none set");
+}  // extern "C"
+
+namespace {
+
+// Enqueues the local steps of one call on stream s and advances the host
+// mirrors (step counts, which workers are fresh).  Every step is a prep
+// launch (the step's scalars, from the device counters) and an AdamW launch.
+int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     const gasloc_hparams &hp = c->hp;
     int32_t hmax = H;
     if (H < 0) hmax = *std::max_element(c->Hi.begin(), c->Hi.end());
@@ -570,6 +587,7 @@ int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
     a.tens = c->tens_d;
     a.tiles = c->tiles_a;
     a.ntiles = c->ntiles_a;
+    a.table = c->table_d;
     a.per_worker_h = hp.per_worker_h;
     a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
     a.beta1 = static_cast<float>(hp.beta1);
@@ -578,42 +596,35 @@ int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
     a.omb2 = static_cast<float>(1.0 - hp.beta2);
     a.eps = static_cast<float>(hp.eps);
     a.sigma = static_cast<float>(hp.noise_sigma);
-    for (int32_t s = 0; s < hmax; ++s) {
+    PrepArgs pa{c->state_d, c->table_d, 0u, c->n, hp.lr, hp.beta1, hp.beta2, c->seed};
+    for (int32_t st = 0; st < hmax; ++st) {
         int na = 0;
+        uint32_t mask = 0;
         for (int32_t i = 0; i < c->n; ++i) {
-            if (H < 0 && s >= c->Hi[i]) continue;
-            const int64_t nstep = c->nsteps[i] + 1;
-            const double p1 = c->p1[i] * hp.beta1, p2 = c->p2[i] * hp.beta2;
-            const double bc1 = 1.0 - p1, bc2 = 1.0 - p2;
-            a.worker[na] = i;
-            a.step[na] = static_cast<float>(hp.lr / bc1);
-            a.isb[na] = static_cast<float>(1.0 / std::sqrt(bc2));
-            const uint64_t key = host_hash(c->seed, 4, static_cast<uint64_t>(i), static_cast<uint64_t>(nstep));
-            a.key_lo[na] = static_cast<uint32_t>(key);
-            a.key_hi[na] = static_cast<uint32_t>(key >> 32);
-            ++na;
+            if (H < 0 && st >= c->Hi[i]) continue;
+            a.worker[na++] = i;
+            mask |= 1u << i;
         }
         if (na == 0) continue;
+        pa.active_mask = mask;
+        int rc = launch_checked(c, launch_prep(pa, s), "step-scalar kernel");
+        if (rc) return rc;
         a.n_active = na;
         a.from_x_mask = ~c->fresh_mask;
-        rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, c->stream), "adamw kernel");
+        rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, s), "adamw kernel");
         if (rc) return rc;
-        for (int q = 0; q < na; ++q) {
-            const int i = a.worker[q];
-            c->nsteps[i] += 1;
-            c->p1[i] *= hp.beta1;
-            c->p2[i] *= hp.beta2;
-            c->fresh_mask |= 1u << i;
-        }
+        for (int q = 0; q < na; ++q) c->nsteps[a.worker[q]] += 1;
+        c->fresh_mask |= mask;
     }
     return GASLOC_OK;
 }
 
-int gasloc_gossip_round(gasloc_ctx *c) {
-    int rc = check_started(c);
-    if (rc) return rc;
+// Enqueues one gossip round (the round's table where the graph is random,
+// then the fused mixing / outer-update / consensus-error kernel) on stream s
+// and advances the host mirrors.
+int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     if (!c->topo_static || !c->topo_ready) {
-        rc = build_topology(c, c->round, c->topo_d);
+        const int rc = build_topology(c, c->round, &c->state_d->round, c->topo_d, s);
         if (rc) return rc;
         c->topo_ready = c->topo_static;
     }
@@ -627,7 +638,7 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     a.n_workers = c->n;
     a.mode = hp.outer_mode;
     a.fresh_mask = c->fresh_mask;
-    a.first_round = c->round == 0 ? 1 : 0;
+    a.state = c->state_d;
     const GossipShape gs = gossip_shape(c->n, hp.outer_mode);
     a.tile = gs.tile;
     a.groups = gs.groups;
@@ -640,9 +651,10 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     a.gamma = static_cast<float>(hp.gamma);
     a.partials = c->partials;
     a.ticket = c->ticket;
-    a.ce_out = c->ce_d;
+    a.ce_ring = c->ce_ring;
+    a.ce_ring_len = kCeRing;
     a.err = c->err_d;
-    rc = launch_checked(c, launch_gossip(a, c->grid_gm[hp.outer_mode], gs.smem, c->stream), "gossip kernel");
+    const int rc = launch_checked(c, launch_gossip(a, c->grid_gm[hp.outer_mode], gs.smem, s), "gossip kernel");
     if (rc) return rc;
     c->round += 1;
     c->fresh_mask = 0;
@@ -650,17 +662,120 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     return GASLOC_OK;
 }
 
+int check_H(const gasloc_ctx *c, int32_t H) {
+    if (H != GASLOC_PER_WORKER_STEPS && (H < 0 || H > kMaxLocalSteps))
+        return fail(GASLOC_EINVAL, "H must be in [0, %d] or GASLOC_PER_WORKER_STEPS", kMaxLocalSteps);
+    if (H == GASLOC_PER_WORKER_STEPS && !c->has_Hi) return fail(GASLOC_ESTATE, "per-worker steps requested but none set");
+    return GASLOC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    rc = check_H(c, H);
+    if (rc) return rc;
+    if (H == 0) return GASLOC_OK;
+    return enqueue_local_steps(c, H, c->stream);
+}
+
+int gasloc_gossip_round(gasloc_ctx *c) {
+    const int rc = check_started(c);
+    if (rc) return rc;
+    return enqueue_gossip(c, c->stream);
+}
+
+int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    rc = check_H(c, H);
+    if (rc) return rc;
+    if (rounds < 0) return fail(GASLOC_EINVAL, "rounds must be >= 0");
+    if (ce_trace_host && rounds > kCeRing) return fail(GASLOC_EINVAL, "a trace holds at most %d rounds", kCeRing);
+    if (c->fresh_mask != 0) return fail(GASLOC_ESTATE, "gasloc_run starts at a round boundary (after a gossip round)");
+    if (rounds == 0) return GASLOC_OK;
+    const int64_t r0 = c->round;
+    if (!c->graph || c->graph_gen != c->gen || c->graph_H != H) {
+        if (c->graph) cudaGraphExecDestroy(c->graph);
+        c->graph = nullptr;
+        if (!c->cap_stream && cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+            cudaGetLastError();
+            return fail(GASLOC_ECUDA, "creating the capture stream failed");
+        }
+        // a static neighbour table is built once, outside the graph
+        if (c->topo_static && !c->topo_ready) {
+            rc = build_topology(c, c->round, nullptr, c->topo_d, c->stream);
+            if (rc) return rc;
+            c->topo_ready = true;
+        }
+        cudaError_t e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+        // capture one round; the host mirrors are restored afterwards and
+        // advanced once per replay
+        const std::vector<int64_t> nsteps0 = c->nsteps;
+        const int64_t round0 = c->round, launches0 = c->launches;
+        const bool ce0 = c->ce_valid;
+        e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+        if (e != cudaSuccess) return cuda_fail(e, "begin capture");
+        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, c->cap_stream);
+        if (!rc) rc = enqueue_gossip(c, c->cap_stream);
+        cudaGraph_t g = nullptr;
+        const cudaError_t e2 = cudaStreamEndCapture(c->cap_stream, &g);
+        c->graph_launches = c->launches - launches0;
+        c->nsteps = nsteps0;
+        c->round = round0;
+        c->launches = launches0;
+        c->ce_valid = ce0;
+        c->fresh_mask = 0;
+        if (rc) {
+            if (g) cudaGraphDestroy(g);
+            return rc;
+        }
+        if (e2 != cudaSuccess) return cuda_fail(e2, "end capture");
+        e = cudaGraphInstantiate(&c->graph, g, 0);
+        cudaGraphDestroy(g);
+        if (e != cudaSuccess) {
+            c->graph = nullptr;
+            return cuda_fail(e, "graph instantiate");
+        }
+        c->graph_gen = c->gen;
+        c->graph_H = H;
+    }
+    for (int32_t r = 0; r < rounds; ++r) {
+        const cudaError_t e = cudaGraphLaunch(c->graph, c->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+        for (int32_t i = 0; i < c->n; ++i) c->nsteps[i] += H < 0 ? c->Hi[i] : H;
+        c->round += 1;
+        c->launches += c->graph_launches;
+    }
+    c->ce_valid = true;
+    if (ce_trace_host) {
+        for (int32_t r = 0; r < rounds; ++r) {
+            const cudaError_t e = cudaMemcpyAsync(ce_trace_host + r, c->ce_ring + (r0 + r) % kCeRing, sizeof(double),
+                                                  cudaMemcpyDeviceToHost, c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "reading the consensus-error trace");
+        }
+        return sync_and_check(c);
+    }
+    return GASLOC_OK;
+}
+
 int gasloc_consensus_error(gasloc_ctx *c, double *out) {
     int rc = check_started(c);
     if (rc) return rc;
     if (!out) return fail(GASLOC_EINVAL, "out is NULL");
-    if (!c->ce_valid) {
+    const double *src = c->ce_d;
+    if (!c->ce_valid || c->round == 0) {
         CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->partials, c->ticket, c->ce_d};
         rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
         if (rc) return rc;
-        c->ce_valid = true;
+    } else {
+        src = c->ce_ring + (c->round - 1) % kCeRing;
     }
-    cudaError_t e = cudaMemcpyAsync(pin_ce(c), c->ce_d, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+    cudaError_t e = cudaMemcpyAsync(pin_ce(c), src, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "reading the consensus error");
     rc = sync_and_check(c);
     if (rc) return rc;
@@ -680,7 +795,7 @@ int gasloc_get_topology(gasloc_ctx *c, int64_t round, int32_t *nbr, float *w, in
     if (rc) return rc;
     if (!nbr || !w || !deg) return fail(GASLOC_EINVAL, "NULL output");
     if (round < 0) return fail(GASLOC_EINVAL, "round must be >= 0");
-    rc = build_topology(c, round, c->topo_scratch);
+    rc = build_topology(c, round, nullptr, c->topo_scratch, c->stream);
     if (rc) return rc;
     cudaError_t e = cudaMemcpyAsync(pin_topo(c), c->topo_scratch, sizeof(Topo), cudaMemcpyDeviceToHost, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "reading the topology");
@@ -954,12 +1069,23 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     c->has_Hi = h.has_Hi != 0;
     c->Hi = Hi;
     c->nsteps = nsteps;
-    for (int32_t i = 0; i < c->n; ++i) {
+    // device counters: beta^n by n successive products from 1, as the device does
+    DevState ds{};
+    ds.round = h.round;
+    for (int32_t i = 0; i < kMaxWorkers; ++i) {
         double a = 1.0, b = 1.0;
-        for (int64_t s = 0; s < nsteps[i]; ++s) { a *= hp.beta1; b *= hp.beta2; }
-        c->p1[i] = a;
-        c->p2[i] = b;
+        const int64_t ns = i < c->n ? nsteps[i] : 0;
+        for (int64_t t = 0; t < ns; ++t) {
+            a *= hp.beta1;
+            b *= hp.beta2;
+        }
+        ds.nsteps[i] = ns;
+        ds.p1[i] = a;
+        ds.p2[i] = b;
     }
+    if (cudaMemcpy(c->state_d, &ds, sizeof ds, cudaMemcpyHostToDevice) != cudaSuccess)
+        return fail(GASLOC_ECUDA, "restoring the step counters failed");
+    c->gen += 1;
     c->ce_valid = false;
     refresh_spec(c);
     return GASLOC_OK;

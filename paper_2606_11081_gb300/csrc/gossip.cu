@@ -180,6 +180,10 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
     const int64_t first = blockIdx.x, gstride = gridDim.x;
     const int64_t my_n = a.ntiles > first ? (a.ntiles - first + gstride - 1) / gstride : 0;
     double ce_acc = 0.0;
+    // the round being executed; every CTA reads it before the last one to
+    // finish advances it
+    const int64_t round = __ldcg(&a.state->round);
+    const bool first_round = round == 0;
 
     if (warp == kConsumers / 32) {
         // ------------------------------------------------------ producer ---
@@ -370,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                         zo.z = __fmaf_rn(a.eta, __fsub_rn(y0.z, xo.z), xo.z);
                         zo.w = __fmaf_rn(a.eta, __fsub_rn(y0.w, xo.w), xo.w);
                     }
-                    const float4 zp = (MODE == kOutEq2 && a.first_round) ? zo : bo;
+                    const float4 zp = (MODE == kOutEq2 && first_round) ? zo : bo;
                     const float xa[4] = {xo.x, xo.y, xo.z, xo.w}, ya[4] = {yo.x, yo.y, yo.z, yo.w};
                     const float za[4] = {zo.x, zo.y, zo.z, zo.w}, zpa[4] = {zp.x, zp.y, zp.z, zp.w};
                     const float aa[4] = {acc.x, acc.y, acc.z, acc.w};
@@ -469,8 +473,9 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
         for (unsigned b = lane; b < gridDim.x; b += 32) s += __ldcg(a.partials + b);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
         if (lane == 0) {
-            *a.ce_out = s / static_cast<double>(n);
+            a.ce_ring[round % a.ce_ring_len] = s / static_cast<double>(n);
             *a.ticket = 0u;
+            a.state->round = round + 1;
         }
     }
 }

@@ -60,17 +60,41 @@ struct InitArgs {
     uint64_t seed;
 };
 
+// Step counters of the replicas, resident on the device so that a round can
+// be replayed from a CUDA graph: every per-step scalar is derived from here.
+struct DevState {
+    int64_t round;                    // completed gossip rounds
+    int64_t nsteps[kMaxWorkers];      // local steps taken by each worker
+    double p1[kMaxWorkers];           // beta1^n (n successive products from 1)
+    double p2[kMaxWorkers];           // beta2^n
+};
+
+// Per-worker scalars of the current local step (written by the prep kernel).
+struct StepTable {
+    float step[kMaxWorkers];          // fl32(lr / (1 - beta1^n))
+    float isb[kMaxWorkers];           // fl32(1 / sqrt(1 - beta2^n))
+    uint32_t key_lo[kMaxWorkers];     // noise key hash(seed, 4, i, n)
+    uint32_t key_hi[kMaxWorkers];
+};
+
+struct PrepArgs {
+    DevState *state;
+    StepTable *table;
+    uint32_t active_mask;             // workers taking this step
+    int32_t n_workers;
+    double lr, beta1, beta2;
+    uint64_t seed;
+};
+
 struct AdamwArgs {
     const TensorDesc *tens;
     const Tile *tiles;
     int64_t ntiles;
+    const StepTable *table;
     int32_t n_active;
     int32_t per_worker_h;
     uint32_t from_x_mask;                 // bit i: worker i starts from x
     int32_t worker[kMaxWorkers];
-    float step[kMaxWorkers];              // lr / (1 - beta1^n)
-    float isb[kMaxWorkers];               // 1 / sqrt(1 - beta2^n)
-    uint32_t key_lo[kMaxWorkers], key_hi[kMaxWorkers];   // noise key of the step
     float decay, beta1, beta2, omb1, omb2, eps, sigma;
 };
 
@@ -83,14 +107,15 @@ struct GossipArgs {
     int32_t n_workers;
     int32_t mode;          // GASLOC_OUTER_*
     uint32_t fresh_mask;   // bit j: worker j took a local step this round
-    int32_t first_round;   // Eq. 2: no momentum term at t = 0
+    DevState *state;       // round counter: t = 0 check, CE slot, advanced by the last CTA
     int32_t tile;          // elements per tile (4 x 256 / groups)
     int32_t groups;        // consumer threads per 16-byte column
     int32_t stages;
     float eta_out, mu, eta, alpha, oma, gamma;
     double *partials;      // [gridDim] per-CTA consensus-error partials
     unsigned int *ticket;  // last-CTA-done counter (returns to 0)
-    double *ce_out;        // consensus error of the new x
+    double *ce_ring;       // consensus error of round t goes to ce_ring[t % ring]
+    int32_t ce_ring_len;
     int32_t *err;
 };
 
@@ -106,7 +131,10 @@ struct CeArgs {
 
 // Launchers (return cudaGetLastError()).
 cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s);
-cudaError_t launch_topo(const TopoSpec &spec, int64_t round, Topo *out, cudaStream_t s);
+// round_ptr != nullptr: the round is read from device memory (graph replay).
+cudaError_t launch_topo(const TopoSpec &spec, int64_t round, const int64_t *round_ptr, Topo *out,
+                        cudaStream_t s);
+cudaError_t launch_prep(const PrepArgs &a, cudaStream_t s);
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s);
 cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream_t s);
 

@@ -53,7 +53,8 @@ __global__ void init_kernel(const InitArgs a) {
 // Neighbour table of round t, one warp.  Lane 0 draws the permutation
 // (Fisher-Yates, Lemire multiply-shift); edges are bitmasks; each lane then
 // applies edge activation to the edges it owns and builds its own row.
-__global__ void topo_kernel(const TopoSpec spec, const int64_t round, Topo *out) {
+__global__ void topo_kernel(const TopoSpec spec, const int64_t round_arg, const int64_t *round_ptr, Topo *out) {
+    const int64_t round = round_ptr ? *round_ptr : round_arg;
     __shared__ uint32_t adj[kMaxWorkers];
     __shared__ int32_t perm[kMaxWorkers];
     __shared__ int32_t deg[kMaxWorkers];
@@ -174,6 +175,27 @@ __global__ void topo_kernel(const TopoSpec spec, const int64_t round, Topo *out)
     }
 }
 
+// Scalars of one local step for every active worker, from the device-resident
+// counters (one warp; lane i = worker i).  Each operation is a single IEEE
+// double rounding, as the host formulas: p <- p * beta; bc = 1 - p;
+// step = fl32(lr / bc1); isb = fl32(1 / sqrt(bc2)); key = hash(seed, 4, i, n).
+__global__ void prep_kernel(const PrepArgs a) {
+    const int i = threadIdx.x;
+    if (i >= a.n_workers || !((a.active_mask >> i) & 1u)) return;
+    const int64_t n = a.state->nsteps[i] + 1;
+    const double p1 = __dmul_rn(a.state->p1[i], a.beta1);
+    const double p2 = __dmul_rn(a.state->p2[i], a.beta2);
+    const double bc1 = __dsub_rn(1.0, p1), bc2 = __dsub_rn(1.0, p2);
+    a.table->step[i] = __double2float_rn(__ddiv_rn(a.lr, bc1));
+    a.table->isb[i] = __double2float_rn(__ddiv_rn(1.0, __dsqrt_rn(bc2)));
+    const uint64_t key = hash4(a.seed, kTagNoise, static_cast<uint64_t>(i), static_cast<uint64_t>(n));
+    a.table->key_lo[i] = static_cast<uint32_t>(key);
+    a.table->key_hi[i] = static_cast<uint32_t>(key >> 32);
+    a.state->nsteps[i] = n;
+    a.state->p1[i] = p1;
+    a.state->p2[i] = p2;
+}
+
 // xbar = (1/n) sum_i x_i: fp32 sum in ascending i, times fl32(1/n).
 __global__ void average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
                                float *dst) {
@@ -248,8 +270,14 @@ cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_topo(const TopoSpec &spec, int64_t round, Topo *out, cudaStream_t s) {
-    topo_kernel<<<1, 32, 0, s>>>(spec, round, out);
+cudaError_t launch_topo(const TopoSpec &spec, int64_t round, const int64_t *round_ptr, Topo *out,
+                        cudaStream_t s) {
+    topo_kernel<<<1, 32, 0, s>>>(spec, round, round_ptr, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prep(const PrepArgs &a, cudaStream_t s) {
+    prep_kernel<<<1, 32, 0, s>>>(a);
     return cudaGetLastError();
 }
 

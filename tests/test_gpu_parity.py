@@ -70,6 +70,8 @@ TOPO_CASES = [
     (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
     (12, "exp", {"weights": "uniform", "edge_prob": 0.3}),
     (9, "ring", {"weights": "lazy", "edge_prob": 0.8}),
+    (8, "exp", {"weights": "metropolis", "edge_prob": 0.0}),    # every edge dropped: W = I
+    (8, "matching", {"weights": "uniform", "edge_prob": 0.0}),
 ]
 
 

@@ -1,0 +1,88 @@
+"""gasloc_run: rounds replayed from a CUDA graph must be exactly the rounds
+the call-by-call API produces (and the oracle's), including random per-round
+graphs (the round number is read on the device), per-worker step counts, a
+hyperparameter change (a new graph is captured) and the consensus-error trace."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2606_11081_gb300 as g
+from paper_2606_11081_gb300 import build as gbuild
+from paper_2606_11081_gb300 import workloads as wl
+
+from _pairs import make_pair
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    gbuild.build()
+    oracle.build()
+
+
+CASES = [
+    (8, "matching", dict(), 2, None),
+    (6, "exp", dict(weights="metropolis", edge_prob=0.5, per_worker_h=True), -1, [1, 3, 2, 1, 2, 3]),
+    (4, "ring", dict(outer="eq2", alpha=0.8, gamma=0.3, eta=0.9), 1, None),
+    (8, "2peer", dict(weights="lazy", outer="local_dadam"), 3, None),
+]
+
+
+@pytest.mark.parametrize("N,topo,kw,H,Hi", CASES)
+def test_run_matches_stepwise_and_oracle(N, topo, kw, H, Hi):
+    P, R = 3 * 1024 + 7, 6
+    hp = dict(kw, lr=2e-3)
+    a, st = make_pair(N, P, topo, seed=42, hp=hp, Hi=Hi)
+    b, _ = make_pair(N, P, topo, seed=42, hp=hp, Hi=Hi)
+    Hc = H if H > 0 else g.PER_WORKER_STEPS
+    with a, b:
+        trace = a.run(R, Hc, trace=True)
+        ces = []
+        for _ in range(R):
+            b.local_steps(Hc)
+            b.gossip_round()
+            ces.append(b.consensus_error())
+            st.local_steps(H if H > 0 else 0, None if Hi is None else np.array(Hi, np.int32))
+            st.gossip_round()
+        np.testing.assert_array_equal(trace, np.array(ces))
+        assert a.round == b.round == R
+        for i in range(N):
+            assert a.steps_taken(i) == b.steps_taken(i) == st.steps_taken(i)
+        for w in ("x", "b", "m", "v", "y"):
+            np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
+        np.testing.assert_array_equal(a.read_all("x"), st.get_all("x").astype(np.float32))
+        # continue call by call after graph rounds, and with graph rounds again
+        a.local_steps(Hc)
+        a.gossip_round()
+        b.run(1, Hc)
+        np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
+
+
+def test_hparam_change_recaptures():
+    P = 5000
+    a, _ = make_pair(8, P, "exp", seed=7, hp=dict(lr=1e-3))
+    b, _ = make_pair(8, P, "exp", seed=7, hp=dict(lr=1e-3))
+    with a, b:
+        a.run(3, 1)
+        for _ in range(3):
+            b.local_steps(1)
+            b.gossip_round()
+        hp2 = g.make_hparams(**dict(wl.COMMON_HP, lr=4e-3, outer="sgdm", outer_momentum=0.5))
+        a.set_hparams(hp2)
+        b.set_hparams(hp2)
+        a.run(4, 2)
+        for _ in range(4):
+            b.local_steps(2)
+            b.gossip_round()
+        np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
+        np.testing.assert_array_equal(a.read_all("b"), b.read_all("b"))
+        assert a.consensus_error() == b.consensus_error()
+        # not at a round boundary: refused
+        a.local_steps(1)
+        with pytest.raises(g.GaslocError) as e:
+            a.run(1, 1)
+        assert e.value.code == g.ESTATE
