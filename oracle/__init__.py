@@ -27,6 +27,7 @@ TOPO = {"none": 0, "ring": 1, "complete": 2, "exp": 3, "torus": 4, "matching": 5
 WEIGHTS = {"uniform": 0, "metropolis": 1, "lazy": 2}
 OUTER = {"sgd": 0, "sgdm": 1, "nesterov": 2, "eq2": 3, "dadam": 4, "local_dadam": 5}
 BUF = {"x": 0, "y": 1, "m": 2, "v": 3, "b": 4, "c": 5, "h": 6}
+STORAGE = {"f32": 0, "bf16": 1}
 
 
 def build(force: bool = False) -> None:
@@ -55,7 +56,7 @@ class Problem(ctypes.Structure):
         ("noise_sigma", ctypes.c_double),
         ("outer_lr", ctypes.c_double), ("outer_momentum", ctypes.c_double),
         ("eta", ctypes.c_double), ("alpha", ctypes.c_double), ("gamma", ctypes.c_double),
-        ("per_worker_h", ctypes.c_int32), ("pad_", ctypes.c_int32),
+        ("per_worker_h", ctypes.c_int32), ("storage", ctypes.c_int32),
     ]
 
 
@@ -65,13 +66,15 @@ def make_problem(n_workers: int, n_params: int, topology: str = "ring", seed: in
                  beta1: float = 0.9, beta2: float = 0.95, eps: float = 1e-8,
                  weight_decay: float = 0.1, noise_sigma: float = 0.01,
                  outer_lr: float = 0.7, outer_momentum: float = 0.9, eta: float = 1.0,
-                 alpha: float = 1.0, gamma: float = 0.0, per_worker_h: bool = False) -> Problem:
+                 alpha: float = 1.0, gamma: float = 0.0, per_worker_h: bool = False,
+                 storage: str = "f32") -> Problem:
     return Problem(n_workers=n_workers, topology=TOPO[topology], n_params=n_params,
                    torus_rows=torus[0], torus_cols=torus[1], weights=WEIGHTS[weights],
                    outer_mode=OUTER[outer], seed=seed, edge_prob=edge_prob, lr=lr,
                    beta1=beta1, beta2=beta2, eps=eps, weight_decay=weight_decay,
                    noise_sigma=noise_sigma, outer_lr=outer_lr, outer_momentum=outer_momentum,
-                   eta=eta, alpha=alpha, gamma=gamma, per_worker_h=int(per_worker_h), pad_=0)
+                   eta=eta, alpha=alpha, gamma=gamma, per_worker_h=int(per_worker_h),
+                   storage=STORAGE[storage])
 
 
 _I64P = ctypes.POINTER(ctypes.c_int64)
@@ -100,6 +103,7 @@ class Oracle:
             "oc_uniform": (dbl, [u64, u64, u64, u64, dbl, dbl]),
             "oc_noise": (dbl, [u64, u64, u64, u64]),
             "oc_real_size": (ctypes.c_int, []), "oc_num_threads": (ctypes.c_int, []),
+            "oc_bf16_round": (dbl, [dbl]),
             "oc_permutation": (None, [u64, i64, i32, _I32P]),
             "oc_draw_local_steps": (None, [u64, i32, i32, _I32P]),
             "oc_topology": (ctypes.c_int, [ctypes.POINTER(Problem), i64, _I32P, _F64P, _I32P]),
@@ -138,6 +142,9 @@ class Oracle:
 
     def noise(self, seed, i, n, k) -> float:
         return self.lib.oc_noise(seed, i, n, k)
+
+    def bf16_round(self, v: float) -> float:
+        return self.lib.oc_bf16_round(v)
 
     def permutation(self, seed: int, t: int, n: int) -> np.ndarray:
         p = np.zeros(n, np.int32)

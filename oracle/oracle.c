@@ -119,6 +119,36 @@ static REAL noise_xi(uint64_t key, uint64_t k)
     return (a - one) * sqrt3;
 }
 
+/* ------------------------------------------------------------------------- */
+/* bfloat16 storage                                                          */
+/* ------------------------------------------------------------------------- */
+
+/* Rounds a binary32 value to the nearest bfloat16 (the upper 16 bits of a
+ * binary32), ties to even: add 0x7FFF plus the lowest kept bit, then clear
+ * the low half.  Infinities pass through; NaNs stay NaN. */
+static float bf16_round_f(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    if ((u & 0x7F800000u) == 0x7F800000u) {
+        if (u & 0x007FFFFFu) u |= 0x00400000u;    /* keep NaN quiet */
+    } else {
+        u += 0x7FFFu + ((u >> 16) & 1u);
+    }
+    u &= 0xFFFF0000u;
+    memcpy(&f, &u, 4);
+    return f;
+}
+
+double oc_bf16_round(double v) { return (double)bf16_round_f((float)v); }
+
+/* The value a store keeps: unchanged in fp32 storage, rounded to bfloat16
+ * in bf16 storage. */
+static REAL stored(int storage, REAL v)
+{
+    return storage == OC_STORE_BF16 ? (REAL)bf16_round_f((float)v) : v;
+}
+
 /* Exported single-value generators (for the property tests). */
 double oc_normal(uint64_t seed, uint64_t tag, uint64_t i, uint64_t k)
 { return (double)normal01(seed, tag, i, k); }
@@ -331,20 +361,21 @@ oc_state *oc_create(const oc_problem *pb, const int64_t *kidx, int64_t nk)
     for (int64_t e = 0; e < nk; ++e) st->kidx[e] = kidx ? kidx[e] : e;
 
     const uint64_t seed = pb->seed;
+    const int sto = pb->storage;
     const REAL x0std = (REAL)0.02, hlo = (REAL)0.1, hspan = (REAL)0.9;
     #pragma omp parallel for schedule(static)
     for (int64_t e = 0; e < nk; ++e) {
         const uint64_t k = (uint64_t)st->kidx[e];
-        const REAL x0 = x0std * normal01(seed, 1, 0, k);
+        const REAL x0 = stored(sto, x0std * normal01(seed, 1, 0, k));
         for (int32_t i = 0; i < n; ++i) {
             const size_t o = (size_t)i * (size_t)nk + (size_t)e;
             st->x[o] = x0;
             st->y[o] = x0;
-            st->c[o] = normal01(seed, 2, (uint64_t)i, k);
+            st->c[o] = stored(sto, normal01(seed, 2, (uint64_t)i, k));
         }
         for (int32_t i = 0; i < nh; ++i)
             st->h[(size_t)i * (size_t)nk + (size_t)e] =
-                uniform_lo_span(seed, 3, (uint64_t)i, k, hlo, hspan);
+                stored(sto, uniform_lo_span(seed, 3, (uint64_t)i, k, hlo, hspan));
     }
     return st;
 }
@@ -383,6 +414,7 @@ static void adamw_step_worker(oc_state *st, int32_t i)
     const REAL eps = (REAL)pb->eps, sigma = (REAL)pb->noise_sigma;
     const uint64_t key = oc_hash(pb->seed, 4, (uint64_t)i, (uint64_t)n);
     const int first = !st->fresh[i];
+    const int sto = pb->storage;
     REAL *x = st->x + (size_t)i * (size_t)nk;
     REAL *y = st->y + (size_t)i * (size_t)nk;
     REAL *m = st->m + (size_t)i * (size_t)nk;
@@ -402,7 +434,7 @@ static void adamw_step_worker(oc_state *st, int32_t i)
         const REAL vv = fma(b2, v[e], omb2 * (g * g));
         const REAL den = fma(sqrt(vv), isb, eps);
         yy = fma(-step, mm / den, yy);
-        y[e] = yy; m[e] = mm; v[e] = vv;
+        y[e] = stored(sto, yy); m[e] = stored(sto, mm); v[e] = stored(sto, vv);
     }
     st->nsteps[i] = n;
     st->fresh[i] = 1;
@@ -525,8 +557,8 @@ int oc_gossip_round(oc_state *st)
         }
         for (int32_t i = 0; i < n; ++i) {
             const size_t o = (size_t)i * (size_t)nk + (size_t)e;
-            st->x[o] = xn[i];
-            st->b[o] = bn[i];
+            st->x[o] = stored(pb->storage, xn[i]);
+            st->b[o] = stored(pb->storage, bn[i]);
         }
     }
     for (int32_t i = 0; i < n; ++i) st->fresh[i] = 0;
@@ -603,12 +635,12 @@ int oc_get(oc_state *st, int32_t which, int32_t worker, double *out)
     return 0;
 }
 
-/* Overwrites a buffer (values are rounded to REAL). */
+/* Overwrites a buffer (values are rounded to REAL, then to the storage type). */
 int oc_set(oc_state *st, int32_t which, int32_t worker, const double *in)
 {
     REAL *p = buf_ptr(st, which, worker);
     if (!p) return -1;
-    for (int64_t e = 0; e < st->nk; ++e) p[e] = (REAL)in[e];
+    for (int64_t e = 0; e < st->nk; ++e) p[e] = stored(st->pb.storage, (REAL)in[e]);
     return 0;
 }
 

@@ -56,8 +56,12 @@ typedef struct {
     double   outer_lr, outer_momentum;              /* eta_out, mu */
     double   eta, alpha, gamma;                     /* Eq. 1 / Eq. 2 */
     int32_t  per_worker_h;    /* 1: curvature h_i per worker, 0: one h shared */
-    int32_t  pad_;
+    int32_t  storage;         /* OC_STORE_F32, or OC_STORE_BF16: every stored
+                                 value is rounded to bfloat16 (nearest, ties
+                                 to even) */
 } oc_problem;
+
+enum { OC_STORE_F32 = 0, OC_STORE_BF16 = 1 };
 
 typedef struct oc_state oc_state;
 

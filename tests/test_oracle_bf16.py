@@ -1,0 +1,62 @@
+"""Pins for the oracle's bfloat16 storage rule: every stored value is the
+binary32 result rounded to bfloat16, nearest with ties to even.  The rounding
+is checked against torch's float32 -> bfloat16 conversion (a library routine),
+including ties, overflow and subnormals; a bf16 run must hold only
+bf16-representable values and stay within bf16 resolution of the fp32 run."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+
+def _torch_bf16(vals):
+    return torch.tensor(vals, dtype=torch.float32).to(torch.bfloat16).to(torch.float32).numpy()
+
+
+def test_bf16_round_matches_torch(orc32):
+    rng = np.random.default_rng(0)
+    vals = np.concatenate([
+        rng.normal(size=4000).astype(np.float32),
+        (rng.normal(size=2000) * 1e-30).astype(np.float32),         # tiny / subnormal range
+        (rng.normal(size=2000) * 1e30).astype(np.float32),
+        np.array([0.0, -0.0, 1.0, -1.0, 3.0e38, -3.39e38, 1e-45, np.finfo(np.float32).max,
+                  np.float32(1.0) + np.float32(2.0 ** -8),                  # tie -> even (1.0)
+                  np.float32(1.0) + np.float32(3 * 2.0 ** -8),              # tie -> even (up)
+                  np.float32(1.0) + np.float32(2.0 ** -8) + np.float32(2.0 ** -20),
+                  np.inf, -np.inf], np.float32),
+    ]).astype(np.float32)
+    ours = np.array([orc32.bf16_round(float(v)) for v in vals], np.float32)
+    np.testing.assert_array_equal(ours, _torch_bf16(vals))
+    assert np.isnan(orc32.bf16_round(float("nan")))
+
+
+def test_bf16_run_stores_bf16_values(orc32):
+    N, P = 6, 777
+    pb = oracle.make_problem(N, P, "exp", seed=5, storage="bf16", weights="metropolis", lr=3e-3)
+    st = orc32.state(pb)
+    for _ in range(4):
+        st.local_steps(2)
+        st.gossip_round()
+    for w in ("x", "y", "m", "v", "b", "c", "h"):
+        a = st.get_all(w).astype(np.float32)
+        low = a.view(np.uint32) & 0xFFFF
+        assert not low.any(), w
+
+
+def test_bf16_run_tracks_f32_run(orc32):
+    N, P, R = 8, 2000, 5
+    common = dict(seed=11, lr=3e-4, noise_sigma=0.01)
+    a = orc32.state(oracle.make_problem(N, P, "exp", storage="bf16", **common))
+    b = orc32.state(oracle.make_problem(N, P, "exp", storage="f32", **common))
+    for _ in range(R):
+        for s in (a, b):
+            s.local_steps(1)
+            s.gossip_round()
+    xa, xb = a.get_all("x"), b.get_all("x")
+    # bf16 keeps 8 significant bits: after R rounds the replicas agree to a
+    # few bf16 steps of the largest value
+    assert np.abs(xa - xb).max() <= R * 2 ** -8 * np.abs(xb).max()
+    # the disagreement between replicas (~1e-4 per element here) is of the
+    # order of one bf16 step, so the consensus error agrees only roughly
+    assert 0.5 < a.consensus_error() / b.consensus_error() < 2.0
