@@ -246,6 +246,7 @@ def workload_config(w, args):
     return {"workload": w.name, "n_workers": w.n_workers, "n_params": w.n_params,
             "topology": w.topology, "H": w.H if w.H > 0 else "H_i~U{1..%d}" % w.draw_hmax,
             "layout": "tensor-list(%d)" % len(w.numels) if w.numels else "flat",
+            "storage": w.hp.get("storage", "f32"),
             "weights": w.hp.get("weights", "uniform"), "outer": "nesterov(0.7, 0.9)",
             "seed": w.seed, "parallelism": "replicas x%d" % args.gpus,
             "l2": "inputs larger than L2 (%.1f GB replica state per GPU, no flush)" % state_gb}
@@ -321,13 +322,14 @@ def main():
     # algorithmic bytes
     N, P = w.n_workers, w.n_params
     per_h = bool(w.hp.get("per_worker_h"))
+    es = 2 if w.hp.get("storage") == "bf16" else 4      # bytes per stored element
     steps = [H] * N if H > 0 else Hi
     adamw_launches = max(steps)
     adamw_bytes = 0
     for s in range(max(steps)):
         act = sum(1 for h in steps if h > s)
-        adamw_bytes += (32 * act if per_h else 28 * act + 4) * P
-    gossip_bytes = 20 * N * P
+        adamw_bytes += (8 * es * act if per_h else 7 * es * act + es) * P
+    gossip_bytes = 5 * es * N * P
     peak, peak_kind = peak_hbm()
     adamw_gbs = adamw_bytes / (local_ms / K / 1e3) / 1e9
     gossip_gbs = gossip_bytes / (gossip_ms / K / 1e3) / 1e9
@@ -352,8 +354,8 @@ def main():
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms / K, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": workload_config(w, args),
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if es == 2 else "f32",
+            "data": "synthetic", "config": workload_config(w, args),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": dom_gbs, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": dom_gbs / peak,
                          "traffic": traffic, "algorithmic_bytes_per_launch": dom_bytes_launch},

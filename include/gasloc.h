@@ -97,8 +97,15 @@ typedef struct gasloc_hparams {
     int32_t outer_mode;     /* GASLOC_OUTER_* */
     int32_t weights;        /* GASLOC_W_*     */
     int32_t per_worker_h;   /* 1: one curvature vector per worker */
-    int32_t reserved;
+    int32_t storage;        /* GASLOC_STORAGE_F32 or GASLOC_STORAGE_BF16 */
 } gasloc_hparams;
+
+/* Element type of the replica store (every array: x, y, m, v, b, c, h).  All
+ * arithmetic is fp32; with bf16 storage each stored value is rounded to
+ * bfloat16 (nearest, ties to even), which halves the bytes each step moves.
+ * The host-facing calls (read, write, gather, average) always take fp32
+ * arrays; gasloc_buffer exposes the raw elements. */
+enum { GASLOC_STORAGE_F32 = 0, GASLOC_STORAGE_BF16 = 1 };
 
 /* Device allocator hooks: alloc returns a device pointer (NULL on failure) of
  * at least `bytes` bytes, 256-byte aligned, usable on `stream`. */
@@ -122,7 +129,7 @@ int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint6
                 gasloc_ctx **out);
 
 /* Sets the hyperparameters (copied).  Before gasloc_start any field may
- * change; afterwards per_worker_h may not (ESTATE).  EINVAL if lr < 0,
+ * change; afterwards per_worker_h and storage may not (ESTATE).  EINVAL if lr < 0,
  * beta not in [0,1), eps <= 0, edge_prob not in [0,1], an unknown mode or
  * weight rule, or eta/alpha/gamma/outer_lr negative. */
 int gasloc_set_hparams(gasloc_ctx *ctx, const gasloc_hparams *hp);
@@ -224,14 +231,16 @@ int gasloc_average(gasloc_ctx *ctx, float *dst_device);
 int gasloc_average_host(gasloc_ctx *ctx, float *dst_host);
 
 /* Device pointer of buffer `which` for tensor `tensor`: worker i's slice
- * starts at *dptr + i * (*worker_stride) floats (worker_stride may be NULL;
- * for GASLOC_BUF_H with a shared curvature it is 0).  Valid until destroy. */
+ * starts at *dptr + i * (*worker_stride) elements (fp32 or bf16 as the
+ * storage type; worker_stride may be NULL; for GASLOC_BUF_H with a shared
+ * curvature it is 0).  Valid until destroy. */
 int gasloc_buffer(gasloc_ctx *ctx, int32_t which, int32_t tensor, void **dptr,
                   int64_t *worker_stride);
 
-/* Copies buffer `which` of `worker` (flat, n_params floats) to or from host
- * memory.  In gasloc_write, worker = -1 writes every worker (x_0 broadcast).
- * Synchronising. */
+/* Copies buffer `which` of `worker` (flat, n_params fp32 values) to or from
+ * host memory (with bf16 storage: widened exactly on read, rounded to nearest
+ * even on write).  In gasloc_write, worker = -1 writes every worker (x_0
+ * broadcast).  Synchronising. */
 int gasloc_read(gasloc_ctx *ctx, int32_t which, int32_t worker, float *host_dst);
 int gasloc_write(gasloc_ctx *ctx, int32_t which, int32_t worker, const float *host_src);
 

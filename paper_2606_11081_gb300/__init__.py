@@ -23,6 +23,7 @@ OK, EINVAL, ENOMEM, ECUDA, ESTATE, EDEVICE, EIO = 0, -1, -2, -3, -4, -5, -6
 OUTER = {"sgd": 0, "sgdm": 1, "nesterov": 2, "eq2": 3, "dadam": 4, "local_dadam": 5}
 WEIGHTS = {"uniform": 0, "metropolis": 1, "lazy": 2}
 BUF = {"x": 0, "y": 1, "m": 2, "v": 3, "b": 4, "c": 5, "h": 6}
+STORAGE = {"f32": 0, "bf16": 1}
 MAX_WORKERS = 32
 PER_WORKER_STEPS = -1
 
@@ -41,7 +42,7 @@ class Hparams(ctypes.Structure):
                 ("alpha", ctypes.c_double), ("gamma", ctypes.c_double),
                 ("edge_prob", ctypes.c_double), ("outer_mode", ctypes.c_int32),
                 ("weights", ctypes.c_int32), ("per_worker_h", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
+                ("storage", ctypes.c_int32)]
 
 
 ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p)
@@ -429,9 +430,22 @@ class Context:
         if rows is None:
             rows = self.n if (which != "h" or self.hparams.per_worker_h) else 1
 
+        if self.hparams.storage == STORAGE["bf16"]:
+            raw = self.view_raw_u16(ptr, stride, rows, numel)
+            return raw.view(torch.bfloat16)
+
         class _Cai:
             __cuda_array_interface__ = {"shape": (rows, numel), "typestr": "<f4", "data": (ptr, False),
                                         "strides": (max(stride, 1) * 4, 4), "version": 3}
+        return torch.as_tensor(_Cai(), device="cuda")
+
+    @staticmethod
+    def view_raw_u16(ptr: int, stride: int, rows: int, numel: int):
+        import torch
+
+        class _Cai:
+            __cuda_array_interface__ = {"shape": (rows, numel), "typestr": "<i2", "data": (ptr, False),
+                                        "strides": (max(stride, 1) * 2, 2), "version": 3}
         return torch.as_tensor(_Cai(), device="cuda")
 
     @property
@@ -469,6 +483,8 @@ def make_hparams(**kw) -> Hparams:
             hp.weights = WEIGHTS[v]
         elif k == "per_worker_h":
             hp.per_worker_h = int(v)
+        elif k == "storage":
+            hp.storage = STORAGE[v] if isinstance(v, str) else int(v)
         else:
             if not hasattr(hp, k):
                 raise KeyError(k)

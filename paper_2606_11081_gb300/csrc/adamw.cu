@@ -3,15 +3,20 @@
 //
 // Memory-bound streaming kernel: per active worker and element it reads the
 // iterate (x on the first step of a round, else y), m, v and the centre c and
-// writes y, m, v -- 28 bytes -- plus 4 bytes of shared curvature h per element
-// (h is per worker in the heterogeneous workload: 32 bytes per worker-element).
-// One thread owns one 16-byte column of a tile and walks the active workers U
-// at a time (U = 4, or 3 with per-worker h), issuing all of their 16-byte loads
-// before any arithmetic so that 15-16 requests per thread stay in flight.  The synthetic gradient g = h (y - c) + sigma xi
-// is formed in registers; xi comes from a 32-bit counter hash of the element
-// index and the step key, so the gradient costs no memory traffic.
+// writes y, m, v -- 28 bytes in fp32 storage, 14 in bf16 -- plus the shared
+// curvature h per element (h is per worker in the heterogeneous workload).
+// One thread owns a column of 4 consecutive elements of a tile and walks the
+// active workers U at a time (U = 4, or 3 with per-worker h), issuing all of
+// their loads before any arithmetic so that 15-16 requests per thread stay in
+// flight.  The synthetic gradient g = h (y - c) + sigma xi is formed in
+// registers; xi comes from a 32-bit counter hash of the element index and the
+// step key, so the gradient costs no memory traffic.  The step's per-worker
+// scalars (bias corrections, noise keys) come from the step table the prep
+// kernel wrote.
 //
-// Per element, one IEEE rounding per line (the order the oracle follows):
+// Per element, in fp32 with one IEEE rounding per line (the oracle's order);
+// with bf16 storage the loads widen exactly and each stored value is rounded
+// to bf16 (nearest, ties to even):
 //   d = y - c;  t = h d;  g = fma(sigma, xi, t)
 //   y = y * decay
 //   m = fma(beta1, m, (1 - beta1) g)
@@ -20,6 +25,7 @@
 //   y = fma(-step, m / den, y)
 #include <cuda_runtime.h>
 
+#include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
@@ -58,8 +64,9 @@ __device__ __forceinline__ float noise_xi(uint32_t k, uint32_t klo, uint32_t khi
     return __fmul_rn(__fsub_rn(a, 1.0f), sqrt3);
 }
 
-template <int U, bool PER_WORKER_H>
+template <int U, bool PER_WORKER_H, typename T>
 __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
+    using E = Elem<T>;
     const Consts kc{a.decay, a.beta1, a.beta2, a.omb1, a.omb2, a.eps, a.sigma};
     // this step's per-worker scalars (written by the prep kernel) -> shared
     __shared__ StepTable tab;
@@ -76,25 +83,29 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
             d = a.tens[tl.tensor];
             cur = tl.tensor;
         }
+        const T *X = as<T>(static_cast<const void *>(d.x));
+        const T *C = as<T>(static_cast<const void *>(d.c));
+        const T *Hh = as<T>(static_cast<const void *>(d.h));
+        T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
         const int64_t off = tl.start + e0;
         const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
         const uint32_t k0 = static_cast<uint32_t>(d.goff + off);
         float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (!PER_WORKER_H) hs = ptx::ld_stream(d.h + off);
+        if (!PER_WORKER_H) hs = E::load4(Hh + off);
 
         for (int a0 = 0; a0 < a.n_active; a0 += U) {
-            float4 Y[U], M[U], V[U], C[U], Hh[U];
+            float4 Y[U], M[U], V[U], Cc[U], Hw[U];
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 if (a0 + u < a.n_active) {
                     const int i = a.worker[a0 + u];
                     const int64_t o = i * d.wstride + off;
-                    const float *src = ((a.from_x_mask >> i) & 1u) ? d.x : d.y;
-                    Y[u] = ptx::ld_stream(src + o);
-                    M[u] = ptx::ld_stream(d.m + o);
-                    V[u] = ptx::ld_stream(d.v + o);
-                    C[u] = ptx::ld_stream(d.c + o);
-                    if (PER_WORKER_H) Hh[u] = ptx::ld_stream(d.h + i * d.hstride + off);
+                    const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
+                    Y[u] = E::load4(src + o);
+                    M[u] = E::load4(Mw + o);
+                    V[u] = E::load4(Vw + o);
+                    Cc[u] = E::load4(C + o);
+                    if (PER_WORKER_H) Hw[u] = E::load4(Hh + i * d.hstride + off);
                 }
             }
 #pragma unroll
@@ -104,29 +115,29 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const float step = tab.step[i];
                     const float isb = tab.isb[i];
                     const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
-                    const float4 h4 = PER_WORKER_H ? Hh[u] : hs;
+                    const float4 h4 = PER_WORKER_H ? Hw[u] : hs;
                     float4 yo, mo, vo;
-                    yo.x = adamw_lane(Y[u].x, M[u].x, V[u].x, C[u].x, h4.x, noise_xi(k0 + 0, klo, khi),
+                    yo.x = adamw_lane(Y[u].x, M[u].x, V[u].x, Cc[u].x, h4.x, noise_xi(k0 + 0, klo, khi),
                                       step, isb, kc, mo.x, vo.x);
-                    yo.y = adamw_lane(Y[u].y, M[u].y, V[u].y, C[u].y, h4.y, noise_xi(k0 + 1, klo, khi),
+                    yo.y = adamw_lane(Y[u].y, M[u].y, V[u].y, Cc[u].y, h4.y, noise_xi(k0 + 1, klo, khi),
                                       step, isb, kc, mo.y, vo.y);
-                    yo.z = adamw_lane(Y[u].z, M[u].z, V[u].z, C[u].z, h4.z, noise_xi(k0 + 2, klo, khi),
+                    yo.z = adamw_lane(Y[u].z, M[u].z, V[u].z, Cc[u].z, h4.z, noise_xi(k0 + 2, klo, khi),
                                       step, isb, kc, mo.z, vo.z);
-                    yo.w = adamw_lane(Y[u].w, M[u].w, V[u].w, C[u].w, h4.w, noise_xi(k0 + 3, klo, khi),
+                    yo.w = adamw_lane(Y[u].w, M[u].w, V[u].w, Cc[u].w, h4.w, noise_xi(k0 + 3, klo, khi),
                                       step, isb, kc, mo.w, vo.w);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
-                        ptx::st_stream(d.y + o, yo);
-                        ptx::st_stream(d.m + o, mo);
-                        ptx::st_stream(d.v + o, vo);
+                        E::store4(Yw + o, yo);
+                        E::store4(Mw + o, mo);
+                        E::store4(Vw + o, vo);
                     } else {
                         const float ya[4] = {yo.x, yo.y, yo.z, yo.w};
                         const float ma[4] = {mo.x, mo.y, mo.z, mo.w};
                         const float va[4] = {vo.x, vo.y, vo.z, vo.w};
                         for (int l = 0; l < nvalid; ++l) {
-                            d.y[o + l] = ya[l];
-                            d.m[o + l] = ma[l];
-                            d.v[o + l] = va[l];
+                            E::store1(Yw + o + l, ya[l]);
+                            E::store1(Mw + o + l, ma[l]);
+                            E::store1(Vw + o + l, va[l]);
                         }
                     }
                 }
@@ -135,23 +146,37 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     }
 }
 
-}  // namespace
-
-int adamw_blocks_per_sm(int block, bool per_worker_h) {
+template <typename T>
+int blocks_per_sm(int block, bool per_worker_h) {
     int nb = 0;
     const cudaError_t e =
-        per_worker_h ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<3, true>, block, 0)
-                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<4, false>, block, 0);
+        per_worker_h ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<3, true, T>, block, 0)
+                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<4, false, T>, block, 0);
     if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
 }
 
+template <typename T>
+void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
+    if (a.per_worker_h)
+        adamw_kernel<3, true, T><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
+    else
+        adamw_kernel<4, false, T><<<grid, kBlock, 0, s>>>(a);
+}
+
+}  // namespace
+
+int adamw_blocks_per_sm(int block, bool per_worker_h, int storage) {
+    return storage == kStoreBF16 ? blocks_per_sm<bf16>(block, per_worker_h)
+                                 : blocks_per_sm<float>(block, per_worker_h);
+}
+
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s) {
     (void)block;
-    if (a.per_worker_h)
-        adamw_kernel<3, true><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
+    if (a.storage == kStoreBF16)
+        launch<bf16>(a, grid, s);
     else
-        adamw_kernel<4, false><<<grid, kBlock, 0, s>>>(a);
+        launch<float>(a, grid, s);
     return cudaGetLastError();
 }
 

@@ -3,15 +3,15 @@
 // for states the gossip kernel has not already reduced (after a checkpoint
 // load, a direct write of x, or before the first round).
 //
-// One thread owns a 16-byte column and loads x_ik for all n workers (8 loads
-// in flight per batch).  The column sum uses the same shifted one-pass form as
-// the fused path, e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with
-// s = x_0k, so both paths give identical per-element values.  Reduction: fp64
-// per thread, warp shuffles, one partial per CTA, last CTA adds the partials
-// in CTA order (atomic ticket; nothing waits).  Reads 4 bytes per
-// worker-element.
+// One thread owns a column of 4 elements and loads x_ik for all n workers (8
+// loads in flight per batch).  Per element the shifted one-pass form
+// e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with s = x_0k, in fp32.
+// Reduction: fp64 per thread, warp shuffles, one partial per CTA, the last
+// CTA adds the partials in CTA order (atomic ticket; nothing waits).  Reads
+// one element per worker-element (4 or 2 bytes).
 #include <cuda_runtime.h>
 
+#include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -21,7 +21,9 @@ namespace {
 
 constexpr int kBlock = 256;
 
+template <typename T>
 __global__ void __launch_bounds__(kBlock) ce_kernel(const CeArgs a) {
+    using E = Elem<T>;
     __shared__ double red[kBlock / 32];
     __shared__ int last;
     const int n = a.n_workers;
@@ -37,19 +39,20 @@ __global__ void __launch_bounds__(kBlock) ce_kernel(const CeArgs a) {
             d = a.tens[tl.tensor];
             cur = tl.tensor;
         }
+        const T *X = as<T>(static_cast<const void *>(d.x));
         const int64_t off = tl.start + e0;
         const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
         float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f}, sh[4];
         constexpr int U = 8;
         for (int i0 = 0; i0 < n; i0 += U) {
-            float4 X[U];
+            float4 Xv[U];
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                if (i0 + u < n) X[u] = ptx::ld_stream(d.x + (i0 + u) * d.wstride + off);
+                if (i0 + u < n) Xv[u] = E::load4(X + (i0 + u) * d.wstride + off);
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 if (i0 + u >= n) continue;
-                const float xa[4] = {X[u].x, X[u].y, X[u].z, X[u].w};
+                const float xa[4] = {Xv[u].x, Xv[u].y, Xv[u].z, Xv[u].w};
 #pragma unroll
                 for (int l = 0; l < 4; ++l) {
                     if (i0 + u == 0) sh[l] = xa[l];
@@ -92,15 +95,21 @@ __global__ void __launch_bounds__(kBlock) ce_kernel(const CeArgs a) {
 
 }  // namespace
 
-int ce_blocks_per_sm(int block) {
+int ce_blocks_per_sm(int block, int storage) {
     int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, ce_kernel, block, 0) != cudaSuccess) return 1;
+    const cudaError_t e = storage == kStoreBF16
+                              ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, ce_kernel<bf16>, block, 0)
+                              : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, ce_kernel<float>, block, 0);
+    if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
 }
 
 cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s) {
     (void)block;
-    ce_kernel<<<grid, kBlock, 0, s>>>(a);
+    if (a.storage == kStoreBF16)
+        ce_kernel<bf16><<<grid, kBlock, 0, s>>>(a);
+    else
+        ce_kernel<float><<<grid, kBlock, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -1,0 +1,82 @@
+// elem.cuh -- loads and stores of the replica store's element type.
+//
+// The store holds fp32 or bfloat16 values; kernels always compute in fp32.
+// Widening bf16 -> fp32 is exact (the bf16 bits are the top half of the
+// fp32); narrowing rounds to nearest, ties to even (__float2bfloat16_rn).
+// Vector accesses move 4 consecutive elements (16 bytes of fp32, 8 bytes of
+// bf16) with streaming (evict-first) cache hints.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+namespace gasloc {
+
+using bf16 = __nv_bfloat16;
+
+template <typename T>
+struct Elem;
+
+template <>
+struct Elem<float> {
+    static constexpr int kBytes = 4;
+    static __device__ __forceinline__ float4 load4(const float *p) {
+        return __ldcs(reinterpret_cast<const float4 *>(p));
+    }
+    static __device__ __forceinline__ void store4(float *p, float4 v) {
+        __stcs(reinterpret_cast<float4 *>(p), v);
+    }
+    static __device__ __forceinline__ float4 load4_smem(const float *p) {
+        return *reinterpret_cast<const float4 *>(p);
+    }
+    static __device__ __forceinline__ void store4_smem(float *p, float4 v) {
+        *reinterpret_cast<float4 *>(p) = v;
+    }
+    static __device__ __forceinline__ float load1(const float *p) { return *p; }
+    static __device__ __forceinline__ void store1(float *p, float v) { *p = v; }
+    // the value a store keeps
+    static __device__ __forceinline__ float round(float v) { return v; }
+};
+
+__device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t bf_pack(float lo, float hi) {
+    const uint32_t a = __bfloat16_as_ushort(__float2bfloat16_rn(lo));
+    const uint32_t b = __bfloat16_as_ushort(__float2bfloat16_rn(hi));
+    return a | (b << 16);
+}
+
+template <>
+struct Elem<bf16> {
+    static constexpr int kBytes = 2;
+    static __device__ __forceinline__ float4 load4(const bf16 *p) {
+        const uint2 u = __ldcs(reinterpret_cast<const uint2 *>(p));
+        return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+    }
+    static __device__ __forceinline__ void store4(bf16 *p, float4 v) {
+        __stcs(reinterpret_cast<uint2 *>(p), make_uint2(bf_pack(v.x, v.y), bf_pack(v.z, v.w)));
+    }
+    static __device__ __forceinline__ float4 load4_smem(const bf16 *p) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(p);
+        return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+    }
+    static __device__ __forceinline__ void store4_smem(bf16 *p, float4 v) {
+        *reinterpret_cast<uint2 *>(p) = make_uint2(bf_pack(v.x, v.y), bf_pack(v.z, v.w));
+    }
+    static __device__ __forceinline__ float load1(const bf16 *p) { return __bfloat162float(*p); }
+    static __device__ __forceinline__ void store1(bf16 *p, float v) { *p = __float2bfloat16_rn(v); }
+    // the value a store keeps
+    static __device__ __forceinline__ float round(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+};
+
+template <typename T>
+__device__ __forceinline__ T *as(void *p) {
+    return static_cast<T *>(p);
+}
+template <typename T>
+__device__ __forceinline__ const T *as(const void *p) {
+    return static_cast<const T *>(p);
+}
+
+}  // namespace gasloc

@@ -47,6 +47,22 @@ constexpr int kCeRing = 4096;
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
+// Host-side conversions of the bf16 store: widening is exact; narrowing
+// rounds to nearest, ties to even (add 0x7FFF plus the lowest kept bit).
+float bf16_to_f32(uint16_t b) {
+    const uint32_t u = static_cast<uint32_t>(b) << 16;
+    float f;
+    std::memcpy(&f, &u, 4);
+    return f;
+}
+uint16_t f32_to_bf16(float f) {
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    if ((u & 0x7F800000u) == 0x7F800000u) return static_cast<uint16_t>((u >> 16) | ((u & 0x007FFFFFu) ? 0x40u : 0u));
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return static_cast<uint16_t>(u >> 16);
+}
+
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -69,14 +85,16 @@ EncodeTiledFn encode_tiled() {
 // 2-D map over one array of one tensor: [n workers][numel] fp32 with a row
 // pitch of wstride floats, boxes of [n x 256]; out-of-range elements read as
 // zero and are not written.
-bool make_map(CUtensorMap *m, float *base, int64_t numel, int64_t wstride, int32_t n) {
+bool make_map(CUtensorMap *m, void *base, int64_t numel, int64_t wstride, int32_t n, int storage) {
     EncodeTiledFn enc = encode_tiled();
     if (!enc) return false;
+    const bool bf = storage == kStoreBF16;
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(numel), static_cast<cuuint64_t>(n)};
-    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(wstride) * 4};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(wstride) * (bf ? 2 : 4)};
     const cuuint32_t box[2] = {256, static_cast<cuuint32_t>(n)};
     const cuuint32_t estr[2] = {1, 1};
-    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+    return enc(m, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -228,6 +246,8 @@ int check_hparams(const gasloc_hparams *hp) {
     if (hp->weights < GASLOC_W_UNIFORM || hp->weights > GASLOC_W_LAZY)
         return fail(GASLOC_EINVAL, "unknown weight rule %d", hp->weights);
     if (hp->per_worker_h != 0 && hp->per_worker_h != 1) return fail(GASLOC_EINVAL, "per_worker_h must be 0 or 1");
+    if (hp->storage != GASLOC_STORAGE_F32 && hp->storage != GASLOC_STORAGE_BF16)
+        return fail(GASLOC_EINVAL, "unknown storage type %d", hp->storage);
     return GASLOC_OK;
 }
 
@@ -272,16 +292,19 @@ int build_topology(gasloc_ctx *c, int64_t round, const int64_t *round_ptr, Topo 
     return launch_checked(c, launch_topo(c->spec, round, round_ptr, dst, s), "topology kernel");
 }
 
-float *buffer_base(const TensorDesc &d, int which, int64_t *stride) {
+size_t esize_of(const gasloc_ctx *c) { return c->hp.storage == GASLOC_STORAGE_BF16 ? 2 : 4; }
+
+// Base address (bytes) of buffer `which` of a tensor; *stride in elements.
+char *buffer_base(const TensorDesc &d, int which, int64_t *stride) {
     *stride = d.wstride;
     switch (which) {
-    case GASLOC_BUF_X: return d.x;
-    case GASLOC_BUF_Y: return d.y;
-    case GASLOC_BUF_M: return d.m;
-    case GASLOC_BUF_V: return d.v;
-    case GASLOC_BUF_B: return d.b;
-    case GASLOC_BUF_C: return d.c;
-    case GASLOC_BUF_H: *stride = d.hstride; return d.h;
+    case GASLOC_BUF_X: return static_cast<char *>(d.x);
+    case GASLOC_BUF_Y: return static_cast<char *>(d.y);
+    case GASLOC_BUF_M: return static_cast<char *>(d.m);
+    case GASLOC_BUF_V: return static_cast<char *>(d.v);
+    case GASLOC_BUF_B: return static_cast<char *>(d.b);
+    case GASLOC_BUF_C: return static_cast<char *>(d.c);
+    case GASLOC_BUF_H: *stride = d.hstride; return static_cast<char *>(d.h);
     default: return nullptr;
     }
 }
@@ -351,8 +374,8 @@ int gasloc_set_hparams(gasloc_ctx *c, const gasloc_hparams *hp) {
     if (!c || !hp) return fail(GASLOC_EINVAL, "NULL argument");
     int rc = check_hparams(hp);
     if (rc) return rc;
-    if (c->started && hp->per_worker_h != c->hp.per_worker_h)
-        return fail(GASLOC_ESTATE, "per_worker_h cannot change after gasloc_start");
+    if (c->started && (hp->per_worker_h != c->hp.per_worker_h || hp->storage != c->hp.storage))
+        return fail(GASLOC_ESTATE, "per_worker_h and storage cannot change after gasloc_start");
     c->hp = *hp;
     c->gen += 1;
     refresh_spec(c);
@@ -411,7 +434,7 @@ int gasloc_start(gasloc_ctx *c) {
     int64_t need = 0;
     for (int64_t ne : c->numels) {
         const int64_t ws = round_up(ne, kPadFloats);
-        need += (6LL * n + nh) * ws * 4;
+        need += (6LL * n + nh) * ws * static_cast<int64_t>(esize_of(c));
     }
     size_t fr = 0, tot = 0;
     if (cudaMemGetInfo(&fr, &tot) == cudaSuccess && static_cast<size_t>(need) > fr)
@@ -420,8 +443,9 @@ int gasloc_start(gasloc_ctx *c) {
     // gossip launch shape (the tile depends on n only; stages and shared
     // memory on the mode's staged rows): size the attribute for the largest
     size_t smem_attr = 0;
-    for (int m = 0; m < 6; ++m) smem_attr = std::max(smem_attr, gossip_shape(n, m).smem);
-    c->tile_g = gossip_shape(n, GASLOC_OUTER_NESTEROV).tile;
+    for (int st = 0; st < 2; ++st)
+        for (int m = 0; m < 6; ++m) smem_attr = std::max(smem_attr, gossip_shape(n, m, st).smem);
+    c->tile_g = gossip_shape(n, GASLOC_OUTER_NESTEROV, c->hp.storage).tile;
     e = gossip_set_smem(smem_attr);
     if (e != cudaSuccess) return cuda_fail(e, "gossip shared-memory attribute");
 
@@ -442,12 +466,12 @@ int gasloc_start(gasloc_ctx *c) {
         d.hstride = c->hp.per_worker_h ? d.wstride : 0;
         d.goff = g;
         g += d.numel;
-        float **arrs[6] = {&d.x, &d.y, &d.m, &d.v, &d.b, &d.c};
-        for (float **a : arrs) {
-            *a = static_cast<float *>(c->dalloc(static_cast<size_t>(n) * d.wstride * 4));
+        void **arrs[6] = {&d.x, &d.y, &d.m, &d.v, &d.b, &d.c};
+        for (void **a : arrs) {
+            *a = c->dalloc(static_cast<size_t>(n) * d.wstride * esize_of(c));
             if (!*a) return oom("replica arrays");
         }
-        d.h = static_cast<float *>(c->dalloc(static_cast<size_t>(nh) * d.wstride * 4));
+        d.h = c->dalloc(static_cast<size_t>(nh) * d.wstride * esize_of(c));
         if (!d.h) return oom("curvature");
         c->tens_h.push_back(d);
         c->goff.push_back(d.goff);
@@ -476,9 +500,9 @@ int gasloc_start(gasloc_ctx *c) {
     std::vector<CUtensorMap> maps(c->tens_h.size() * 3);
     for (size_t t = 0; t < c->tens_h.size(); ++t) {
         const TensorDesc &d = c->tens_h[t];
-        float *arrs[3] = {d.x, d.y, d.b};
+        void *arrs[3] = {d.x, d.y, d.b};
         for (int k = 0; k < 3; ++k)
-            if (!make_map(&maps[t * 3 + k], arrs[k], d.numel, d.wstride, n)) {
+            if (!make_map(&maps[t * 3 + k], arrs[k], d.numel, d.wstride, n, c->hp.storage)) {
                 c->release_all();
                 return fail(GASLOC_ECUDA, "cuTensorMapEncodeTiled failed for tensor %zu", t);
             }
@@ -520,14 +544,14 @@ int gasloc_start(gasloc_ctx *c) {
     e = cudaStreamSynchronize(c->stream);
     if (e != cudaSuccess) { c->release_all(); return cuda_fail(e, "table upload"); }
 
-    c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0);
+    c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0, c->hp.storage);
     for (int m = 0; m < 6; ++m) {
-        const GossipShape sm = gossip_shape(n, m);
-        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, sm.smem));
+        const GossipShape sm = gossip_shape(n, m, c->hp.storage);
+        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm.smem));
     }
-    c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256));
+    c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
 
-    InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed};
+    InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed, c->hp.storage};
     int rc = launch_checked(c, launch_init(ia, c->sms * 8, c->stream), "init kernel");
     if (rc) { c->release_all(); return rc; }
     c->started = true;
@@ -589,6 +613,7 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.ntiles = c->ntiles_a;
     a.table = c->table_d;
     a.per_worker_h = hp.per_worker_h;
+    a.storage = hp.storage;
     a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
     a.beta1 = static_cast<float>(hp.beta1);
     a.beta2 = static_cast<float>(hp.beta2);
@@ -635,11 +660,12 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     a.ntiles = c->ntiles_g;
     a.topo = c->topo_d;
     a.maps = c->maps_d;
+    a.storage = hp.storage;
     a.n_workers = c->n;
     a.mode = hp.outer_mode;
     a.fresh_mask = c->fresh_mask;
     a.state = c->state_d;
-    const GossipShape gs = gossip_shape(c->n, hp.outer_mode);
+    const GossipShape gs = gossip_shape(c->n, hp.outer_mode, hp.storage);
     a.tile = gs.tile;
     a.groups = gs.groups;
     a.stages = gs.stages;
@@ -769,7 +795,7 @@ int gasloc_consensus_error(gasloc_ctx *c, double *out) {
     if (!out) return fail(GASLOC_EINVAL, "out is NULL");
     const double *src = c->ce_d;
     if (!c->ce_valid || c->round == 0) {
-        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->partials, c->ticket, c->ce_d};
+        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d};
         rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
         if (rc) return rc;
     } else {
@@ -817,7 +843,8 @@ int gasloc_average(gasloc_ctx *c, float *dst) {
     int rc = check_started(c);
     if (rc) return rc;
     if (!dst) return fail(GASLOC_EINVAL, "dst is NULL");
-    return launch_checked(c, launch_average(c->tens_d, c->tiles_a, c->ntiles_a, c->n, dst, c->sms * 8, c->stream),
+    return launch_checked(c, launch_average(c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, dst, c->sms * 8,
+                                            c->stream),
                           "average kernel");
 }
 
@@ -844,7 +871,7 @@ int gasloc_buffer(gasloc_ctx *c, int32_t which, int32_t tensor, void **dptr, int
     if (!dptr) return fail(GASLOC_EINVAL, "dptr is NULL");
     if (tensor < 0 || tensor >= static_cast<int32_t>(c->tens_h.size())) return fail(GASLOC_EINVAL, "tensor out of range");
     int64_t stride = 0;
-    float *p = buffer_base(c->tens_h[tensor], which, &stride);
+    char *p = buffer_base(c->tens_h[tensor], which, &stride);
     if (!p) return fail(GASLOC_EINVAL, "unknown buffer %d", which);
     *dptr = p;
     if (worker_stride) *worker_stride = stride;
@@ -857,12 +884,23 @@ int gasloc_read(gasloc_ctx *c, int32_t which, int32_t worker, float *host) {
     if (!host) return fail(GASLOC_EINVAL, "host buffer is NULL");
     rc = check_which_worker(c, which, worker, false);
     if (rc) return rc;
+    const size_t es = esize_of(c);
+    std::vector<uint16_t> tmp;
     for (const TensorDesc &d : c->tens_h) {
         int64_t stride = 0;
-        const float *p = buffer_base(d, which, &stride);
-        cudaError_t e = cudaMemcpyAsync(host + d.goff, p + worker * stride, static_cast<size_t>(d.numel) * 4,
-                                        cudaMemcpyDeviceToHost, c->stream);
+        const char *p = buffer_base(d, which, &stride) + static_cast<size_t>(worker * stride) * es;
+        void *dst = host + d.goff;
+        if (es == 2) {
+            tmp.resize(static_cast<size_t>(d.numel));
+            dst = tmp.data();
+        }
+        cudaError_t e = cudaMemcpyAsync(dst, p, static_cast<size_t>(d.numel) * es, cudaMemcpyDeviceToHost, c->stream);
         if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
+        if (es == 2) {
+            rc = sync_and_check(c);
+            if (rc) return rc;
+            for (int64_t k = 0; k < d.numel; ++k) host[d.goff + k] = bf16_to_f32(tmp[static_cast<size_t>(k)]);
+        }
     }
     return sync_and_check(c);
 }
@@ -875,15 +913,28 @@ int gasloc_write(gasloc_ctx *c, int32_t which, int32_t worker, const float *host
     if (rc) return rc;
     const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
     const int32_t w0 = worker < 0 ? 0 : worker, w1 = worker < 0 ? rows : worker + 1;
+    const size_t es = esize_of(c);
+    std::vector<uint16_t> tmp;
     for (const TensorDesc &d : c->tens_h) {
         int64_t stride = 0;
-        float *p = buffer_base(d, which, &stride);
-        cudaError_t e = cudaMemcpyAsync(p + w0 * stride, host + d.goff, static_cast<size_t>(d.numel) * 4,
-                                        cudaMemcpyHostToDevice, c->stream);
+        char *p = buffer_base(d, which, &stride);
+        const size_t bytes = static_cast<size_t>(d.numel) * es;
+        const void *src = host + d.goff;
+        if (es == 2) {
+            tmp.resize(static_cast<size_t>(d.numel));
+            for (int64_t k = 0; k < d.numel; ++k) tmp[static_cast<size_t>(k)] = f32_to_bf16(host[d.goff + k]);
+            src = tmp.data();
+        }
+        char *row0 = p + static_cast<size_t>(w0 * stride) * es;
+        cudaError_t e = cudaMemcpyAsync(row0, src, bytes, cudaMemcpyHostToDevice, c->stream);
         if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
+        if (es == 2) {   // tmp is reused for the next tensor
+            e = cudaStreamSynchronize(c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+        }
         for (int32_t i = w0 + 1; i < w1; ++i) {
-            e = cudaMemcpyAsync(p + i * stride, p + w0 * stride, static_cast<size_t>(d.numel) * 4,
-                                cudaMemcpyDeviceToDevice, c->stream);
+            e = cudaMemcpyAsync(p + static_cast<size_t>(i * stride) * es, row0, bytes, cudaMemcpyDeviceToDevice,
+                                c->stream);
             if (e != cudaSuccess) return cuda_fail(e, "device-to-device copy");
         }
     }
@@ -909,7 +960,8 @@ int gasloc_gather(gasloc_ctx *c, int32_t which, int32_t worker, int64_t n, const
     }
     cudaError_t e = cudaMemcpyAsync(di, idx, static_cast<size_t>(n) * 8, cudaMemcpyHostToDevice, c->stream);
     if (e == cudaSuccess) {
-        rc = launch_checked(c, launch_gather(c->tens_d, static_cast<int32_t>(c->tens_h.size()), which, worker, di, n,
+        rc = launch_checked(c, launch_gather(c->tens_d, static_cast<int32_t>(c->tens_h.size()), c->hp.storage, which,
+                                             worker, di, n,
                                              dout, c->err_d, c->stream),
                             "gather kernel");
         if (!rc) {
@@ -966,6 +1018,8 @@ struct CkptHeader {
     int64_t round;
     uint32_t fresh_mask;
     int32_t has_Hi;
+    int32_t storage;
+    int32_t pad;
 };
 }  // namespace
 
@@ -978,8 +1032,8 @@ int gasloc_save(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "wb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s' for writing", path);
     CkptHeader h{};
-    std::memcpy(h.magic, "GASLOCK1", 8);
-    h.version = 1;
+    std::memcpy(h.magic, "GASLOCK2", 8);
+    h.version = 2;
     h.n = c->n;
     h.P = c->P;
     h.n_tensors = static_cast<int64_t>(c->numels.size());
@@ -991,24 +1045,27 @@ int gasloc_save(gasloc_ctx *c, const char *path) {
     h.round = c->round;
     h.fresh_mask = c->fresh_mask;
     h.has_Hi = c->has_Hi ? 1 : 0;
+    h.storage = c->hp.storage;
     bool ok = std::fwrite(&h, sizeof h, 1, f) == 1;
     ok = ok && std::fwrite(c->numels.data(), 8, c->numels.size(), f) == c->numels.size();
     ok = ok && std::fwrite(&c->hp, sizeof c->hp, 1, f) == 1;
     ok = ok && std::fwrite(c->nsteps.data(), 8, c->n, f) == static_cast<size_t>(c->n);
     ok = ok && std::fwrite(c->Hi.data(), 4, c->n, f) == static_cast<size_t>(c->n);
-    std::vector<float> buf;
+    const size_t es = esize_of(c);
+    std::vector<char> buf;
     for (const TensorDesc &d : c->tens_h) {
-        buf.resize(static_cast<size_t>(d.numel));
+        buf.resize(static_cast<size_t>(d.numel) * es);
         for (int which = GASLOC_BUF_X; ok && which <= GASLOC_BUF_H; ++which) {
             const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
             int64_t stride = 0;
-            const float *p = buffer_base(d, which, &stride);
+            const char *p = buffer_base(d, which, &stride);
             for (int32_t i = 0; ok && i < rows; ++i) {
-                if (cudaMemcpy(buf.data(), p + i * stride, buf.size() * 4, cudaMemcpyDeviceToHost) != cudaSuccess) {
+                if (cudaMemcpy(buf.data(), p + static_cast<size_t>(i * stride) * es, buf.size(),
+                               cudaMemcpyDeviceToHost) != cudaSuccess) {
                     std::fclose(f);
                     return fail(GASLOC_ECUDA, "checkpoint copy failed");
                 }
-                ok = std::fwrite(buf.data(), 4, buf.size(), f) == buf.size();
+                ok = std::fwrite(buf.data(), 1, buf.size(), f) == buf.size();
             }
         }
     }
@@ -1024,11 +1081,11 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "rb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s'", path);
     CkptHeader h{};
-    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK1", 8) == 0 && h.version == 1;
+    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK2", 8) == 0 && h.version == 2;
     if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "'%s' is not a checkpoint", path); }
     if (h.n != c->n || h.P != c->P || h.n_tensors != static_cast<int64_t>(c->numels.size()) || h.seed != c->seed ||
         h.kind != c->spec.kind || h.rows != c->spec.rows || h.cols != c->spec.cols ||
-        h.per_worker_h != c->hp.per_worker_h) {
+        h.per_worker_h != c->hp.per_worker_h || h.storage != c->hp.storage) {
         std::fclose(f);
         return fail(GASLOC_EINVAL, "checkpoint does not match this context");
     }
@@ -1043,16 +1100,18 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "truncated checkpoint header"); }
     rc = sync_and_check(c);
     if (rc) { std::fclose(f); return rc; }
-    std::vector<float> buf;
+    const size_t es = esize_of(c);
+    std::vector<char> buf;
     for (const TensorDesc &d : c->tens_h) {
-        buf.resize(static_cast<size_t>(d.numel));
+        buf.resize(static_cast<size_t>(d.numel) * es);
         for (int which = GASLOC_BUF_X; ok && which <= GASLOC_BUF_H; ++which) {
             const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
             int64_t stride = 0;
-            float *p = buffer_base(d, which, &stride);
+            char *p = buffer_base(d, which, &stride);
             for (int32_t i = 0; ok && i < rows; ++i) {
-                ok = std::fread(buf.data(), 4, buf.size(), f) == buf.size();
-                if (ok && cudaMemcpy(p + i * stride, buf.data(), buf.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+                ok = std::fread(buf.data(), 1, buf.size(), f) == buf.size();
+                if (ok && cudaMemcpy(p + static_cast<size_t>(i * stride) * es, buf.data(), buf.size(),
+                                     cudaMemcpyHostToDevice) != cudaSuccess) {
                     std::fclose(f);
                     return fail(GASLOC_ECUDA, "checkpoint upload failed");
                 }

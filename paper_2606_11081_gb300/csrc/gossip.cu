@@ -37,6 +37,7 @@
 // ticket protocol completes.
 #include <cuda_runtime.h>
 
+#include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -104,8 +105,6 @@ __device__ __forceinline__ float outer_update(float acc, float x, float y, float
     }
 }
 
-__device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
-__device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
@@ -140,9 +139,10 @@ __device__ __forceinline__ void consumer_barrier() {
     asm volatile("barrier.sync 1, %0;" ::"r"(kConsumers) : "memory");
 }
 
-template <int MODE>
+template <int MODE, typename T>
 __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a) {
     using R = ModeRows<MODE>;
+    using E = Elem<T>;
     extern __shared__ __align__(128) unsigned char smem[];
     Topo *tp = reinterpret_cast<Topo *>(smem);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + kOffFull);
@@ -150,14 +150,15 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
     double *red = reinterpret_cast<double *>(smem + kOffRed);
     volatile int *flags = reinterpret_cast<volatile int *>(smem + kOffFlags);   // [0] abort, [1] last
     float4 *cebuf = reinterpret_cast<float4 *>(smem + kOffCe);
-    float *stages = reinterpret_cast<float *>(smem + kOffStages);
+    T *stages = reinterpret_cast<T *>(smem + kOffStages);
 
     const int n = a.n_workers;
     const int TILE = a.tile;
     const int G = a.groups;
     const int cols = TILE / 4;
     const int S = a.stages;
-    const size_t stage_floats = static_cast<size_t>(R::kRows) * n * TILE;
+    const size_t stage_elems = static_cast<size_t>(R::kRows) * n * TILE;
+    constexpr int kVec = 16 / static_cast<int>(sizeof(T));   // elements per 16 bytes
     const int NQ = TILE / kBox;   // sub-boxes per tile: kind k, sub-box q, worker j at ((k NQ + q) n + j) kBox
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -200,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
         const bool none_fresh = (a.fresh_mask & all_mask) == 0u;
         const bool uniform = all_fresh || none_fresh;
         const int kvar = R::kMixX ? 1 : 0;   // the kind whose source depends on freshness
-        auto blk = [&](float *st, int k, int q) { return st + static_cast<size_t>(k * NQ + q) * n * kBox; };
+        auto blk = [&](T *st, int k, int q) { return st + static_cast<size_t>(k * NQ + q) * n * kBox; };
         auto tmap = [&](int tensor, int arr) {   // arr: 0 x, 1 y, 2 b
             return static_cast<const unsigned char *>(a.maps) + (static_cast<size_t>(tensor) * 3 + arr) * 128;
         };
@@ -218,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
         auto store_tile = [&](int64_t j) {   // box stores of tile j, spread over lanes
             const Tile tl = a.tiles[first + j * gstride];
             const int nq = (tl.len + kBox - 1) / kBox;
-            float *st = stages + (j % S) * stage_floats;
+            T *st = stages + (j % S) * stage_elems;
             const int nops = (R::kHasB ? 2 : 1) * nq;
             fence_maps(tl.tensor);
             for (int o = lane; o < nops; o += 32) {
@@ -253,14 +254,14 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
             const Tile tl = a.tiles[first + it * gstride];
             const TensorDesc &d = a.tens[tl.tensor];
             const int nq = (tl.len + kBox - 1) / kBox;
-            const int lenr = (tl.len + 3) & ~3;
-            float *st = stages + s * stage_floats;
+            const int lenr = (tl.len + kVec - 1) / kVec * kVec;   // whole 16-byte chunks
+            T *st = stages + s * stage_elems;
             fence_maps(tl.tensor);
             // bytes this stage will receive
             uint32_t tx = 0;
             for (int k = 0; k < R::kRows; ++k) {
-                if (k == kvar && !uniform) tx += static_cast<uint32_t>(n) * static_cast<uint32_t>(lenr) * 4u;
-                else tx += static_cast<uint32_t>(nq) * static_cast<uint32_t>(n * kBox * 4);
+                if (k == kvar && !uniform) tx += static_cast<uint32_t>(n) * static_cast<uint32_t>(lenr) * sizeof(T);
+                else tx += static_cast<uint32_t>(nq) * static_cast<uint32_t>(n * kBox * sizeof(T));
             }
             if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], tx);
             __syncwarp();
@@ -274,11 +275,11 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
             if (!uniform) {   // per-worker source: y if the worker is fresh, else x
                 for (int j = lane; j < n; j += 32) {
                     const bool fresh = (a.fresh_mask >> j) & 1u;
-                    const float *src = (fresh ? d.y : d.x) + j * d.wstride + tl.start;
+                    const T *src = static_cast<const T *>(fresh ? d.y : d.x) + j * d.wstride + tl.start;
                     for (int q = 0; q < nq; ++q) {
                         const int w = lenr - q * kBox < kBox ? lenr - q * kBox : kBox;
                         ptx::bulk_g2s(blk(st, kvar, q) + static_cast<size_t>(j) * kBox, src + q * kBox,
-                                      static_cast<uint32_t>(w) * 4u, &full[s]);
+                                      static_cast<uint32_t>(w * sizeof(T)), &full[s]);
                     }
                 }
             }
@@ -320,7 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                 atomicCAS(a.err, kDevOk, kDevWaitTimeout);
             }
             const int tlen = a.tiles[first + it * gstride].len;
-            float *st = stages + s * stage_floats;
+            T *st = stages + s * stage_elems;
             // row of worker j, kind k, at this thread's column
             auto cp = [&](int k, int j) {
                 return st + (static_cast<size_t>(k) * NQ + qb) * n * kBox + static_cast<size_t>(j) * kBox + rb;
@@ -333,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                 // shift of the consensus-error sums: worker 0's new x when one
                 // thread sees every worker of the column (G = 1), else worker
                 // 0's sent value, which every group can read
-                const float4 shift = ld4(cp(0, 0));
+                const float4 shift = E::load4_smem(cp(0, 0));
                 float sh[4] = {shift.x, shift.y, shift.z, shift.w};
                 int nr = 0;
                 for (int i = g; i < n; i += G) {
@@ -342,9 +343,9 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
                         const float w = tp->w[i][q];
-                        float4 sj = ld4(cp(0, j));
+                        float4 sj = E::load4_smem(cp(0, j));
                         if (MODE == kOutEq2) {
-                            const float4 xj = ld4(cp(1, j));
+                            const float4 xj = E::load4_smem(cp(1, j));
                             sj.x = __fmaf_rn(a.eta, __fsub_rn(sj.x, xj.x), xj.x);
                             sj.y = __fmaf_rn(a.eta, __fsub_rn(sj.y, xj.y), xj.y);
                             sj.z = __fmaf_rn(a.eta, __fsub_rn(sj.z, xj.z), xj.z);
@@ -355,20 +356,20 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                         acc.z = __fmaf_rn(w, sj.z, acc.z);
                         acc.w = __fmaf_rn(w, sj.w, acc.w);
                     }
-                    float *p0 = cp(0, i);   // mixed row i
-                    float *p1 = cp(1, i);   // own x (own y in the DAdam modes)
-                    float *p2 = cp(2, i);   // own b
+                    T *p0 = cp(0, i);   // mixed row i
+                    T *p1 = cp(1, i);   // own x (own y in the DAdam modes)
+                    T *p2 = cp(2, i);   // own b
                     float4 xo, yo, zo = make_float4(0.f, 0.f, 0.f, 0.f), bo = make_float4(0.f, 0.f, 0.f, 0.f);
                     if (R::kMixX) {
-                        xo = ld4(p0);
-                        yo = ld4(p1);
+                        xo = E::load4_smem(p0);
+                        yo = E::load4_smem(p1);
                     } else {
-                        xo = ld4(p1);
+                        xo = E::load4_smem(p1);
                         yo = xo;
                     }
-                    if (R::kHasB) bo = ld4(p2);
+                    if (R::kHasB) bo = E::load4_smem(p2);
                     if (MODE == kOutEq2) {
-                        const float4 y0 = ld4(p0);
+                        const float4 y0 = E::load4_smem(p0);
                         zo.x = __fmaf_rn(a.eta, __fsub_rn(y0.x, xo.x), xo.x);
                         zo.y = __fmaf_rn(a.eta, __fsub_rn(y0.y, xo.y), xo.y);
                         zo.z = __fmaf_rn(a.eta, __fsub_rn(y0.z, xo.z), xo.z);
@@ -383,7 +384,8 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
 #pragma unroll
                     for (int l = 0; l < 4; ++l) {
                         if (l < nvalid) {
-                            xn[l] = outer_update<MODE>(aa[l], xa[l], ya[l], ba[l], za[l], zpa[l], a);
+                            // the consensus error is that of the replicas as stored
+                            xn[l] = E::round(outer_update<MODE>(aa[l], xa[l], ya[l], ba[l], za[l], zpa[l], a));
                             if (G == 1 && i == 0) sh[l] = xn[l];
                             const float dv = __fsub_rn(xn[l], sh[l]);
                             s1[l] = __fadd_rn(s1[l], dv);
@@ -399,8 +401,8 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                         br[nr] = bn4;
                         ++nr;
                     } else {
-                        st4(p1, xn4);   // own row: read by this thread only
-                        if (R::kHasB) st4(p2, bn4);
+                        E::store4_smem(p1, xn4);   // own row: read by this thread only
+                        if (R::kHasB) E::store4_smem(p2, bn4);
                     }
                 }
             }
@@ -412,8 +414,8 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
                 if (active) {
                     int r = 0;
                     for (int i = g; i < n; i += G, ++r) {
-                        st4(cp(1, i), xr[r]);
-                        st4(cp(2, i), br[r]);
+                        E::store4_smem(cp(1, i), xr[r]);
+                        E::store4_smem(cp(2, i), br[r]);
                     }
                 }
             }
@@ -481,31 +483,45 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
 }
 
 template <int MODE>
-void *kernel_ptr() {
-    return reinterpret_cast<void *>(gossip_kernel<MODE>);
+void *kernel_ptr(int storage) {
+    return storage == kStoreBF16 ? reinterpret_cast<void *>(gossip_kernel<MODE, bf16>)
+                                 : reinterpret_cast<void *>(gossip_kernel<MODE, float>);
 }
 
-void *mode_kernel(int mode) {
+void *mode_kernel(int mode, int storage) {
     switch (mode) {
-    case kOutSgd: return kernel_ptr<kOutSgd>();
-    case kOutSgdm: return kernel_ptr<kOutSgdm>();
-    case kOutNesterov: return kernel_ptr<kOutNesterov>();
-    case kOutEq2: return kernel_ptr<kOutEq2>();
-    case kOutDadam: return kernel_ptr<kOutDadam>();
-    default: return kernel_ptr<kOutLocalDadam>();
+    case kOutSgd: return kernel_ptr<kOutSgd>(storage);
+    case kOutSgdm: return kernel_ptr<kOutSgdm>(storage);
+    case kOutNesterov: return kernel_ptr<kOutNesterov>(storage);
+    case kOutEq2: return kernel_ptr<kOutEq2>(storage);
+    case kOutDadam: return kernel_ptr<kOutDadam>(storage);
+    default: return kernel_ptr<kOutLocalDadam>(storage);
     }
 }
 
 int mode_rows(int mode) { return (mode == kOutSgd || mode == kOutDadam) ? 2 : 3; }
 
+template <typename T>
+void launch_t(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
+    switch (a.mode) {
+    case kOutSgd: gossip_kernel<kOutSgd, T><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutSgdm: gossip_kernel<kOutSgdm, T><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutNesterov: gossip_kernel<kOutNesterov, T><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutEq2: gossip_kernel<kOutEq2, T><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutDadam: gossip_kernel<kOutDadam, T><<<grid, kThreads, smem, s>>>(a); break;
+    default: gossip_kernel<kOutLocalDadam, T><<<grid, kThreads, smem, s>>>(a); break;
+    }
+}
+
 }  // namespace
 
-GossipShape gossip_shape(int n, int mode) {
+GossipShape gossip_shape(int n, int mode, int storage) {
     GossipShape sh{};
     sh.groups = n <= 8 ? 1 : (n <= 16 ? 2 : 4);
     sh.tile = 4 * (kConsumers / sh.groups);
     sh.block = kThreads;
-    const size_t stage = static_cast<size_t>(mode_rows(mode)) * n * sh.tile * sizeof(float);
+    const size_t esize = storage == kStoreBF16 ? 2 : 4;
+    const size_t stage = static_cast<size_t>(mode_rows(mode)) * n * sh.tile * esize;
     const size_t budget = 232448 - kOffStages;
     int st = static_cast<int>(budget / stage);
     sh.stages = st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
@@ -514,17 +530,19 @@ GossipShape gossip_shape(int n, int mode) {
 }
 
 cudaError_t gossip_set_smem(size_t smem) {
-    for (int m = 0; m <= kOutLocalDadam; ++m) {
-        const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-    }
+    for (int st = 0; st <= kStoreBF16; ++st)
+        for (int m = 0; m <= kOutLocalDadam; ++m) {
+            const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m, st),
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                       static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+        }
     return cudaSuccess;
 }
 
-int gossip_blocks_per_sm(int mode, size_t smem) {
+int gossip_blocks_per_sm(int mode, int storage, size_t smem) {
     int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, reinterpret_cast<const void *>(mode_kernel(mode)),
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, reinterpret_cast<const void *>(mode_kernel(mode, storage)),
                                                       kThreads, smem) != cudaSuccess)
         return 1;
     return nb > 0 ? nb : 1;
@@ -534,14 +552,10 @@ cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream
     if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups) ||
         a.tile % kBox != 0 || a.maps == nullptr)
         return cudaErrorInvalidValue;
-    switch (a.mode) {
-    case kOutSgd: gossip_kernel<kOutSgd><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutSgdm: gossip_kernel<kOutSgdm><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutNesterov: gossip_kernel<kOutNesterov><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutEq2: gossip_kernel<kOutEq2><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutDadam: gossip_kernel<kOutDadam><<<grid, kThreads, smem, s>>>(a); break;
-    default: gossip_kernel<kOutLocalDadam><<<grid, kThreads, smem, s>>>(a); break;
-    }
+    if (a.storage == kStoreBF16)
+        launch_t<bf16>(a, grid, smem, s);
+    else
+        launch_t<float>(a, grid, smem, s);
     return cudaGetLastError();
 }
 

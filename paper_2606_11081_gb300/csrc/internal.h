@@ -9,12 +9,16 @@ namespace gasloc {
 
 constexpr int kMaxWorkers = 32;
 
+// Element type of the replica store.
+enum Storage : int32_t { kStoreF32 = 0, kStoreBF16 = 1 };
+
 // One parameter tensor of the replica store.  Every array is one allocation
-// of shape [n_workers][wstride] fp32 (h: [1 or n_workers][wstride]);
-// wstride = numel rounded up to 64 floats so each worker slice is 256-byte
-// aligned.  Padding is zero-filled at start and never written afterwards.
+// of shape [n_workers][wstride] elements (fp32 or bf16; h: [1 or n][wstride]);
+// wstride = numel rounded up to 64 elements so each worker slice is 128- or
+// 256-byte aligned.  Padding is zero-filled at start and never written
+// afterwards.  Kernels cast the pointers to their element type.
 struct TensorDesc {
-    float *x, *y, *m, *v, *b, *c, *h;
+    void *x, *y, *m, *v, *b, *c, *h;
     int64_t numel;     // valid elements per worker
     int64_t wstride;   // floats between consecutive workers
     int64_t hstride;   // floats between workers in h (0 when shared)
@@ -58,6 +62,7 @@ struct InitArgs {
     int32_t n_workers;
     int32_t per_worker_h;
     uint64_t seed;
+    int32_t storage;
 };
 
 // Step counters of the replicas, resident on the device so that a round can
@@ -93,6 +98,7 @@ struct AdamwArgs {
     const StepTable *table;
     int32_t n_active;
     int32_t per_worker_h;
+    int32_t storage;
     uint32_t from_x_mask;                 // bit i: worker i starts from x
     int32_t worker[kMaxWorkers];
     float decay, beta1, beta2, omb1, omb2, eps, sigma;
@@ -104,6 +110,7 @@ struct GossipArgs {
     int64_t ntiles;
     const Topo *topo;
     const void *maps;      // per tensor: 2-D tensor maps of x, y, b (128 bytes each)
+    int32_t storage;
     int32_t n_workers;
     int32_t mode;          // GASLOC_OUTER_*
     uint32_t fresh_mask;   // bit j: worker j took a local step this round
@@ -124,6 +131,7 @@ struct CeArgs {
     const Tile *tiles;
     int64_t ntiles;
     int32_t n_workers;
+    int32_t storage;
     double *partials;
     unsigned int *ticket;
     double *ce_out;
@@ -143,20 +151,20 @@ struct GossipShape {
     int groups, tile, block, stages;
     size_t smem;
 };
-GossipShape gossip_shape(int n, int mode);
+GossipShape gossip_shape(int n, int mode, int storage);
 cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s);
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
-                           int32_t n_workers, float *dst, int grid, cudaStream_t s);
-cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
-                          const int64_t *idx, int64_t n, float *out, int32_t *err,
+                           int32_t n_workers, int32_t storage, float *dst, int grid, cudaStream_t s);
+cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t storage, int32_t which,
+                          int32_t worker, const int64_t *idx, int64_t n, float *out, int32_t *err,
                           cudaStream_t s);
 
 cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s);
 
 // Occupancy-derived persistent grid sizes.
-int adamw_blocks_per_sm(int block, bool per_worker_h);
-int gossip_blocks_per_sm(int mode, size_t smem);
-int ce_blocks_per_sm(int block);
+int adamw_blocks_per_sm(int block, bool per_worker_h, int storage);
+int gossip_blocks_per_sm(int mode, int storage, size_t smem);
+int ce_blocks_per_sm(int block, int storage);
 cudaError_t gossip_set_smem(size_t smem);
 
 // Sets the thread-local message returned by gasloc_last_error().

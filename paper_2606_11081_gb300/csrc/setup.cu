@@ -3,6 +3,7 @@
 // Algorithm 1) and an index gather used for sampled checks.
 #include <cuda_runtime.h>
 
+#include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
@@ -28,24 +29,28 @@ __device__ __forceinline__ float curvature(uint64_t seed, uint64_t i, uint64_t k
     return __fmaf_rn(static_cast<float>(0.9), u, static_cast<float>(0.1));
 }
 
+// Initial state (stored values rounded to the element type).
+template <typename T>
 __global__ void init_kernel(const InitArgs a) {
+    using E = Elem<T>;
     const float x0std = static_cast<float>(0.02);
     for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
         const Tile tl = a.tiles[ti];
         const TensorDesc d = a.tens[tl.tensor];
+        T *X = as<T>(d.x), *Y = as<T>(d.y), *C = as<T>(d.c), *Hh = as<T>(d.h);
         for (int e = threadIdx.x; e < tl.len; e += blockDim.x) {
             const int64_t off = tl.start + e;
             const uint64_t k = static_cast<uint64_t>(d.goff + off);
             const float x0 = __fmul_rn(x0std, normal_std(a.seed, kTagX0, 0, k));
             for (int i = 0; i < a.n_workers; ++i) {
                 const int64_t o = i * d.wstride + off;
-                d.x[o] = x0;
-                d.y[o] = x0;
-                d.c[o] = normal_std(a.seed, kTagCentre, static_cast<uint64_t>(i), k);
+                E::store1(X + o, x0);
+                E::store1(Y + o, x0);
+                E::store1(C + o, normal_std(a.seed, kTagCentre, static_cast<uint64_t>(i), k));
             }
             const int nh = a.per_worker_h ? a.n_workers : 1;
             for (int i = 0; i < nh; ++i)
-                d.h[i * d.hstride + off] = curvature(a.seed, static_cast<uint64_t>(i), k);
+                E::store1(Hh + i * d.hstride + off, curvature(a.seed, static_cast<uint64_t>(i), k));
         }
     }
 }
@@ -196,22 +201,26 @@ __global__ void prep_kernel(const PrepArgs a) {
     a.state->p2[i] = p2;
 }
 
-// xbar = (1/n) sum_i x_i: fp32 sum in ascending i, times fl32(1/n).
+// xbar = (1/n) sum_i x_i: fp32 sum in ascending i, times fl32(1/n); fp32 out.
+template <typename T>
 __global__ void average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
                                float *dst) {
+    using E = Elem<T>;
     const float inv_n = static_cast<float>(1.0 / n);
     for (int64_t ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
         const Tile tl = tiles[ti];
         const TensorDesc d = tens[tl.tensor];
+        const T *X = as<T>(static_cast<const void *>(d.x));
         for (int e = threadIdx.x; e < tl.len; e += blockDim.x) {
             const int64_t off = tl.start + e;
             float s = 0.0f;
-            for (int i = 0; i < n; ++i) s = __fadd_rn(s, d.x[i * d.wstride + off]);
+            for (int i = 0; i < n; ++i) s = __fadd_rn(s, E::load1(X + i * d.wstride + off));
             dst[d.goff + off] = __fmul_rn(s, inv_n);
         }
     }
 }
 
+template <typename T>
 __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
                               const int64_t *idx, int64_t n, float *out, int32_t *err) {
     const int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
@@ -230,7 +239,7 @@ __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t whi
         out[q] = 0.0f;
         return;
     }
-    const float *base;
+    const void *base;
     int64_t stride = d.wstride;
     switch (which) {
     case 0: base = d.x; break;
@@ -241,7 +250,7 @@ __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t whi
     case 5: base = d.c; break;
     default: base = d.h; stride = d.hstride; break;
     }
-    out[q] = base[worker * stride + off];
+    out[q] = Elem<T>::load1(static_cast<const T *>(base) + worker * stride + off);
 }
 
 // A wait on an mbarrier that nothing ever completes, through the bounded-wait
@@ -266,7 +275,10 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s
 }
 
 cudaError_t launch_init(const InitArgs &a, int grid, cudaStream_t s) {
-    init_kernel<<<grid, 256, 0, s>>>(a);
+    if (a.storage == kStoreBF16)
+        init_kernel<bf16><<<grid, 256, 0, s>>>(a);
+    else
+        init_kernel<float><<<grid, 256, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -282,17 +294,23 @@ cudaError_t launch_prep(const PrepArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
-                           float *dst, int grid, cudaStream_t s) {
-    average_kernel<<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
+                           int32_t storage, float *dst, int grid, cudaStream_t s) {
+    if (storage == kStoreBF16)
+        average_kernel<bf16><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
+    else
+        average_kernel<float><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
     return cudaGetLastError();
 }
 
-cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t which, int32_t worker,
-                          const int64_t *idx, int64_t n, float *out, int32_t *err, cudaStream_t s) {
+cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t storage, int32_t which,
+                          int32_t worker, const int64_t *idx, int64_t n, float *out, int32_t *err,
+                          cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
-    const int64_t grid = (n + 255) / 256;
-    gather_kernel<<<static_cast<unsigned>(grid), 256, 0, s>>>(tens, ntens, which, worker, idx, n,
-                                                               out, err);
+    const unsigned grid = static_cast<unsigned>((n + 255) / 256);
+    if (storage == kStoreBF16)
+        gather_kernel<bf16><<<grid, 256, 0, s>>>(tens, ntens, which, worker, idx, n, out, err);
+    else
+        gather_kernel<float><<<grid, 256, 0, s>>>(tens, ntens, which, worker, idx, n, out, err);
     return cudaGetLastError();
 }
 

@@ -53,12 +53,14 @@ class Workload:
 
     def bytes_per_round(self, H_i: Optional[List[int]] = None) -> int:
         """Algorithmic HBM bytes of one round: every local step reads the
-        iterate, m, v, c and writes y, m, v (28 B per worker-element) plus the
-        shared curvature (4 B per element; 4 B per worker-element when each
-        worker has its own), and the gossip round reads the sent y once and
-        x, b, and writes x, b (20 B per worker-element)."""
+        iterate, m, v, c and writes y, m, v (7 elements per worker-element:
+        28 B in fp32, 14 B in bf16) plus the shared curvature (one element per
+        element; per worker-element when each worker has its own), and the
+        gossip round reads the sent y once and x, b, and writes x, b (5
+        elements per worker-element)."""
         N, P = self.n_workers, self.n_params
         per_h = bool(self.hp.get("per_worker_h", False))
+        es = 2 if self.hp.get("storage") == "bf16" else 4
         if self.H > 0:
             steps = [self.H] * N
         else:
@@ -67,8 +69,8 @@ class Workload:
         local = 0
         for s in range(max(steps)):
             act = sum(1 for h in steps if h > s)
-            local += (32 * act if per_h else 28 * act + 4) * P
-        return local + 20 * N * P
+            local += (8 * es * act if per_h else 7 * es * act + es) * P
+        return local + 5 * es * N * P
 
 
 WORKLOADS = {
@@ -102,7 +104,18 @@ PROFILE_WORKLOADS = {
         draw_hmax=8),
 }
 
-ALL_WORKLOADS = dict(WORKLOADS, **PROFILE_WORKLOADS)
+# The benchmark workload with a bfloat16 replica store (the paper trains in
+# bf16): same arithmetic in fp32, every stored value rounded to bf16.
+BF16_WORKLOADS = {
+    "exp_n8_gpt2s_bf16": Workload(
+        "exp_n8_gpt2s_bf16", 8, GPT2_SMALL_P, "exp", 1, 200,
+        hp=dict(weights="uniform", noise_sigma=0.01, storage="bf16")),
+    "exp_n8_p16m_bf16": Workload(
+        "exp_n8_p16m_bf16", 8, 1 << 24, "exp", 1, 10,
+        hp=dict(weights="uniform", noise_sigma=0.01, storage="bf16")),
+}
+
+ALL_WORKLOADS = dict(WORKLOADS, **PROFILE_WORKLOADS, **BF16_WORKLOADS)
 
 # AdamW settings shared by every workload (App. B: weight decay 0.1,
 # betas (0.9, 0.95)); constant lr 3e-4; Nesterov outer step 0.7 / 0.9.

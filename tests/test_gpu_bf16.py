@@ -1,0 +1,114 @@
+"""bf16 replica store vs the oracle's bf16 rule (fp32 arithmetic, every stored
+value rounded to bfloat16 with ties to even): bit-exact everywhere."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2606_11081_gb300 as g
+from paper_2606_11081_gb300 import build as gbuild
+from paper_2606_11081_gb300 import workloads as wl
+
+from _pairs import make_pair, workload_pair
+
+pytestmark = pytest.mark.gpu
+BF = dict(storage="bf16")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    gbuild.build()
+    oracle.build()
+    yield
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def same(ctx, st, which):
+    for w in which:
+        a = ctx.read_all(w)
+        b = st.get_all(w).astype(np.float32)
+        assert not (a.view(np.uint32) & 0xFFFF).any(), w
+        np.testing.assert_array_equal(a, b, err_msg=w)
+
+
+def test_bf16_init_and_steps():
+    ctx, st = make_pair(5, 4099, "ring", seed=3, hp=dict(BF, per_worker_h=True, lr=2e-3))
+    with ctx:
+        same(ctx, st, ("x", "y", "c", "h"))
+        ctx.local_steps(3)
+        st.local_steps(3)
+        same(ctx, st, ("y", "m", "v"))
+
+
+@pytest.mark.parametrize("mode", ["nesterov", "sgd", "eq2", "local_dadam"])
+@pytest.mark.parametrize("N,topo,kw", [(8, "exp", {}), (16, "matching", {}),
+                                       (32, "exp", {"weights": "metropolis", "edge_prob": 0.5})])
+def test_bf16_trajectory(mode, N, topo, kw):
+    P, R, H = 2 * 1024 + 5, 4, 2
+    hp = dict(kw, **BF, outer=mode, lr=2e-3, eta=0.9, alpha=0.8, gamma=0.3, noise_sigma=0.02)
+    ctx, st = make_pair(N, P, topo, seed=500 + N, hp=hp)
+    with ctx:
+        for _ in range(R):
+            ctx.local_steps(H)
+            st.local_steps(H)
+            ctx.gossip_round()
+            st.gossip_round()
+            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+        same(ctx, st, ("x", "b", "m", "v"))
+
+
+def test_bf16_heterogeneous_and_graph_rounds():
+    Hi = np.array([0, 2, 1, 3], np.int32)
+    ctx, st = make_pair(4, 3001, "complete", seed=8, hp=dict(BF, lr=1e-3), Hi=Hi)
+    with ctx:
+        ctx.run(3, g.PER_WORKER_STEPS)
+        for _ in range(3):
+            st.local_steps(0, Hi)
+            st.gossip_round()
+        same(ctx, st, ("x", "b", "y"))
+
+
+def test_bf16_layout_and_host_conversion():
+    numels = [1000, 3, 4097, 64, 1, 2048, 5]
+    P = sum(numels)
+    a, _ = make_pair(8, P, "torus:2x4", seed=11, hp=dict(BF, weights="metropolis"))
+    b, _ = make_pair(8, P, "torus:2x4", seed=11, hp=dict(BF, weights="metropolis"), numels=numels)
+    with a, b:
+        for c in (a, b):
+            c.local_steps(2)
+            c.gossip_round()
+        for w in ("x", "y", "m", "v", "b"):
+            np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
+        # fp32 written from the host is rounded to nearest even bf16
+        vals = np.random.default_rng(0).normal(size=P).astype(np.float32)
+        a.write("x", 3, vals)
+        ref = torch.tensor(vals).to(torch.bfloat16).to(torch.float32).numpy()
+        np.testing.assert_array_equal(a.read("x", 3), ref)
+        v = b.view("x", 2, numels[2])
+        assert v.dtype == torch.bfloat16 and tuple(v.shape) == (8, numels[2])
+        np.testing.assert_array_equal(v.float().cpu().numpy(), b.read_all("x")[:, 1003:1003 + 4097])
+
+
+def test_bf16_bench_workload_full_size_sampled():
+    w = wl.ALL_WORKLOADS["exp_n8_gpt2s_bf16"]
+    rng = np.random.default_rng(1)
+    kidx = np.unique(np.concatenate([[0, 1, 1023, 1024, w.n_params - 1, w.n_params - 4],
+                                     rng.integers(0, w.n_params, 1500)])).astype(np.int64)
+    ctx, st = make_pair(w.n_workers, w.n_params, w.topology, w.seed, wl.hparams_of(w), kidx=kidx)
+    try:
+        for _ in range(w.rounds):
+            ctx.local_steps(w.H)
+            ctx.gossip_round()
+            st.local_steps(w.H)
+            st.gossip_round()
+        for which in ("x", "b", "m", "v"):
+            for i in range(w.n_workers):
+                np.testing.assert_array_equal(ctx.gather(which, i, kidx), st.get(which, i).astype(np.float32))
+        assert ctx.consensus_error() == pytest.approx(ctx.consensus_error_now(), rel=1e-6)
+    finally:
+        ctx.close()
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
