@@ -6,9 +6,9 @@
 // writes y, m, v -- 28 bytes in fp32 storage, 14 in bf16 -- plus the shared
 // curvature h per element (h is per worker in the heterogeneous workload).
 // One thread owns a column of 4 consecutive elements of a tile and walks the
-// active workers U at a time (U = 4, or 3 with per-worker h), issuing all of
-// their loads before any arithmetic so that 15-16 requests per thread stay in
-// flight.  The synthetic gradient g = h (y - c) + sigma xi is formed in
+// active workers U at a time (fp32: U = 4, or 3 with per-worker h; bf16: 8 or
+// 6), issuing all of their loads before any arithmetic so that about 256
+// bytes of requests per thread stay in flight.  The synthetic gradient g = h (y - c) + sigma xi is formed in
 // registers; xi comes from a 32-bit counter hash of the element index and the
 // step key, so the gradient costs no memory traffic.  The step's per-worker
 // scalars (bias corrections, noise keys) come from the step table the prep
@@ -94,18 +94,20 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
         if (!PER_WORKER_H) hs = E::load4(Hh + off);
 
         for (int a0 = 0; a0 < a.n_active; a0 += U) {
-            float4 Y[U], M[U], V[U], Cc[U], Hw[U];
+            // every load of the batch is issued before any arithmetic; the
+            // raw words stay packed until their worker is processed
+            typename E::Raw Y[U], M[U], V[U], Cc[U], Hw[U];
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 if (a0 + u < a.n_active) {
                     const int i = a.worker[a0 + u];
                     const int64_t o = i * d.wstride + off;
                     const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
-                    Y[u] = E::load4(src + o);
-                    M[u] = E::load4(Mw + o);
-                    V[u] = E::load4(Vw + o);
-                    Cc[u] = E::load4(C + o);
-                    if (PER_WORKER_H) Hw[u] = E::load4(Hh + i * d.hstride + off);
+                    Y[u] = E::load_raw(src + o);
+                    M[u] = E::load_raw(Mw + o);
+                    V[u] = E::load_raw(Vw + o);
+                    Cc[u] = E::load_raw(C + o);
+                    if (PER_WORKER_H) Hw[u] = E::load_raw(Hh + i * d.hstride + off);
                 }
             }
 #pragma unroll
@@ -115,16 +117,18 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const float step = tab.step[i];
                     const float isb = tab.isb[i];
                     const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
-                    const float4 h4 = PER_WORKER_H ? Hw[u] : hs;
+                    const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
+                    const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
+                                 Cu = E::unpack(Cc[u]);
                     float4 yo, mo, vo;
-                    yo.x = adamw_lane(Y[u].x, M[u].x, V[u].x, Cc[u].x, h4.x, noise_xi(k0 + 0, klo, khi),
-                                      step, isb, kc, mo.x, vo.x);
-                    yo.y = adamw_lane(Y[u].y, M[u].y, V[u].y, Cc[u].y, h4.y, noise_xi(k0 + 1, klo, khi),
-                                      step, isb, kc, mo.y, vo.y);
-                    yo.z = adamw_lane(Y[u].z, M[u].z, V[u].z, Cc[u].z, h4.z, noise_xi(k0 + 2, klo, khi),
-                                      step, isb, kc, mo.z, vo.z);
-                    yo.w = adamw_lane(Y[u].w, M[u].w, V[u].w, Cc[u].w, h4.w, noise_xi(k0 + 3, klo, khi),
-                                      step, isb, kc, mo.w, vo.w);
+                    yo.x = adamw_lane(Yu.x, Mu.x, Vu.x, Cu.x, h4.x, noise_xi(k0 + 0, klo, khi), step, isb, kc,
+                                      mo.x, vo.x);
+                    yo.y = adamw_lane(Yu.y, Mu.y, Vu.y, Cu.y, h4.y, noise_xi(k0 + 1, klo, khi), step, isb, kc,
+                                      mo.y, vo.y);
+                    yo.z = adamw_lane(Yu.z, Mu.z, Vu.z, Cu.z, h4.z, noise_xi(k0 + 2, klo, khi), step, isb, kc,
+                                      mo.z, vo.z);
+                    yo.w = adamw_lane(Yu.w, Mu.w, Vu.w, Cu.w, h4.w, noise_xi(k0 + 3, klo, khi), step, isb, kc,
+                                      mo.w, vo.w);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
                         E::store4(Yw + o, yo);
@@ -146,12 +150,18 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     }
 }
 
+// Workers per load batch: 16 (fp32) or 8 (bf16) bytes per load, so that a
+// thread keeps about 256 bytes of loads in flight in both storage types.
+template <typename T> struct Batch { static constexpr int kShared = 4, kPerWorkerH = 3; };
+template <> struct Batch<bf16> { static constexpr int kShared = 8, kPerWorkerH = 6; };
+
 template <typename T>
 int blocks_per_sm(int block, bool per_worker_h) {
     int nb = 0;
     const cudaError_t e =
-        per_worker_h ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<3, true, T>, block, 0)
-                     : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<4, false, T>, block, 0);
+        per_worker_h
+            ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kPerWorkerH, true, T>, block, 0)
+            : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kShared, false, T>, block, 0);
     if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
 }
@@ -159,9 +169,9 @@ int blocks_per_sm(int block, bool per_worker_h) {
 template <typename T>
 void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
     if (a.per_worker_h)
-        adamw_kernel<3, true, T><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
+        adamw_kernel<Batch<T>::kPerWorkerH, true, T><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
     else
-        adamw_kernel<4, false, T><<<grid, kBlock, 0, s>>>(a);
+        adamw_kernel<Batch<T>::kShared, false, T><<<grid, kBlock, 0, s>>>(a);
 }
 
 }  // namespace

@@ -21,6 +21,12 @@ struct Elem;
 template <>
 struct Elem<float> {
     static constexpr int kBytes = 4;
+    // 4 elements as loaded (kept in registers until used)
+    using Raw = float4;
+    static __device__ __forceinline__ Raw load_raw(const float *p) {
+        return __ldcs(reinterpret_cast<const float4 *>(p));
+    }
+    static __device__ __forceinline__ float4 unpack(Raw r) { return r; }
     static __device__ __forceinline__ float4 load4(const float *p) {
         return __ldcs(reinterpret_cast<const float4 *>(p));
     }
@@ -41,15 +47,22 @@ struct Elem<float> {
 
 __device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
+// two fp32 -> one bf16x2 word (low half = lo), each rounded to nearest even
 __device__ __forceinline__ uint32_t bf_pack(float lo, float hi) {
-    const uint32_t a = __bfloat16_as_ushort(__float2bfloat16_rn(lo));
-    const uint32_t b = __bfloat16_as_ushort(__float2bfloat16_rn(hi));
-    return a | (b << 16);
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&v);
 }
 
 template <>
 struct Elem<bf16> {
     static constexpr int kBytes = 2;
+    using Raw = uint2;
+    static __device__ __forceinline__ Raw load_raw(const bf16 *p) {
+        return __ldcs(reinterpret_cast<const uint2 *>(p));
+    }
+    static __device__ __forceinline__ float4 unpack(Raw u) {
+        return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+    }
     static __device__ __forceinline__ float4 load4(const bf16 *p) {
         const uint2 u = __ldcs(reinterpret_cast<const uint2 *>(p));
         return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));

@@ -54,11 +54,14 @@ constexpr size_t kOffFull = sizeof(Topo);            // 8320
 constexpr size_t kOffEmpty = kOffFull + 8 * kMaxStages;
 constexpr size_t kOffRed = kOffEmpty + 8 * kMaxStages;
 constexpr size_t kOffFlags = kOffRed + 8 * (kThreads / 32);
-constexpr size_t kOffCe = 8704;                      // 2 x [G][cols] x (S1, S2) float4
+constexpr size_t kOffCe = 8704;                      // 2 x [G][cols] x (S1, S2) float4, only if G > 1
 constexpr size_t kCeBytes = 2 * kConsumers * 32;
-constexpr size_t kOffStages = kOffCe + kCeBytes;     // 25088, 128-byte aligned
 static_assert(kOffFlags + 16 <= kOffCe, "smem layout");
-static_assert(kOffStages % 128 == 0, "stage alignment");
+static_assert(kOffCe % 128 == 0 && kCeBytes % 128 == 0, "stage alignment");
+
+// Stages start after the consensus-error exchange buffer, which only the
+// G > 1 layouts (several threads per column) need.
+__host__ __device__ constexpr size_t stage_offset(int groups) { return kOffCe + (groups > 1 ? kCeBytes : 0); }
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr int kBox = 256;                            // elements per TMA box row
 
@@ -140,7 +143,7 @@ __device__ __forceinline__ void consumer_barrier() {
 }
 
 template <int MODE, typename T>
-__global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a) {
+__global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kernel(const GossipArgs a) {
     using R = ModeRows<MODE>;
     using E = Elem<T>;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -150,7 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1) gossip_kernel(const GossipArgs a)
     double *red = reinterpret_cast<double *>(smem + kOffRed);
     volatile int *flags = reinterpret_cast<volatile int *>(smem + kOffFlags);   // [0] abort, [1] last
     float4 *cebuf = reinterpret_cast<float4 *>(smem + kOffCe);
-    T *stages = reinterpret_cast<T *>(smem + kOffStages);
+    T *stages = reinterpret_cast<T *>(smem + stage_offset(a.groups));
 
     const int n = a.n_workers;
     const int TILE = a.tile;
@@ -522,10 +525,18 @@ GossipShape gossip_shape(int n, int mode, int storage) {
     sh.block = kThreads;
     const size_t esize = storage == kStoreBF16 ? 2 : 4;
     const size_t stage = static_cast<size_t>(mode_rows(mode)) * n * sh.tile * esize;
-    const size_t budget = 232448 - kOffStages;
-    int st = static_cast<int>(budget / stage);
-    sh.stages = st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
-    sh.smem = kOffStages + sh.stages * stage;
+    const size_t off = stage_offset(sh.groups);
+    // two CTAs per SM (twice the consumer warps) when two stages fit in half
+    // of the SM's shared memory; otherwise one CTA with up to four stages
+    const size_t half = (233472 - 2 * 1024) / 2;
+    const int st2 = static_cast<int>((half - off) / stage);
+    if (mode != kOutEq2 && half > off && st2 >= 2) {
+        sh.stages = st2 > kMaxStages ? kMaxStages : st2;
+    } else {
+        const int st = static_cast<int>((232448 - off) / stage);
+        sh.stages = st < 2 ? 2 : (st > kMaxStages ? kMaxStages : st);
+    }
+    sh.smem = off + sh.stages * stage;
     return sh;
 }
 
