@@ -16,6 +16,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>   // header-only: ranges are no-ops unless a profiler is attached
+
 #include "../../include/gasloc.h"
 #include "internal.h"
 
@@ -46,6 +48,12 @@ constexpr int kMaxLocalSteps = 1024;
 constexpr int kCeRing = 4096;
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
+
+// Names the host-side span of an API call on profiler timelines.
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
 
 // Host-side conversions of the bf16 store: widening is exact; narrowing
 // rounds to nearest, ties to even (add 0x7FFF plus the lowest kept bit).
@@ -420,6 +428,7 @@ int gasloc_set_stream(gasloc_ctx *c, void *s) {
 }
 
 int gasloc_start(gasloc_ctx *c) {
+    NvtxRange r("gasloc_start");
     if (!c) return fail(GASLOC_EINVAL, "context is NULL");
     if (c->started) return fail(GASLOC_ESTATE, "context already started");
     int dev = 0;
@@ -700,6 +709,7 @@ int check_H(const gasloc_ctx *c, int32_t H) {
 extern "C" {
 
 int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
+    NvtxRange r("gasloc_local_steps");
     int rc = check_started(c);
     if (rc) return rc;
     rc = check_H(c, H);
@@ -709,12 +719,14 @@ int gasloc_local_steps(gasloc_ctx *c, int32_t H) {
 }
 
 int gasloc_gossip_round(gasloc_ctx *c) {
+    NvtxRange r("gasloc_gossip_round");
     const int rc = check_started(c);
     if (rc) return rc;
     return enqueue_gossip(c, c->stream);
 }
 
 int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) {
+    NvtxRange range("gasloc_run");
     int rc = check_started(c);
     if (rc) return rc;
     rc = check_H(c, H);
@@ -790,6 +802,7 @@ int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) 
 }
 
 int gasloc_consensus_error(gasloc_ctx *c, double *out) {
+    NvtxRange r("gasloc_consensus_error");
     int rc = check_started(c);
     if (rc) return rc;
     if (!out) return fail(GASLOC_EINVAL, "out is NULL");
