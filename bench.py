@@ -343,6 +343,9 @@ def main():
         ctx.close()
         torch.cuda.empty_cache()
         e2e = measure_e2e(g, torch, w, hp, H, K)
+        # whole job: every rank's units over the slowest rank's time
+        _, e2e["value"] = aggregate(e2e["seconds"] * 1e3, float(w.n_workers) * w.n_params * K, pg,
+                                    torch.device("cuda", local) if pg else None)
     else:
         ctx.close()
 
