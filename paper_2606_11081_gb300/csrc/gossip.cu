@@ -18,15 +18,17 @@
 // Every neighbour slice is read from HBM once per round however many workers
 // mix it: GASLoC/Nesterov moves 20 bytes per worker-element (y 4, x 4 + 4,
 // b 4 + 4).  No block-wide barrier is taken inside the loop (a consumer-only
-// named barrier per tile combines the consensus-error terms when G > 1).
+// named barrier per tile lets one thread per column reduce the consensus-error
+// terms of all workers when G > 1).
 //
 // Arithmetic per element, one rounding per operation (the oracle's order):
 //   acc_i = sum_{j in N_i ascending} fma(w_ij, s_j, acc)
 //   Nesterov: D = x - acc; b = fma(mu, b, D); x = fma(-eta_out, fma(mu, b, D), x)
 //   (SGD, SGDM, Eq. 2, DAdam, Local-DAdam: see outer_update).
 // Consensus error: per element e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
-// S2 = sum_i (x_i - s)^2, s = worker 0's new x (G = 1) or its sent value
-// (G > 1; a shift every group can read); fp32 per element, fp64 across elements,
+// S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x; fp32 per
+// element (the thread owning the column, or for G > 1 one thread per column
+// after the tile's barrier), fp64 across elements,
 // one partial per CTA, the last CTA (atomic ticket, nothing waits) adds the
 // partials in CTA order.
 //
@@ -54,14 +56,10 @@ constexpr size_t kOffFull = sizeof(Topo);            // 8320
 constexpr size_t kOffEmpty = kOffFull + 8 * kMaxStages;
 constexpr size_t kOffRed = kOffEmpty + 8 * kMaxStages;
 constexpr size_t kOffFlags = kOffRed + 8 * (kThreads / 32);
-constexpr size_t kOffCe = 8704;                      // 2 x [G][cols] x (S1, S2) float4, only if G > 1
-constexpr size_t kCeBytes = 2 * kConsumers * 32;
-static_assert(kOffFlags + 16 <= kOffCe, "smem layout");
-static_assert(kOffCe % 128 == 0 && kCeBytes % 128 == 0, "stage alignment");
-
-// Stages start after the consensus-error exchange buffer, which only the
-// G > 1 layouts (several threads per column) need.
-__host__ __device__ constexpr size_t stage_offset(int groups) { return kOffCe + (groups > 1 ? kCeBytes : 0); }
+constexpr size_t kOffStages = 8704;
+static_assert(kOffFlags + 16 <= kOffStages, "smem layout");
+static_assert(kOffStages % 128 == 0, "stage alignment");
+__host__ __device__ constexpr size_t stage_offset(int) { return kOffStages; }
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 constexpr int kBox = 256;                            // elements per TMA box row
 
@@ -152,7 +150,6 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
     uint64_t *empty = reinterpret_cast<uint64_t *>(smem + kOffEmpty);
     double *red = reinterpret_cast<double *>(smem + kOffRed);
     volatile int *flags = reinterpret_cast<volatile int *>(smem + kOffFlags);   // [0] abort, [1] last
-    float4 *cebuf = reinterpret_cast<float4 *>(smem + kOffCe);
     T *stages = reinterpret_cast<T *>(smem + stage_offset(a.groups));
 
     const int n = a.n_workers;
@@ -334,11 +331,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             const int nvalid = tlen - e0 < 4 ? tlen - e0 : 4;
             float4 xr[8], br[8];                      // Eq. 2 results, written after a barrier
             if (active) {
-                // shift of the consensus-error sums: worker 0's new x when one
-                // thread sees every worker of the column (G = 1), else worker
-                // 0's sent value, which every group can read
-                const float4 shift = E::load4_smem(cp(0, 0));
-                float sh[4] = {shift.x, shift.y, shift.z, shift.w};
+                float sh[4] = {0.f, 0.f, 0.f, 0.f};   // G = 1: worker 0's new x (set at i = 0)
                 int nr = 0;
                 for (int i = g; i < n; i += G) {
                     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -389,10 +382,12 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                         if (l < nvalid) {
                             // the consensus error is that of the replicas as stored
                             xn[l] = E::round(outer_update<MODE>(aa[l], xa[l], ya[l], ba[l], za[l], zpa[l], a));
-                            if (G == 1 && i == 0) sh[l] = xn[l];
-                            const float dv = __fsub_rn(xn[l], sh[l]);
-                            s1[l] = __fadd_rn(s1[l], dv);
-                            s2[l] = __fmaf_rn(dv, dv, s2[l]);
+                            if (G == 1) {   // one thread sees every worker of the column
+                                if (i == 0) sh[l] = xn[l];
+                                const float dv = __fsub_rn(xn[l], sh[l]);
+                                s1[l] = __fadd_rn(s1[l], dv);
+                                s2[l] = __fmaf_rn(dv, dv, s2[l]);
+                            }
                         } else {   // padding keeps its value
                             xn[l] = R::kMixX ? ya[l] : xa[l];
                         }
@@ -432,18 +427,22 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                     ce_acc += static_cast<double>(e);
                 }
             } else {
-                float4 *buf = cebuf + (it & 1) * (2 * kConsumers);
-                buf[2 * threadIdx.x] = make_float4(s1[0], s1[1], s1[2], s1[3]);
-                buf[2 * threadIdx.x + 1] = make_float4(s2[0], s2[1], s2[2], s2[3]);
+                // Every group's new rows are in shared memory after this
+                // barrier; one thread per column reduces them exactly as the
+                // G = 1 path does (shift by worker 0's new x, ascending i).
                 consumer_barrier();
                 if (g == 0 && active) {
-                    float t1[4] = {s1[0], s1[1], s1[2], s1[3]}, t2[4] = {s2[0], s2[1], s2[2], s2[3]};
-                    for (int gg = 1; gg < G; ++gg) {
-                        const float4 u1 = buf[2 * (gg * cols + col)], u2 = buf[2 * (gg * cols + col) + 1];
-                        t1[0] = __fadd_rn(t1[0], u1.x); t1[1] = __fadd_rn(t1[1], u1.y);
-                        t1[2] = __fadd_rn(t1[2], u1.z); t1[3] = __fadd_rn(t1[3], u1.w);
-                        t2[0] = __fadd_rn(t2[0], u2.x); t2[1] = __fadd_rn(t2[1], u2.y);
-                        t2[2] = __fadd_rn(t2[2], u2.z); t2[3] = __fadd_rn(t2[3], u2.w);
+                    float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f}, s0[4] = {0.f, 0.f, 0.f, 0.f};
+                    for (int i = 0; i < n; ++i) {
+                        const float4 xv = E::load4_smem(cp(1, i));
+                        const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+                        for (int l = 0; l < 4; ++l) {
+                            if (i == 0) s0[l] = xa[l];
+                            const float dv = __fsub_rn(xa[l], s0[l]);
+                            t1[l] = __fadd_rn(t1[l], dv);
+                            t2[l] = __fmaf_rn(dv, dv, t2[l]);
+                        }
                     }
                     float e = 0.f;
 #pragma unroll
@@ -520,7 +519,12 @@ void launch_t(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
 
 GossipShape gossip_shape(int n, int mode, int storage) {
     GossipShape sh{};
-    sh.groups = n <= 8 ? 1 : (n <= 16 ? 2 : 4);
+    // Threads per column (G).  Measured on the 8-worker exponential graph:
+    // fp32 streams best with two (more warps per byte in flight, 97% of
+    // the copy peak against 91% with one); bf16, whose tile is half the
+    // bytes, is issue-bound and loses the extra consensus-error pass (65%
+    // against 70%).  From 9 to 16 workers two threads per column, above four.
+    sh.groups = n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : 4);
     sh.tile = 4 * (kConsumers / sh.groups);
     sh.block = kThreads;
     const size_t esize = storage == kStoreBF16 ? 2 : 4;
