@@ -238,9 +238,12 @@ int gasloc_buffer(gasloc_ctx *ctx, int32_t which, int32_t tensor, void **dptr,
                   int64_t *worker_stride);
 
 /* Copies buffer `which` of `worker` (flat, n_params fp32 values) to or from
- * host memory (with bf16 storage: widened exactly on read, rounded to nearest
- * even on write).  In gasloc_write, worker = -1 writes every worker (x_0
- * broadcast).  Synchronising. */
+ * host memory.  With bf16 storage the values pass through an fp32 staging
+ * buffer on the device (the largest tensor, at most 32 Mi elements, taken
+ * from the context's allocator for the call) and are widened exactly on read
+ * or rounded to nearest even on write by a kernel; GASLOC_ENOMEM if the
+ * staging buffer cannot be had.  In gasloc_write, worker = -1 writes every
+ * worker (x_0 broadcast).  Synchronising. */
 int gasloc_read(gasloc_ctx *ctx, int32_t which, int32_t worker, float *host_dst);
 int gasloc_write(gasloc_ctx *ctx, int32_t which, int32_t worker, const float *host_src);
 

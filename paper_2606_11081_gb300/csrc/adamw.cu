@@ -8,15 +8,16 @@
 // One thread owns a column of 4 consecutive elements of a tile and walks the
 // active workers U at a time (fp32: U = 4, or 3 with per-worker h; bf16: 8 or
 // 6), issuing all of their loads before any arithmetic so that about 256
-// bytes of requests per thread stay in flight.  The synthetic gradient g = h (y - c) + sigma xi is formed in
-// registers; xi comes from a 32-bit counter hash of the element index and the
-// step key, so the gradient costs no memory traffic.  The step's per-worker
-// scalars (bias corrections, noise keys) come from the step table the prep
-// kernel wrote.
+// bytes of requests per thread stay in flight.  The synthetic gradient
+// g = h (y - c) + sigma xi is formed in registers; xi comes from a 32-bit
+// counter hash of the element index and the step key, so the gradient costs
+// no memory traffic.  The step's per-worker scalars (bias corrections, noise
+// keys) come from the step table the prep kernel wrote.
 //
-// Per element, in fp32 with one IEEE rounding per line (the oracle's order);
-// with bf16 storage the loads widen exactly and each stored value is rounded
-// to bf16 (nearest, ties to even):
+// Per element, in fp32 with one IEEE rounding per operation (the oracle's
+// order; pairs of lanes share f32x2 instructions, which round each lane as
+// the scalar operation does); with bf16 storage the loads widen exactly and
+// each stored value is rounded to bf16 (nearest, ties to even):
 //   d = y - c;  t = h d;  g = fma(sigma, xi, t)
 //   y = y * decay
 //   m = fma(beta1, m, (1 - beta1) g)
@@ -26,6 +27,7 @@
 #include <cuda_runtime.h>
 
 #include "elem.cuh"
+#include "f32x2.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
@@ -36,38 +38,47 @@ namespace {
 
 constexpr int kBlock = 256;   // threads; a tile is 4 * kBlock elements
 
+// Per-step constants, each in both halves of a register pair.
 struct Consts {
-    float decay, b1, b2, omb1, omb2, eps, sigma;
+    float2 decay, b1, b2, omb1, omb2, eps, sigma;
 };
 
-__device__ __forceinline__ float adamw_lane(float y, float m_in, float v_in, float c, float h,
-                                            float xi, float step, float isb, const Consts &k,
-                                            float &m_out, float &v_out) {
-    const float d = __fsub_rn(y, c);
-    const float t = __fmul_rn(h, d);
-    const float g = __fmaf_rn(k.sigma, xi, t);
-    y = __fmul_rn(y, k.decay);
-    const float m = __fmaf_rn(k.b1, m_in, __fmul_rn(k.omb1, g));
-    const float v = __fmaf_rn(k.b2, v_in, __fmul_rn(k.omb2, __fmul_rn(g, g)));
-    const float den = __fmaf_rn(__fsqrt_rn(v), isb, k.eps);
-    y = __fmaf_rn(-step, __fdiv_rn(m, den), y);
+// Two lanes of the step; each paired operation rounds each lane exactly as
+// the scalar operation does (f32x2.cuh), so the sequence is the one above.
+__device__ __forceinline__ float2 adamw_pair(float2 y, float2 m_in, float2 v_in, float2 c, float2 h, float2 xi,
+                                             float2 nstep, float2 isb, const Consts &k, float2 &m_out,
+                                             float2 &v_out) {
+    const float2 d = x2::sub(y, c);
+    const float2 t = x2::mul(h, d);
+    const float2 g = x2::fma(k.sigma, xi, t);
+    y = x2::mul(y, k.decay);
+    const float2 m = x2::fma(k.b1, m_in, x2::mul(k.omb1, g));
+    const float2 v = x2::fma(k.b2, v_in, x2::mul(k.omb2, x2::mul(g, g)));
+    const float2 den = x2::fma(make_float2(__fsqrt_rn(v.x), __fsqrt_rn(v.y)), isb, k.eps);
+    y = x2::fma(nstep, make_float2(__fdiv_rn(m.x, den.x), __fdiv_rn(m.y, den.y)), y);
     m_out = m;
     v_out = v;
     return y;
 }
 
-// xi = ((u >> 8) * 2^-23 - 1) * sqrt3: uniform on [-sqrt3, sqrt3), unit variance.
-__device__ __forceinline__ float noise_xi(uint32_t k, uint32_t klo, uint32_t khi) {
-    const float sqrt3 = static_cast<float>(1.7320508075688772);
+// xi = ((u >> 8) * 2^-23 - 1) * sqrt3: uniform on [-sqrt3, sqrt3), unit
+// variance.  (u >> 8) * 2^-23 - 1 = ((u >> 8) - 2^23) * 2^-23 exactly, and
+// sqrt3 * 2^-23 is exact, so xi = fl(((u >> 8) - 2^23) * (sqrt3 * 2^-23)):
+// the same real product rounded once.
+__device__ __forceinline__ float noise_int(uint32_t k, uint32_t klo, uint32_t khi) {
     const uint32_t u = noise_bits(k, klo, khi);
-    const float a = __fmul_rn(__uint2float_rn(u >> 8), 0x1p-23f);
-    return __fmul_rn(__fsub_rn(a, 1.0f), sqrt3);
+    return __int2float_rn(static_cast<int32_t>(u >> 8) - (1 << 23));
+}
+__device__ __forceinline__ float2 noise_pair(uint32_t k, uint32_t klo, uint32_t khi) {
+    const float scale = static_cast<float>(1.7320508075688772) * 0x1p-23f;
+    return x2::mul(make_float2(noise_int(k, klo, khi), noise_int(k + 1, klo, khi)), x2::splat(scale));
 }
 
 template <int U, bool PER_WORKER_H, typename T>
 __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     using E = Elem<T>;
-    const Consts kc{a.decay, a.beta1, a.beta2, a.omb1, a.omb2, a.eps, a.sigma};
+    const Consts kc{x2::splat(a.decay), x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1),
+                    x2::splat(a.omb2), x2::splat(a.eps), x2::splat(a.sigma)};
     // this step's per-worker scalars (written by the prep kernel) -> shared
     __shared__ StepTable tab;
     for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += blockDim.x)
@@ -114,21 +125,18 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
             for (int u = 0; u < U; ++u) {
                 if (a0 + u < a.n_active) {
                     const int i = a.worker[a0 + u];
-                    const float step = tab.step[i];
-                    const float isb = tab.isb[i];
+                    const float2 nstep = x2::splat(-tab.step[i]);
+                    const float2 isb = x2::splat(tab.isb[i]);
                     const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
                     const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
                     const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
                                  Cu = E::unpack(Cc[u]);
-                    float4 yo, mo, vo;
-                    yo.x = adamw_lane(Yu.x, Mu.x, Vu.x, Cu.x, h4.x, noise_xi(k0 + 0, klo, khi), step, isb, kc,
-                                      mo.x, vo.x);
-                    yo.y = adamw_lane(Yu.y, Mu.y, Vu.y, Cu.y, h4.y, noise_xi(k0 + 1, klo, khi), step, isb, kc,
-                                      mo.y, vo.y);
-                    yo.z = adamw_lane(Yu.z, Mu.z, Vu.z, Cu.z, h4.z, noise_xi(k0 + 2, klo, khi), step, isb, kc,
-                                      mo.z, vo.z);
-                    yo.w = adamw_lane(Yu.w, Mu.w, Vu.w, Cu.w, h4.w, noise_xi(k0 + 3, klo, khi), step, isb, kc,
-                                      mo.w, vo.w);
+                    float2 m01, v01, m23, v23;
+                    const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
+                                                  noise_pair(k0, klo, khi), nstep, isb, kc, m01, v01);
+                    const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
+                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, kc, m23, v23);
+                    const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
                         E::store4(Yw + o, yo);

@@ -43,6 +43,7 @@ struct Elem<float> {
     static __device__ __forceinline__ void store1(float *p, float v) { *p = v; }
     // the value a store keeps
     static __device__ __forceinline__ float round(float v) { return v; }
+    static __device__ __forceinline__ float2 round2(float2 v) { return v; }
 };
 
 __device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
@@ -81,6 +82,10 @@ struct Elem<bf16> {
     static __device__ __forceinline__ void store1(bf16 *p, float v) { *p = __float2bfloat16_rn(v); }
     // the value a store keeps
     static __device__ __forceinline__ float round(float v) { return __bfloat162float(__float2bfloat16_rn(v)); }
+    static __device__ __forceinline__ float2 round2(float2 v) {
+        const uint32_t u = bf_pack(v.x, v.y);
+        return make_float2(bf_lo(u), bf_hi(u));
+    }
 };
 
 template <typename T>

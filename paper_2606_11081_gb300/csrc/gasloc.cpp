@@ -55,22 +55,6 @@ struct NvtxRange {
     ~NvtxRange() { nvtxRangePop(); }
 };
 
-// Host-side conversions of the bf16 store: widening is exact; narrowing
-// rounds to nearest, ties to even (add 0x7FFF plus the lowest kept bit).
-float bf16_to_f32(uint16_t b) {
-    const uint32_t u = static_cast<uint32_t>(b) << 16;
-    float f;
-    std::memcpy(&f, &u, 4);
-    return f;
-}
-uint16_t f32_to_bf16(float f) {
-    uint32_t u;
-    std::memcpy(&u, &f, 4);
-    if ((u & 0x7F800000u) == 0x7F800000u) return static_cast<uint16_t>((u >> 16) | ((u & 0x007FFFFFu) ? 0x40u : 0u));
-    u += 0x7FFFu + ((u >> 16) & 1u);
-    return static_cast<uint16_t>(u >> 16);
-}
-
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
                                    CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -301,6 +285,30 @@ int build_topology(gasloc_ctx *c, int64_t round, const int64_t *round_ptr, Topo 
 }
 
 size_t esize_of(const gasloc_ctx *c) { return c->hp.storage == GASLOC_STORAGE_BF16 ? 2 : 4; }
+
+// fp32 staging buffer on the device for host transfers of a bf16 store: the
+// largest tensor, capped at 32 Mi elements (128 MiB).  The stream is
+// synchronized before the buffer is released.
+struct StagingBuffer {
+    static constexpr int64_t kMaxElems = int64_t(1) << 25;
+    gasloc_ctx *c;
+    float *p = nullptr;
+    int64_t elems = 0;
+    explicit StagingBuffer(gasloc_ctx *ctx, bool want = true) : c(ctx) {
+        if (!want) return;
+        int64_t mx = 1;
+        for (const TensorDesc &d : c->tens_h) mx = d.numel > mx ? d.numel : mx;
+        elems = mx < kMaxElems ? mx : kMaxElems;
+        p = static_cast<float *>(c->dalloc(static_cast<size_t>(elems) * 4));
+    }
+    ~StagingBuffer() {
+        if (!p) return;
+        cudaStreamSynchronize(c->stream);
+        c->dfree(p);
+    }
+    StagingBuffer(const StagingBuffer &) = delete;
+    StagingBuffer &operator=(const StagingBuffer &) = delete;
+};
 
 // Base address (bytes) of buffer `which` of a tensor; *stride in elements.
 char *buffer_base(const TensorDesc &d, int which, int64_t *stride) {
@@ -898,21 +906,30 @@ int gasloc_read(gasloc_ctx *c, int32_t which, int32_t worker, float *host) {
     rc = check_which_worker(c, which, worker, false);
     if (rc) return rc;
     const size_t es = esize_of(c);
-    std::vector<uint16_t> tmp;
+    if (es == 4) {
+        for (const TensorDesc &d : c->tens_h) {
+            int64_t stride = 0;
+            const char *p = buffer_base(d, which, &stride) + static_cast<size_t>(worker * stride) * es;
+            cudaError_t e = cudaMemcpyAsync(host + d.goff, p, static_cast<size_t>(d.numel) * 4,
+                                            cudaMemcpyDeviceToHost, c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
+        }
+        return sync_and_check(c);
+    }
+    // bf16 store: widen on the device into an fp32 staging buffer, copy that
+    StagingBuffer st(c);
+    if (!st.p) return fail(GASLOC_ENOMEM, "device allocation failed (staging)");
     for (const TensorDesc &d : c->tens_h) {
         int64_t stride = 0;
         const char *p = buffer_base(d, which, &stride) + static_cast<size_t>(worker * stride) * es;
-        void *dst = host + d.goff;
-        if (es == 2) {
-            tmp.resize(static_cast<size_t>(d.numel));
-            dst = tmp.data();
-        }
-        cudaError_t e = cudaMemcpyAsync(dst, p, static_cast<size_t>(d.numel) * es, cudaMemcpyDeviceToHost, c->stream);
-        if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
-        if (es == 2) {
-            rc = sync_and_check(c);
+        for (int64_t k0 = 0; k0 < d.numel; k0 += st.elems) {
+            const int64_t len = d.numel - k0 < st.elems ? d.numel - k0 : st.elems;
+            rc = launch_checked(c, launch_convert(p + static_cast<size_t>(k0) * es, st.p, len, false, c->stream),
+                                "widen kernel");
             if (rc) return rc;
-            for (int64_t k = 0; k < d.numel; ++k) host[d.goff + k] = bf16_to_f32(tmp[static_cast<size_t>(k)]);
+            cudaError_t e = cudaMemcpyAsync(host + d.goff + k0, st.p, static_cast<size_t>(len) * 4,
+                                            cudaMemcpyDeviceToHost, c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
         }
     }
     return sync_and_check(c);
@@ -927,23 +944,28 @@ int gasloc_write(gasloc_ctx *c, int32_t which, int32_t worker, const float *host
     const int32_t rows = (which == GASLOC_BUF_H && !c->hp.per_worker_h) ? 1 : c->n;
     const int32_t w0 = worker < 0 ? 0 : worker, w1 = worker < 0 ? rows : worker + 1;
     const size_t es = esize_of(c);
-    std::vector<uint16_t> tmp;
+    // bf16 store: copy fp32 into a staging buffer, narrow it on the device
+    StagingBuffer st(c, es == 2);
+    if (es == 2 && !st.p) return fail(GASLOC_ENOMEM, "device allocation failed (staging)");
     for (const TensorDesc &d : c->tens_h) {
         int64_t stride = 0;
         char *p = buffer_base(d, which, &stride);
         const size_t bytes = static_cast<size_t>(d.numel) * es;
-        const void *src = host + d.goff;
-        if (es == 2) {
-            tmp.resize(static_cast<size_t>(d.numel));
-            for (int64_t k = 0; k < d.numel; ++k) tmp[static_cast<size_t>(k)] = f32_to_bf16(host[d.goff + k]);
-            src = tmp.data();
-        }
         char *row0 = p + static_cast<size_t>(w0 * stride) * es;
-        cudaError_t e = cudaMemcpyAsync(row0, src, bytes, cudaMemcpyHostToDevice, c->stream);
-        if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
-        if (es == 2) {   // tmp is reused for the next tensor
-            e = cudaStreamSynchronize(c->stream);
-            if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+        cudaError_t e = cudaSuccess;
+        if (es == 4) {
+            e = cudaMemcpyAsync(row0, host + d.goff, bytes, cudaMemcpyHostToDevice, c->stream);
+            if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
+        } else {
+            for (int64_t k0 = 0; k0 < d.numel; k0 += st.elems) {
+                const int64_t len = d.numel - k0 < st.elems ? d.numel - k0 : st.elems;
+                e = cudaMemcpyAsync(st.p, host + d.goff + k0, static_cast<size_t>(len) * 4, cudaMemcpyHostToDevice,
+                                    c->stream);
+                if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
+                rc = launch_checked(c, launch_convert(st.p, row0 + static_cast<size_t>(k0) * es, len, true, c->stream),
+                                    "narrow kernel");
+                if (rc) return rc;
+            }
         }
         for (int32_t i = w0 + 1; i < w1; ++i) {
             e = cudaMemcpyAsync(p + static_cast<size_t>(i * stride) * es, row0, bytes, cudaMemcpyDeviceToDevice,

@@ -2,19 +2,23 @@
 // DAdam / Local-DAdam) for all workers, fused with the outer optimizer and the
 // consensus-error reduction of the new replicas.
 //
-// Pipeline (one CTA per SM, persistent, static round-robin over tiles):
-//  * one producer warp (lane j handles worker j) moves ALL data with the
-//    TMA engine: for each tile it issues one 1-D bulk copy per staged row --
-//    every worker's sent slice (y_j, or x_j if the worker took no local step)
-//    plus the worker's own rows the update needs (x_i, b_i) -- into an
-//    S-stage shared-memory ring whose "full" mbarrier counts the bytes, and
-//    after the consumers release a stage ("empty" mbarrier) it writes the
-//    updated rows back with bulk stores before refilling the stage;
+// Pipeline (persistent grid, one or two CTAs per SM, static round-robin over
+// tiles):
+//  * one producer warp moves ALL data with the TMA engine: each array of a
+//    tile goes as 2-D tensor-map boxes of [n workers x 256 elements] -- every
+//    worker's sent slice (y_j, or x_j if no worker took a local step) plus
+//    the workers' own rows the update needs (x_i, b_i) -- into an S-stage
+//    shared-memory ring whose "full" mbarrier counts the bytes (one 1-D bulk
+//    copy per worker instead when only some workers took local steps); after
+//    the consumers release a stage ("empty" mbarrier) it writes the updated
+//    rows back with box stores before refilling the stage;
 //  * 256 consumer threads never touch global memory in the loop: thread
-//    (g, c) owns 16-byte column c of the tile for workers g, g+G, ...
-//    (G = 1, 2, 4 for n <= 8, 16, 32), reads the neighbours' rows from shared
-//    memory, applies the outer update in place and accumulates the column's
-//    consensus-error terms.
+//    (g, c) owns the 4-element column c of the tile for workers g, g+G, ...
+//    (G = 1 or 2 for n <= 8, 2 for n <= 16, 4 for n <= 32), reads the
+//    neighbours' rows from shared memory, applies the outer update in place
+//    and accumulates the column's consensus-error terms.  Lanes are processed
+//    in pairs with f32x2 instructions (each lane rounded as the scalar
+//    operation would round it).
 // Every neighbour slice is read from HBM once per round however many workers
 // mix it: GASLoC/Nesterov moves 20 bytes per worker-element (y 4, x 4 + 4,
 // b 4 + 4).  No block-wide barrier is taken inside the loop (a consumer-only
@@ -24,7 +28,7 @@
 // Arithmetic per element, one rounding per operation (the oracle's order):
 //   acc_i = sum_{j in N_i ascending} fma(w_ij, s_j, acc)
 //   Nesterov: D = x - acc; b = fma(mu, b, D); x = fma(-eta_out, fma(mu, b, D), x)
-//   (SGD, SGDM, Eq. 2, DAdam, Local-DAdam: see outer_update).
+//   (SGD, SGDM, Eq. 2, DAdam, Local-DAdam: see outer_pair).
 // Consensus error: per element e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
 // S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x; fp32 per
 // element (the thread owning the column, or for G > 1 one thread per column
@@ -40,6 +44,7 @@
 #include <cuda_runtime.h>
 
 #include "elem.cuh"
+#include "f32x2.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -72,40 +77,59 @@ struct ModeRows {
     static constexpr bool kHasB = kRows == 3;
 };
 
+// Outer-step constants, each in both halves of a register pair.
+struct OuterK {
+    float2 neta_out, mu, alpha, oma, gamma, eta;
+};
+
+// Two lanes of the outer update (f32x2.cuh: each lane rounds as the scalar
+// operation would).  acc = mixed value, x = own x, y = own y (DAdam modes),
+// b = own b (updated), z / zprev = Eq. 2's z_t and z_{t-1}.
 template <int MODE>
-__device__ __forceinline__ float outer_update(float acc, float x, float y, float &b, float z,
-                                              float zprev, const GossipArgs &a) {
+__device__ __forceinline__ float2 outer_pair(float2 acc, float2 x, float2 y, float2 &b, float2 z, float2 zprev,
+                                             const OuterK &k) {
     switch (MODE) {
-    case kOutSgd: {
-        const float D = __fsub_rn(x, acc);
-        return __fmaf_rn(-a.eta_out, D, x);
-    }
+    case kOutSgd:
+        return x2::fma(k.neta_out, x2::sub(x, acc), x);
     case kOutSgdm: {
-        const float D = __fsub_rn(x, acc);
-        b = __fmaf_rn(a.mu, b, D);
-        return __fmaf_rn(-a.eta_out, b, x);
+        const float2 D = x2::sub(x, acc);
+        b = x2::fma(k.mu, b, D);
+        return x2::fma(k.neta_out, b, x);
     }
     case kOutNesterov: {
-        const float D = __fsub_rn(x, acc);
-        b = __fmaf_rn(a.mu, b, D);
-        return __fmaf_rn(-a.eta_out, __fmaf_rn(a.mu, b, D), x);
+        const float2 D = x2::sub(x, acc);
+        b = x2::fma(k.mu, b, D);
+        return x2::fma(k.neta_out, x2::fma(k.mu, b, D), x);
     }
     case kOutEq2: {
-        float xn = __fmaf_rn(a.alpha, acc, __fmul_rn(a.oma, z));
-        xn = __fmaf_rn(a.gamma, __fsub_rn(z, zprev), xn);
+        const float2 xn = x2::fma(k.alpha, acc, x2::mul(k.oma, z));
         b = z;
-        return xn;
+        return x2::fma(k.gamma, x2::sub(z, zprev), xn);
     }
     case kOutDadam:
-        return __fadd_rn(acc, __fsub_rn(y, x));
+        return x2::add(acc, x2::sub(y, x));
     default: {  // Local-DAdam
-        const float D = __fsub_rn(x, acc);
-        b = __fmaf_rn(a.mu, b, D);
-        return __fmaf_rn(-a.eta_out, __fmaf_rn(a.mu, b, D), y);
+        const float2 D = x2::sub(x, acc);
+        b = x2::fma(k.mu, b, D);
+        return x2::fma(k.neta_out, x2::fma(k.mu, b, D), y);
     }
     }
 }
 
+// Lanes at or past nvalid (>= 1) take keep's value.
+__device__ __forceinline__ float4 keep_tail(float4 v, float4 keep, int nvalid) {
+    if (nvalid < 2) v.y = keep.y;
+    if (nvalid < 3) v.z = keep.z;
+    if (nvalid < 4) v.w = keep.w;
+    return v;
+}
+
+// Consensus-error sums of two lanes: dv = x - shift, s1 += dv, s2 += dv dv.
+__device__ __forceinline__ void ce_terms(float2 x, float2 shift, float2 &s1, float2 &s2) {
+    const float2 dv = x2::sub(x, shift);
+    s1 = x2::add(s1, dv);
+    s2 = x2::fma(dv, dv, s2);
+}
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
@@ -312,6 +336,8 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         const int e0 = 4 * col;
         const int qb = e0 / kBox, rb = e0 % kBox;   // sub-box of the column, offset in it
         const float inv_n = static_cast<float>(1.0 / n);
+        const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
+                         x2::splat(a.gamma), x2::splat(a.eta)};
         for (int64_t it = 0; it < my_n; ++it) {
             const int s = static_cast<int>(it % S);
             bool ok = !flags[0];
@@ -326,31 +352,28 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             auto cp = [&](int k, int j) {
                 return st + (static_cast<size_t>(k) * NQ + qb) * n * kBox + static_cast<size_t>(j) * kBox + rb;
             };
-            float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f};
+            float2 s1a = x2::splat(0.f), s1b = s1a, s2a = s1a, s2b = s1a;   // lanes 0-1, 2-3
             const bool active = ok && e0 < tlen;
             const int nvalid = tlen - e0 < 4 ? tlen - e0 : 4;
             float4 xr[8], br[8];                      // Eq. 2 results, written after a barrier
             if (active) {
-                float sh[4] = {0.f, 0.f, 0.f, 0.f};   // G = 1: worker 0's new x (set at i = 0)
+                float4 sh = make_float4(0.f, 0.f, 0.f, 0.f);   // G = 1: worker 0's new x (set at i = 0)
                 int nr = 0;
                 for (int i = g; i < n; i += G) {
-                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                    float2 acc01 = x2::splat(0.f), acc23 = acc01;
                     const int dg = tp->deg[i];
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
-                        const float w = tp->w[i][q];
-                        float4 sj = E::load4_smem(cp(0, j));
-                        if (MODE == kOutEq2) {
+                        const float2 w = x2::splat(tp->w[i][q]);
+                        const float4 sj = E::load4_smem(cp(0, j));
+                        float2 s01 = x2::lo(sj), s23 = x2::hi(sj);
+                        if (MODE == kOutEq2) {   // z_j = x_j + eta (y_j - x_j)
                             const float4 xj = E::load4_smem(cp(1, j));
-                            sj.x = __fmaf_rn(a.eta, __fsub_rn(sj.x, xj.x), xj.x);
-                            sj.y = __fmaf_rn(a.eta, __fsub_rn(sj.y, xj.y), xj.y);
-                            sj.z = __fmaf_rn(a.eta, __fsub_rn(sj.z, xj.z), xj.z);
-                            sj.w = __fmaf_rn(a.eta, __fsub_rn(sj.w, xj.w), xj.w);
+                            s01 = x2::fma(ok2.eta, x2::sub(s01, x2::lo(xj)), x2::lo(xj));
+                            s23 = x2::fma(ok2.eta, x2::sub(s23, x2::hi(xj)), x2::hi(xj));
                         }
-                        acc.x = __fmaf_rn(w, sj.x, acc.x);
-                        acc.y = __fmaf_rn(w, sj.y, acc.y);
-                        acc.z = __fmaf_rn(w, sj.z, acc.z);
-                        acc.w = __fmaf_rn(w, sj.w, acc.w);
+                        acc01 = x2::fma(w, s01, acc01);
+                        acc23 = x2::fma(w, s23, acc23);
                     }
                     T *p0 = cp(0, i);   // mixed row i
                     T *p1 = cp(1, i);   // own x (own y in the DAdam modes)
@@ -366,34 +389,26 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                     if (R::kHasB) bo = E::load4_smem(p2);
                     if (MODE == kOutEq2) {
                         const float4 y0 = E::load4_smem(p0);
-                        zo.x = __fmaf_rn(a.eta, __fsub_rn(y0.x, xo.x), xo.x);
-                        zo.y = __fmaf_rn(a.eta, __fsub_rn(y0.y, xo.y), xo.y);
-                        zo.z = __fmaf_rn(a.eta, __fsub_rn(y0.z, xo.z), xo.z);
-                        zo.w = __fmaf_rn(a.eta, __fsub_rn(y0.w, xo.w), xo.w);
+                        zo = x2::join(x2::fma(ok2.eta, x2::sub(x2::lo(y0), x2::lo(xo)), x2::lo(xo)),
+                                      x2::fma(ok2.eta, x2::sub(x2::hi(y0), x2::hi(xo)), x2::hi(xo)));
                     }
                     const float4 zp = (MODE == kOutEq2 && first_round) ? zo : bo;
-                    const float xa[4] = {xo.x, xo.y, xo.z, xo.w}, ya[4] = {yo.x, yo.y, yo.z, yo.w};
-                    const float za[4] = {zo.x, zo.y, zo.z, zo.w}, zpa[4] = {zp.x, zp.y, zp.z, zp.w};
-                    const float aa[4] = {acc.x, acc.y, acc.z, acc.w};
-                    float ba[4] = {bo.x, bo.y, bo.z, bo.w};
-                    float xn[4];
-#pragma unroll
-                    for (int l = 0; l < 4; ++l) {
-                        if (l < nvalid) {
-                            // the consensus error is that of the replicas as stored
-                            xn[l] = E::round(outer_update<MODE>(aa[l], xa[l], ya[l], ba[l], za[l], zpa[l], a));
-                            if (G == 1) {   // one thread sees every worker of the column
-                                if (i == 0) sh[l] = xn[l];
-                                const float dv = __fsub_rn(xn[l], sh[l]);
-                                s1[l] = __fadd_rn(s1[l], dv);
-                                s2[l] = __fmaf_rn(dv, dv, s2[l]);
-                            }
-                        } else {   // padding keeps its value
-                            xn[l] = R::kMixX ? ya[l] : xa[l];
-                        }
+                    float2 b01 = x2::lo(bo), b23 = x2::hi(bo);
+                    // the consensus error is that of the replicas as stored
+                    const float2 n01 = E::round2(outer_pair<MODE>(acc01, x2::lo(xo), x2::lo(yo), b01, x2::lo(zo),
+                                                                  x2::lo(zp), ok2));
+                    const float2 n23 = E::round2(outer_pair<MODE>(acc23, x2::hi(xo), x2::hi(yo), b23, x2::hi(zo),
+                                                                  x2::hi(zp), ok2));
+                    float4 xn4 = x2::join(n01, n23), bn4 = x2::join(b01, b23);
+                    if (nvalid < 4) {   // padding keeps its value
+                        xn4 = keep_tail(xn4, R::kMixX ? yo : xo, nvalid);
+                        bn4 = keep_tail(bn4, bo, nvalid);
                     }
-                    const float4 xn4 = make_float4(xn[0], xn[1], xn[2], xn[3]);
-                    const float4 bn4 = make_float4(ba[0], ba[1], ba[2], ba[3]);
+                    if (G == 1) {   // one thread sees every worker of the column
+                        if (i == 0) sh = xn4;
+                        ce_terms(x2::lo(xn4), x2::lo(sh), s1a, s2a);
+                        ce_terms(x2::hi(xn4), x2::hi(sh), s1b, s2b);
+                    }
                     if (MODE == kOutEq2) {
                         xr[nr] = xn4;
                         br[nr] = bn4;
@@ -417,39 +432,28 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                     }
                 }
             }
-            // consensus-error terms of the column
-            if (G == 1) {
-                if (active) {
-                    float e = 0.f;
-#pragma unroll
-                    for (int l = 0; l < 4; ++l)
-                        if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
-                    ce_acc += static_cast<double>(e);
-                }
-            } else {
+            if (G > 1) {
                 // Every group's new rows are in shared memory after this
                 // barrier; one thread per column reduces them exactly as the
                 // G = 1 path does (shift by worker 0's new x, ascending i).
                 consumer_barrier();
                 if (g == 0 && active) {
-                    float t1[4] = {0.f, 0.f, 0.f, 0.f}, t2[4] = {0.f, 0.f, 0.f, 0.f}, s0[4] = {0.f, 0.f, 0.f, 0.f};
+                    const float4 x0 = E::load4_smem(cp(1, 0));
                     for (int i = 0; i < n; ++i) {
                         const float4 xv = E::load4_smem(cp(1, i));
-                        const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-                        for (int l = 0; l < 4; ++l) {
-                            if (i == 0) s0[l] = xa[l];
-                            const float dv = __fsub_rn(xa[l], s0[l]);
-                            t1[l] = __fadd_rn(t1[l], dv);
-                            t2[l] = __fmaf_rn(dv, dv, t2[l]);
-                        }
+                        ce_terms(x2::lo(xv), x2::lo(x0), s1a, s2a);
+                        ce_terms(x2::hi(xv), x2::hi(x0), s1b, s2b);
                     }
-                    float e = 0.f;
-#pragma unroll
-                    for (int l = 0; l < 4; ++l)
-                        if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(t1[l], inv_n), t1[l], t2[l]));
-                    ce_acc += static_cast<double>(e);
                 }
+            }
+            // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
+            if (active && (G == 1 || g == 0)) {
+                const float s1[4] = {s1a.x, s1a.y, s1b.x, s1b.y}, s2[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
+                float e = 0.f;
+#pragma unroll
+                for (int l = 0; l < 4; ++l)
+                    if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
+                ce_acc += static_cast<double>(e);
             }
             ptx::fence_proxy_async_smem();   // outputs visible to the bulk stores
             __syncwarp();

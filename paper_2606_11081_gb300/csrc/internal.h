@@ -159,6 +159,8 @@ cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t storage
                           int32_t worker, const int64_t *idx, int64_t n, float *out, int32_t *err,
                           cudaStream_t s);
 
+// fp32 -> bf16 (narrow, nearest even) or bf16 -> fp32 (widen) of n elements.
+cudaError_t launch_convert(const void *src, void *dst, int64_t n, bool narrow, cudaStream_t s);
 cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s);
 
 // Occupancy-derived persistent grid sizes.

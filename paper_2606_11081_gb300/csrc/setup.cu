@@ -253,6 +253,20 @@ __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t whi
     out[q] = Elem<T>::load1(static_cast<const T *>(base) + worker * stride + off);
 }
 
+// Host transfers of a bf16 store pass through an fp32 staging buffer on the
+// device: narrowing rounds to nearest, ties to even; widening is exact.
+__global__ void narrow_kernel(const float *src, bf16 *dst, int64_t n) {
+    const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t k = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; k < n; k += step)
+        dst[k] = __float2bfloat16_rn(src[k]);
+}
+
+__global__ void widen_kernel(const bf16 *src, float *dst, int64_t n) {
+    const int64_t step = static_cast<int64_t>(gridDim.x) * blockDim.x;
+    for (int64_t k = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; k < n; k += step)
+        dst[k] = __bfloat162float(src[k]);
+}
+
 // A wait on an mbarrier that nothing ever completes, through the bounded-wait
 // routine the pipeline kernels use: it must give up after limit_ns, record
 // kDevWaitTimeout and return.
@@ -311,6 +325,17 @@ cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t storage
         gather_kernel<bf16><<<grid, 256, 0, s>>>(tens, ntens, which, worker, idx, n, out, err);
     else
         gather_kernel<float><<<grid, 256, 0, s>>>(tens, ntens, which, worker, idx, n, out, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert(const void *src, void *dst, int64_t n, bool narrow, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t want = (n + 255) / 256;
+    const unsigned grid = static_cast<unsigned>(want < 152 * 16 ? want : 152 * 16);
+    if (narrow)
+        narrow_kernel<<<grid, 256, 0, s>>>(static_cast<const float *>(src), static_cast<bf16 *>(dst), n);
+    else
+        widen_kernel<<<grid, 256, 0, s>>>(static_cast<const bf16 *>(src), static_cast<float *>(dst), n);
     return cudaGetLastError();
 }
 

@@ -112,3 +112,20 @@ def test_bf16_bench_workload_full_size_sampled():
         ctx.close()
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
+
+
+def test_bf16_host_transfer_over_staging_chunks():
+    # one tensor longer than the 32 Mi-element staging buffer: two chunks
+    P = (1 << 25) + 4099
+    bits = np.array([0x3F808000, 0x3F818000, 0xBF808000, 0x7F7FFFFF, 0xFF7FFFFF, 0x7F800000,
+                     0xFF800000, 0x00000001, 0x80000001, 0x007FFFFF, 0x3F80FFFF, 0x00000000,
+                     0x80000000], np.uint32)
+    vals = np.random.default_rng(5).normal(size=P).astype(np.float32)
+    vals[:bits.size] = bits.view(np.float32)
+    vals[(1 << 25) - 2:(1 << 25) + 2] = bits[:4].view(np.float32)   # across the chunk seam
+    ref = torch.from_numpy(vals).to(torch.bfloat16).to(torch.float32).numpy()
+    with g.Context(2, P, "ring", 1, hparams=g.make_hparams(storage="bf16")) as ctx:
+        ctx.write("c", -1, vals)
+        for i in range(2):
+            got = ctx.read("c", i)
+            np.testing.assert_array_equal(got.view(np.uint32), ref.view(np.uint32))
