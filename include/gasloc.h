@@ -195,6 +195,18 @@ int gasloc_consensus_error(gasloc_ctx *ctx, double *out);
  * reduction kernel (ignores the value the last gossip round produced). */
 int gasloc_consensus_error_now(gasloc_ctx *ctx, double *out);
 
+/* The quantity gasloc_consensus_error returns, copied to host_dst (caller
+ * memory; page-locked memory keeps the copy asynchronous) on the context's
+ * stream without waiting for it: the per-round metric of a training loop
+ * can be logged without draining the GPU's queue after every round.
+ * *host_dst holds the value once the stream has passed the copy, e.g. after
+ * gasloc_synchronize; later rounds do not disturb a copy already enqueued. */
+int gasloc_consensus_error_async(gasloc_ctx *ctx, double *host_dst);
+
+/* Waits until every call enqueued on the context's stream has finished;
+ * EDEVICE if a kernel reported an error (the flag is then cleared). */
+int gasloc_synchronize(gasloc_ctx *ctx);
+
 /* Consensus error of caller-owned replicas, for callers that cannot allocate
  * device memory at the point they need it: a framework that owns all device
  * memory through its own pool (a side cudaMalloc could fail or fragment it),

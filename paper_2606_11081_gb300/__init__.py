@@ -71,6 +71,8 @@ SIGNATURES = {
     "gasloc_run": (ctypes.c_int, [_P, _I32, _I32, _DP]),
     "gasloc_consensus_error": (ctypes.c_int, [_P, _DP]),
     "gasloc_consensus_error_now": (ctypes.c_int, [_P, _DP]),
+    "gasloc_consensus_error_async": (ctypes.c_int, [_P, _P]),
+    "gasloc_synchronize": (ctypes.c_int, [_P]),
     "gasloc_consensus_error_noalloc": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P]),
     "gasloc_get_topology": (ctypes.c_int, [_P, _I64, _I32P, _FP, _I32P]),
     "gasloc_average": (ctypes.c_int, [_P, _P]),
@@ -211,6 +213,16 @@ def gasloc_consensus_error_now(ctx) -> float:
     out = ctypes.c_double()
     _check(_lib.gasloc_consensus_error_now(ctx, ctypes.byref(out)))
     return out.value
+
+
+def gasloc_consensus_error_async(ctx, host_ptr: int) -> None:
+    """Enqueues the copy of the consensus error to host address host_ptr
+    (8 bytes; pinned memory keeps it asynchronous)."""
+    _check(_lib.gasloc_consensus_error_async(ctx, ctypes.c_void_p(host_ptr)))
+
+
+def gasloc_synchronize(ctx) -> None:
+    _check(_lib.gasloc_synchronize(ctx))
 
 
 def gasloc_consensus_error_noalloc(x_ptr: int, n_workers: int, n_params: int, worker_stride: int,
@@ -400,6 +412,12 @@ class Context:
 
     def consensus_error_now(self) -> float:
         return gasloc_consensus_error_now(self.h)
+
+    def consensus_error_async(self, host_ptr: int) -> None:
+        gasloc_consensus_error_async(self.h, host_ptr)
+
+    def synchronize(self) -> None:
+        gasloc_synchronize(self.h)
 
     def topology(self, round_: int):
         return gasloc_get_topology(self.h, round_, self.n)

@@ -830,6 +830,30 @@ int gasloc_consensus_error(gasloc_ctx *c, double *out) {
     return GASLOC_OK;
 }
 
+int gasloc_consensus_error_async(gasloc_ctx *c, double *host_dst) {
+    NvtxRange r("gasloc_consensus_error_async");
+    int rc = check_started(c);
+    if (rc) return rc;
+    if (!host_dst) return fail(GASLOC_EINVAL, "host_dst is NULL");
+    const double *src = c->ce_d;
+    if (!c->ce_valid || c->round == 0) {
+        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d};
+        rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
+        if (rc) return rc;
+    } else {
+        src = c->ce_ring + (c->round - 1) % kCeRing;
+    }
+    cudaError_t e = cudaMemcpyAsync(host_dst, src, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "copying the consensus error");
+    return GASLOC_OK;
+}
+
+int gasloc_synchronize(gasloc_ctx *c) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    return sync_and_check(c);
+}
+
 int gasloc_consensus_error_now(gasloc_ctx *c, double *out) {
     int rc = check_started(c);
     if (rc) return rc;

@@ -86,3 +86,37 @@ def test_hparam_change_recaptures():
         with pytest.raises(g.GaslocError) as e:
             a.run(1, 1)
         assert e.value.code == g.ESTATE
+
+
+def test_async_consensus_error_reads():
+    """Per-round values copied without waiting equal the blocking reads of
+    the same rounds on an identical context (and the oracle's), including a
+    read before any round (standalone reduction) and one after a write of x."""
+    import torch
+    N, P, R = 8, 5 * 1024 + 3, 7
+    hp = dict(lr=2e-3, weights="metropolis", edge_prob=0.5)
+    a, st = make_pair(N, P, "exp", seed=9, hp=hp)
+    b, _ = make_pair(N, P, "exp", seed=9, hp=hp)
+    host = torch.full((R + 2,), -1.0, dtype=torch.float64, pin_memory=True)
+    base = host.data_ptr()
+    with a, b:
+        a.consensus_error_async(base)
+        want = [b.consensus_error()]
+        for r in range(R):
+            a.local_steps(2)
+            a.gossip_round()
+            a.consensus_error_async(base + 8 * (r + 1))
+            b.local_steps(2)
+            b.gossip_round()
+            want.append(b.consensus_error())
+            st.local_steps(2)
+            st.gossip_round()
+        x3 = b.read("x", 3) * np.float32(1.5)
+        a.write("x", 3, x3)
+        b.write("x", 3, x3)
+        a.consensus_error_async(base + 8 * (R + 1))
+        want.append(b.consensus_error())
+        a.synchronize()
+        got = host.numpy().tolist()
+    assert got == want
+    assert want[R] == pytest.approx(st.consensus_error(), rel=1e-5)
