@@ -92,12 +92,22 @@ WORKLOADS = {
         draw_hmax=8),
 }
 
-# A reduced copy of the benchmark workload for profiler captures: 16 Mi
-# parameters (3.2 GB of replica state, well above the 129 MB L2).
+# GPT-2 medium's position table, first layer and final norm: its tensor-list
+# layout (ragged 1024-element tensors among large ones) at 13.6 M parameters.
+GPT2_MEDIUM_1L = GPT2_MEDIUM[1:14] + GPT2_MEDIUM[-2:]
+
+# Reduced copies of the workloads for profiler captures: a few GB of replica
+# state each, well above the 129 MB L2.
 PROFILE_WORKLOADS = {
     "exp_n8_p16m": Workload(
         "exp_n8_p16m", 8, 1 << 24, "exp", 1, 10,
         hp=dict(weights="uniform", noise_sigma=0.01)),
+    "matching_n16_p8m_h8": Workload(
+        "matching_n16_p8m_h8", 16, 1 << 23, "matching", 8, 10,
+        hp=dict(weights="uniform", noise_sigma=0.05)),
+    "torus2x4_n8_gpt2m1l_h4": Workload(
+        "torus2x4_n8_gpt2m1l_h4", 8, sum(GPT2_MEDIUM_1L), "torus:2x4", 4, 10,
+        hp=dict(weights="metropolis", noise_sigma=0.01), numels=GPT2_MEDIUM_1L),
     "exp_n32_p4m_hetero": Workload(
         "exp_n32_p4m_hetero", 32, 1 << 22, "exp", -1, 10,
         hp=dict(weights="metropolis", noise_sigma=0.01, edge_prob=0.5, per_worker_h=True),
