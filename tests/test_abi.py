@@ -90,8 +90,11 @@ def test_layout_validation(lib):
 def test_calls_before_start_are_state_errors(lib):
     c = g.gasloc_init(2, 100, "ring", 1)
     try:
+        host = ctypes.c_double()
         for fn in (lambda: g.gasloc_local_steps(c, 1), lambda: g.gasloc_gossip_round(c),
-                   lambda: g.gasloc_consensus_error(c), lambda: g.gasloc_buffer(c, "x")):
+                   lambda: g.gasloc_consensus_error(c), lambda: g.gasloc_buffer(c, "x"),
+                   lambda: g.gasloc_consensus_error_async(c, ctypes.addressof(host)),
+                   lambda: g.gasloc_synchronize(c)):
             with pytest.raises(g.GaslocError) as e:
                 fn()
             assert e.value.code == g.ESTATE
