@@ -43,6 +43,8 @@
 // ticket protocol completes.
 #include <cuda_runtime.h>
 
+#include <cstddef>
+
 #include "elem.cuh"
 #include "f32x2.cuh"
 #include "internal.h"
@@ -186,10 +188,19 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
     const int NQ = TILE / kBox;   // sub-boxes per tile: kind k, sub-box q, worker j at ((k NQ + q) n + j) kBox
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    {   // neighbour table -> shared memory
-        const int *src = reinterpret_cast<const int *>(a.topo);
-        int *dst = reinterpret_cast<int *>(tp);
-        for (int q = threadIdx.x; q < static_cast<int>(sizeof(Topo) / 4); q += blockDim.x) dst[q] = src[q];
+    {   // neighbour table -> shared memory: rows 0..n-1 of nbr and w, and deg,
+        // in 16-byte pieces (one or two per thread)
+        static_assert(sizeof(Topo) % 16 == 0 && kMaxWorkers * 4 % 16 == 0, "Topo layout");
+        constexpr int kRow = kMaxWorkers * 4 / 16;                         // pieces per row
+        constexpr int kW = offsetof(Topo, w) / 16, kDeg = offsetof(Topo, deg) / 16;
+        constexpr int kAll = sizeof(Topo) / 16;
+        const int rows = n * kRow;
+        const int4 *src = reinterpret_cast<const int4 *>(a.topo);
+        int4 *dst = reinterpret_cast<int4 *>(tp);
+        for (int q = threadIdx.x; q < 2 * rows + (kAll - kDeg); q += blockDim.x) {
+            const int at = q < rows ? q : (q < 2 * rows ? kW + q - rows : kDeg + q - 2 * rows);
+            dst[at] = src[at];
+        }
     }
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
