@@ -339,6 +339,11 @@ def main():
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
     traffic = kernel_traffic(dom, w.name)
 
+    # the standalone consensus-error reduction, timed on its own
+    ce_ms = measure_ce(ctx, torch, stream, 10)
+    ce_bytes = es * N * P
+    ce_gbs = ce_bytes / (ce_ms / 1e3) / 1e9
+
     e2e = None
     if not args.no_e2e:
         ctx.close()
@@ -370,6 +375,11 @@ def main():
                         "gossip": {"gbs": gossip_gbs, "frac": gossip_gbs / peak,
                                    "frac_of_nominal_8tbs": gossip_gbs / NOMINAL_HBM_GBS,
                                    "ms_per_round": gossip_ms / K, "bytes_per_round": gossip_bytes},
+                        "ce": {"gbs": ce_gbs, "frac": ce_gbs / peak, "frac_of_nominal_8tbs": ce_gbs / NOMINAL_HBM_GBS,
+                               "ms_per_launch": ce_ms, "bytes_per_launch": ce_bytes,
+                               "traffic": kernel_traffic("ce", w.name),
+                               "note": "standalone reduction (after a direct write of x); each round's "
+                                       "value comes fused from the gossip kernel"},
                         "round": {"bytes": adamw_bytes + gossip_bytes,
                                   "gbs": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9,
                                   "frac": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / peak,
@@ -383,6 +393,27 @@ def main():
         pg.barrier()
         pg.destroy_process_group()
     return 0
+
+
+def measure_ce(ctx, torch, stream, reps):
+    """Mean duration (ms) of the standalone consensus-error reduction: once x
+    has been written directly, every read runs it.  The reads are enqueued
+    without waiting (each copies 8 bytes to pinned memory) between two events."""
+    ctx.write("x", 0, ctx.read("x", 0))   # same values; the fused value is no longer current
+    host = torch.zeros(reps + 1, dtype=torch.float64, pin_memory=True)
+    ctx.consensus_error_async(host.data_ptr())   # warm-up
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for r in range(reps):
+        ctx.consensus_error_async(host.data_ptr() + 8 * (r + 1))
+    e1.record(stream)
+    torch.cuda.synchronize()
+    vals = host.numpy()
+    if not (vals == vals[0]).all():
+        raise RuntimeError("standalone consensus-error reductions disagree")
+    return e0.elapsed_time(e1) / reps
 
 
 def measure_e2e(g, torch, w, hp, H, K):

@@ -4,7 +4,9 @@
 // load, a direct write of x, or before the first round).
 //
 // One thread owns a column of 4 elements and loads x_ik for all n workers (8
-// loads in flight per batch).  Per element the shifted one-pass form
+// loads in flight per batch; with bf16 storage the columns of two tiles are
+// loaded together, so that a thread keeps as many bytes in flight as with
+// fp32).  Per element the shifted one-pass form
 // e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with s = x_0k, in fp32.
 // Reduction: fp64 per thread, warp shuffles, one partial per CTA, the last
 // CTA adds the partials in CTA order (atomic ticket; nothing waits).  Reads
@@ -21,52 +23,81 @@ namespace {
 
 constexpr int kBlock = 256;
 
+// TPI tiles per iteration: their loads are all issued before any arithmetic
+// (bf16 takes two, so that a thread keeps as many bytes in flight as fp32).
+template <typename T> struct CeShape { static constexpr int kTiles = 1; };
+template <> struct CeShape<bf16> { static constexpr int kTiles = 2; };
+
 template <typename T>
-__global__ void __launch_bounds__(kBlock) ce_kernel(const CeArgs a) {
+__global__ void __launch_bounds__(kBlock, 3) ce_kernel(const CeArgs a) {
     using E = Elem<T>;
+    constexpr int TPI = CeShape<T>::kTiles;
     __shared__ double red[kBlock / 32];
     __shared__ int last;
     const int n = a.n_workers;
     const float inv_n = static_cast<float>(1.0 / n);
+    const int e0 = 4 * threadIdx.x;
     double acc = 0.0;
-    int32_t cur = -1;
-    TensorDesc d{};
-    for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
-        const Tile tl = a.tiles[ti];
-        const int e0 = 4 * threadIdx.x;
-        if (e0 >= tl.len) continue;
-        if (tl.tensor != cur) {
-            d = a.tens[tl.tensor];
-            cur = tl.tensor;
-        }
-        const T *X = as<T>(static_cast<const void *>(d.x));
-        const int64_t off = tl.start + e0;
-        const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-        float s1[4] = {0.f, 0.f, 0.f, 0.f}, s2[4] = {0.f, 0.f, 0.f, 0.f}, sh[4];
-        constexpr int U = 8;
-        for (int i0 = 0; i0 < n; i0 += U) {
-            float4 Xv[U];
+    for (int64_t t0 = blockIdx.x; t0 < a.ntiles; t0 += static_cast<int64_t>(TPI) * gridDim.x) {
+        const T *X[TPI];
+        int64_t off[TPI], ws[TPI];   // column start; worker i's row starts at i * ws
+        int nvalid[TPI];             // 0: this thread has no column in the tile
 #pragma unroll
-            for (int u = 0; u < U; ++u)
-                if (i0 + u < n) Xv[u] = E::load4(X + (i0 + u) * d.wstride + off);
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                if (i0 + u >= n) continue;
-                const float xa[4] = {Xv[u].x, Xv[u].y, Xv[u].z, Xv[u].w};
-#pragma unroll
-                for (int l = 0; l < 4; ++l) {
-                    if (i0 + u == 0) sh[l] = xa[l];
-                    const float dv = __fsub_rn(xa[l], sh[l]);
-                    s1[l] = __fadd_rn(s1[l], dv);
-                    s2[l] = __fmaf_rn(dv, dv, s2[l]);
+        for (int p = 0; p < TPI; ++p) {
+            const int64_t ti = t0 + static_cast<int64_t>(p) * gridDim.x;
+            nvalid[p] = 0;
+            X[p] = nullptr;
+            off[p] = ws[p] = 0;
+            if (ti < a.ntiles) {
+                const Tile tl = a.tiles[ti];
+                if (e0 < tl.len) {
+                    const TensorDesc &d = a.tens[tl.tensor];
+                    X[p] = as<T>(static_cast<const void *>(d.x));
+                    off[p] = tl.start + e0;
+                    ws[p] = d.wstride;
+                    nvalid[p] = tl.len - e0 < 4 ? tl.len - e0 : 4;
                 }
             }
         }
-        float e = 0.f;
+        float s1[TPI][4], s2[TPI][4], sh[TPI][4];
 #pragma unroll
-        for (int l = 0; l < 4; ++l)
-            if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
-        acc += static_cast<double>(e);
+        for (int p = 0; p < TPI; ++p)
+#pragma unroll
+            for (int l = 0; l < 4; ++l) s1[p][l] = s2[p][l] = sh[p][l] = 0.f;
+        constexpr int U = 8;
+        for (int i0 = 0; i0 < n; i0 += U) {
+            typename E::Raw Xv[TPI][U];
+#pragma unroll
+            for (int p = 0; p < TPI; ++p)
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+                    if (nvalid[p] && i0 + u < n) Xv[p][u] = E::load_raw(X[p] + (i0 + u) * ws[p] + off[p]);
+#pragma unroll
+            for (int p = 0; p < TPI; ++p) {
+                if (!nvalid[p]) continue;
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    if (i0 + u >= n) continue;
+                    const float4 xv = E::unpack(Xv[p][u]);
+                    const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+                    for (int l = 0; l < 4; ++l) {
+                        if (i0 + u == 0) sh[p][l] = xa[l];
+                        const float dv = __fsub_rn(xa[l], sh[p][l]);
+                        s1[p][l] = __fadd_rn(s1[p][l], dv);
+                        s2[p][l] = __fmaf_rn(dv, dv, s2[p][l]);
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int p = 0; p < TPI; ++p) {
+            float e = 0.f;
+#pragma unroll
+            for (int l = 0; l < 4; ++l)
+                if (l < nvalid[p]) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[p][l], inv_n), s1[p][l], s2[p][l]));
+            acc += static_cast<double>(e);
+        }
     }
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
