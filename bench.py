@@ -339,6 +339,10 @@ def main():
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
     traffic = kernel_traffic(dom, w.name)
 
+    # the network average (Algorithm 1's output), timed on its own
+    avg_ms = measure_average(g, ctx, torch, stream, P, 5)
+    avg_bytes = es * N * P + 4 * P
+    avg_gbs = avg_bytes / (avg_ms / 1e3) / 1e9
     # the standalone consensus-error reduction, timed on its own
     ce_ms = measure_ce(ctx, torch, stream, 10)
     ce_bytes = es * N * P
@@ -380,6 +384,11 @@ def main():
                                "traffic": kernel_traffic("ce", w.name),
                                "note": "standalone reduction (after a direct write of x); each round's "
                                        "value comes fused from the gossip kernel"},
+                        "average": {"gbs": avg_gbs, "frac": avg_gbs / peak,
+                                    "frac_of_nominal_8tbs": avg_gbs / NOMINAL_HBM_GBS,
+                                    "ms_per_launch": avg_ms, "bytes_per_launch": avg_bytes,
+                                    "traffic": kernel_traffic("average", w.name),
+                                    "note": "network average x-bar (end of a run)"},
                         "round": {"bytes": adamw_bytes + gossip_bytes,
                                   "gbs": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9,
                                   "frac": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / peak,
@@ -393,6 +402,21 @@ def main():
         pg.barrier()
         pg.destroy_process_group()
     return 0
+
+
+def measure_average(g, ctx, torch, stream, P, reps):
+    """Mean duration (ms) of the network-average kernel into a device buffer."""
+    dst = torch.empty(P, dtype=torch.float32, device="cuda")
+    g.gasloc_average(ctx.h, dst.data_ptr())   # warm-up
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(reps):
+        g.gasloc_average(ctx.h, dst.data_ptr())
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
 
 
 def measure_ce(ctx, torch, stream, reps):

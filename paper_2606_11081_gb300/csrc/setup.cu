@@ -201,21 +201,49 @@ __global__ void prep_kernel(const PrepArgs a) {
     a.state->p2[i] = p2;
 }
 
-// xbar = (1/n) sum_i x_i: fp32 sum in ascending i, times fl32(1/n); fp32 out.
+// xbar = (1/n) sum_i x_i: per element an fp32 sum in ascending i, times
+// fl32(1/n); fp32 out.  One thread owns a column of 4 elements of a tile and
+// loads all n workers' values of it, 8 workers at a time (their loads issued
+// together).  The output is stored as one 16-byte vector where its address
+// allows (tensor offsets in a list layout can be odd), else element by element.
 template <typename T>
-__global__ void average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
-                               float *dst) {
+__global__ void __launch_bounds__(256) average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
+                                                      int32_t n, float *dst) {
     using E = Elem<T>;
     const float inv_n = static_cast<float>(1.0 / n);
+    const int e0 = 4 * threadIdx.x;
     for (int64_t ti = blockIdx.x; ti < ntiles; ti += gridDim.x) {
         const Tile tl = tiles[ti];
-        const TensorDesc d = tens[tl.tensor];
+        if (e0 >= tl.len) continue;
+        const TensorDesc &d = tens[tl.tensor];
         const T *X = as<T>(static_cast<const void *>(d.x));
-        for (int e = threadIdx.x; e < tl.len; e += blockDim.x) {
-            const int64_t off = tl.start + e;
-            float s = 0.0f;
-            for (int i = 0; i < n; ++i) s = __fadd_rn(s, E::load1(X + i * d.wstride + off));
-            dst[d.goff + off] = __fmul_rn(s, inv_n);
+        const int64_t off = tl.start + e0;
+        const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
+        float s[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        constexpr int U = 8;
+        for (int i0 = 0; i0 < n; i0 += U) {
+            typename E::Raw xv[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                if (i0 + u < n) xv[u] = E::load_raw(X + (i0 + u) * d.wstride + off);
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                if (i0 + u >= n) continue;
+                const float4 v = E::unpack(xv[u]);
+                s[0] = __fadd_rn(s[0], v.x);
+                s[1] = __fadd_rn(s[1], v.y);
+                s[2] = __fadd_rn(s[2], v.z);
+                s[3] = __fadd_rn(s[3], v.w);
+            }
+        }
+        float *o = dst + d.goff + off;
+        const float4 r = make_float4(__fmul_rn(s[0], inv_n), __fmul_rn(s[1], inv_n), __fmul_rn(s[2], inv_n),
+                                     __fmul_rn(s[3], inv_n));
+        if (nvalid == 4 && (reinterpret_cast<uintptr_t>(o) & 15u) == 0) {
+            *reinterpret_cast<float4 *>(o) = r;
+        } else {
+            const float ra[4] = {r.x, r.y, r.z, r.w};
+            for (int l = 0; l < nvalid; ++l) o[l] = ra[l];
         }
     }
 }

@@ -190,6 +190,25 @@ def test_consensus_error_closed_form_and_paths():
         assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-6)
 
 
+@pytest.mark.parametrize("storage", ["f32", "bf16"])
+@pytest.mark.parametrize("numels", [None, [1000, 3, 4097, 64, 1, 2048, 5]])
+def test_average_is_the_fp32_mean_of_the_replicas(storage, numels):
+    # Per element: fp32 sum over ascending workers, then times fl32(1/n).  The
+    # tensor list puts tensors at odd offsets of the output (element stores)
+    # next to 16-byte-aligned ones (vector stores).
+    N, P = 6, 7218
+    ctx, _ = make_pair(N, P, "ring", seed=5, hp=dict(lr=2e-3, storage=storage), numels=numels)
+    with ctx:
+        ctx.local_steps(2)
+        ctx.gossip_round()
+        X = ctx.read_all("x")
+        s = np.zeros(P, np.float32)
+        for i in range(N):
+            s = (s + X[i]).astype(np.float32)
+        ref = (s * np.float32(1.0 / N)).astype(np.float32)
+        np.testing.assert_array_equal(ctx.average_host(), ref)
+
+
 # ------------------------------------------------------ layout / resume ---
 
 def test_tensor_list_equals_flat():
