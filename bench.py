@@ -64,11 +64,14 @@ def peak_hbm():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+KERNEL_SOURCE = {"adamw": "adamw.cu", "gossip": "gossip.cu", "ce": "ce.cu", "average": "setup.cu"}
+
+
 def kernel_traffic(kernel: str, workload: str):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel
-    source is unchanged since the capture (else None)."""
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's
+    source file is unchanged since the capture (else None)."""
     prof = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
-    src = os.path.join(ROOT, "paper_2606_11081_gb300", "csrc", "%s.cu" % kernel)
+    src = os.path.join(ROOT, "paper_2606_11081_gb300", "csrc", KERNEL_SOURCE[kernel])
     try:
         text = open(prof).read()
         m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
