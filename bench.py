@@ -342,6 +342,8 @@ def main():
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
     traffic = kernel_traffic(dom, w.name)
 
+    # the same rounds replayed from a CUDA graph (gasloc_run)
+    graph_ms = measure_graph(ctx, torch, stream, K, H)
     # the network average (Algorithm 1's output), timed on its own
     avg_ms = measure_average(g, ctx, torch, stream, P, 5)
     avg_bytes = es * N * P + 4 * P
@@ -397,6 +399,9 @@ def main():
                                   "frac": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / peak,
                                   "frac_of_nominal_8tbs":
                                       (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / NOMINAL_HBM_GBS}},
+            "graph": {"ms_per_step": graph_ms, "value": units / (graph_ms * K / 1e3),
+                      "note": "the same rounds through gasloc_run (one captured round replayed), "
+                              "timed after the main measurement; this GPU's replica set"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clk,
             "consensus_error": ce,
         }
@@ -405,6 +410,19 @@ def main():
         pg.barrier()
         pg.destroy_process_group()
     return 0
+
+
+def measure_graph(ctx, torch, stream, K, H):
+    """Mean round time (ms) of K rounds run by gasloc_run from its CUDA graph."""
+    ctx.run(1, H)   # capture (and one round)
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    ctx.run(K, H)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / K
 
 
 def measure_average(g, ctx, torch, stream, P, reps):
