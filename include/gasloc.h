@@ -284,6 +284,20 @@ int gasloc_load(gasloc_ctx *ctx, const char *path);
  * side of that.)  Synchronising. */
 int gasloc_selftest_bounded_wait(gasloc_ctx *ctx, int64_t limit_ns);
 
+/* Index checks, the stand-in for a memory sanitizer (none can be run on the
+ * GPUs this library targets).  The same sources built with the checks
+ * (build.build(checked=True) -> libgasloc_checked.so) test every worker row,
+ * column range, neighbour index and TMA offset a kernel uses before the
+ * access; a failed test skips the access and is reported as GASLOC_EDEVICE by
+ * the next synchronising call.  Nothing traps.  The paper has no counterpart.
+ * gasloc_checked_build returns 1 for the checked library, 0 for the normal one
+ * (whose checks compile to nothing).  gasloc_selftest_index_check evaluates
+ * one failing check on the device without touching memory: GASLOC_EDEVICE
+ * from the checked library, GASLOC_OK from the normal one; the context stays
+ * usable.  Synchronising. */
+int gasloc_checked_build(void);
+int gasloc_selftest_index_check(gasloc_ctx *ctx);
+
 /* Launch counter of the library's kernels on this context (for accounting). */
 int gasloc_launch_count(const gasloc_ctx *ctx, int64_t *count);
 

@@ -17,7 +17,9 @@ from typing import Optional, Sequence
 import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "libgasloc.so")
+# GASLOC_LIBRARY selects another build of the library (the index-checked one,
+# libgasloc_checked.so, in its tests).
+LIB_PATH = os.environ.get("GASLOC_LIBRARY") or os.path.join(HERE, "libgasloc.so")
 
 OK, EINVAL, ENOMEM, ECUDA, ESTATE, EDEVICE, EIO = 0, -1, -2, -3, -4, -5, -6
 OUTER = {"sgd": 0, "sgdm": 1, "nesterov": 2, "eq2": 3, "dadam": 4, "local_dadam": 5}
@@ -87,6 +89,8 @@ SIGNATURES = {
     "gasloc_load": (ctypes.c_int, [_P, ctypes.c_char_p]),
     "gasloc_launch_count": (ctypes.c_int, [_P, _I64P]),
     "gasloc_selftest_bounded_wait": (ctypes.c_int, [_P, _I64]),
+    "gasloc_checked_build": (ctypes.c_int, []),
+    "gasloc_selftest_index_check": (ctypes.c_int, [_P]),
     "gasloc_last_error": (ctypes.c_char_p, []),
     "gasloc_destroy": (None, [_P]),
 }
@@ -311,6 +315,17 @@ def gasloc_selftest_bounded_wait(ctx, limit_ns: int) -> int:
     """Runs the bounded-wait self-test; returns the status code (EDEVICE is
     the expected outcome: the wait expired and was reported)."""
     return _lib.gasloc_selftest_bounded_wait(ctx, limit_ns)
+
+
+def gasloc_checked_build() -> bool:
+    """True if the loaded library is the index-checked build."""
+    return bool(load_library().gasloc_checked_build())
+
+
+def gasloc_selftest_index_check(ctx) -> int:
+    """Evaluates one failing index check on the device; returns the status
+    code (EDEVICE from the checked build, OK from the normal one)."""
+    return _lib.gasloc_selftest_index_check(ctx)
 
 
 def gasloc_last_error() -> str:

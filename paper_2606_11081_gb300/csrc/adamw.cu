@@ -26,6 +26,7 @@
 //   y = fma(-step, m / den, y)
 #include <cuda_runtime.h>
 
+#include "check.cuh"
 #include "elem.cuh"
 #include "f32x2.cuh"
 #include "internal.h"
@@ -102,15 +103,17 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
         const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
         const uint32_t k0 = static_cast<uint32_t>(d.goff + off);
         float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (!PER_WORKER_H) hs = E::load4(Hh + off);
+        if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::load4(Hh + off);
 
         for (int a0 = 0; a0 < a.n_active; a0 += U) {
             // every load of the batch is issued before any arithmetic; the
             // raw words stay packed until their worker is processed
             typename E::Raw Y[U], M[U], V[U], Cc[U], Hw[U];
+            bool okr[U];   // worker row and column inside its buffers (checked build)
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                if (a0 + u < a.n_active) {
+                okr[u] = a0 + u < a.n_active && row_ok(a.worker[a0 + u], a.n_workers, off, 4, d.wstride, a.err);
+                if (okr[u]) {
                     const int i = a.worker[a0 + u];
                     const int64_t o = i * d.wstride + off;
                     const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
@@ -123,7 +126,7 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
             }
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                if (a0 + u < a.n_active) {
+                if (okr[u]) {
                     const int i = a.worker[a0 + u];
                     const float2 nstep = x2::splat(-tab.step[i]);
                     const float2 isb = x2::splat(tab.isb[i]);

@@ -13,6 +13,7 @@
 // one element per worker-element (4 or 2 bytes).
 #include <cuda_runtime.h>
 
+#include "check.cuh"
 #include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
@@ -71,7 +72,10 @@ __global__ void __launch_bounds__(kBlock, 3) ce_kernel(const CeArgs a) {
             for (int p = 0; p < TPI; ++p)
 #pragma unroll
                 for (int u = 0; u < U; ++u)
-                    if (nvalid[p] && i0 + u < n) Xv[p][u] = E::load_raw(X[p] + (i0 + u) * ws[p] + off[p]);
+                    if (nvalid[p] && i0 + u < n)
+                        Xv[p][u] = row_ok(i0 + u, n, off[p], 4, ws[p], a.err)
+                                       ? E::load_raw(X[p] + (i0 + u) * ws[p] + off[p])
+                                       : typename E::Raw{};
 #pragma unroll
             for (int p = 0; p < TPI; ++p) {
                 if (!nvalid[p]) continue;

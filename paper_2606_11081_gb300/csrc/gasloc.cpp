@@ -568,7 +568,7 @@ int gasloc_start(gasloc_ctx *c) {
     }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
 
-    InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed, c->hp.storage};
+    InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed, c->hp.storage, c->err_d};
     int rc = launch_checked(c, launch_init(ia, c->sms * 8, c->stream), "init kernel");
     if (rc) { c->release_all(); return rc; }
     c->started = true;
@@ -628,6 +628,8 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.tens = c->tens_d;
     a.tiles = c->tiles_a;
     a.ntiles = c->ntiles_a;
+    a.n_workers = c->n;
+    a.err = c->err_d;
     a.table = c->table_d;
     a.per_worker_h = hp.per_worker_h;
     a.storage = hp.storage;
@@ -816,7 +818,7 @@ int gasloc_consensus_error(gasloc_ctx *c, double *out) {
     if (!out) return fail(GASLOC_EINVAL, "out is NULL");
     const double *src = c->ce_d;
     if (!c->ce_valid || c->round == 0) {
-        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d};
+        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d, c->err_d};
         rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
         if (rc) return rc;
     } else {
@@ -837,7 +839,7 @@ int gasloc_consensus_error_async(gasloc_ctx *c, double *host_dst) {
     if (!host_dst) return fail(GASLOC_EINVAL, "host_dst is NULL");
     const double *src = c->ce_d;
     if (!c->ce_valid || c->round == 0) {
-        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d};
+        CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d, c->err_d};
         rc = launch_checked(c, launch_ce(a, c->grid_ce, 256, c->stream), "consensus-error kernel");
         if (rc) return rc;
     } else {
@@ -888,8 +890,8 @@ int gasloc_average(gasloc_ctx *c, float *dst) {
     int rc = check_started(c);
     if (rc) return rc;
     if (!dst) return fail(GASLOC_EINVAL, "dst is NULL");
-    return launch_checked(c, launch_average(c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, dst, c->sms * 8,
-                                            c->stream),
+    return launch_checked(c, launch_average(c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, dst, c->P,
+                                            c->err_d, c->sms * 8, c->stream),
                           "average kernel");
 }
 
@@ -1047,6 +1049,16 @@ int gasloc_steps_taken(const gasloc_ctx *c, int32_t worker, int64_t *steps) {
     if (worker < 0 || worker >= c->n) return fail(GASLOC_EINVAL, "worker out of range");
     *steps = c->nsteps[worker];
     return GASLOC_OK;
+}
+
+int gasloc_checked_build(void) { return checked_build(); }
+
+int gasloc_selftest_index_check(gasloc_ctx *c) {
+    int rc = check_started(c);
+    if (rc) return rc;
+    rc = launch_checked(c, launch_check_selftest(c->err_d, c->stream), "index-check self-test kernel");
+    if (rc) return rc;
+    return sync_and_check(c);
 }
 
 int gasloc_selftest_bounded_wait(gasloc_ctx *c, int64_t limit_ns) {

@@ -45,6 +45,7 @@
 
 #include <cstddef>
 
+#include "check.cuh"
 #include "elem.cuh"
 #include "f32x2.cuh"
 #include "internal.h"
@@ -260,6 +261,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             for (int o = lane; o < nops; o += 32) {
                 const int k = 1 + o / nq, q = o % nq;
                 const int arr = k == 1 ? 0 : 2;
+                if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
                 tma_store_2d(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * kBox), 0, blk(st, k, q));
             }
             bulk_commit();
@@ -304,6 +306,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             for (int o = lane; o < nbox; o += 32) {
                 const int k = o / nq, q = o % nq;
                 if (k == kvar && !uniform) continue;
+                if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
                 tma_load_2d(blk(st, k, q), tmap(tl.tensor, arr_of(k)), static_cast<int32_t>(tl.start + q * kBox), 0,
                             &full[s]);
             }
@@ -313,6 +316,9 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                     const T *src = static_cast<const T *>(fresh ? d.y : d.x) + j * d.wstride + tl.start;
                     for (int q = 0; q < nq; ++q) {
                         const int w = lenr - q * kBox < kBox ? lenr - q * kBox : kBox;
+                        if (!row_ok(j, n, tl.start + q * kBox, w, d.wstride, a.err) ||
+                            !aligned16_ok(static_cast<int64_t>(w) * sizeof(T), a.err))
+                            continue;
                         ptx::bulk_g2s(blk(st, kvar, q) + static_cast<size_t>(j) * kBox, src + q * kBox,
                                       static_cast<uint32_t>(w * sizeof(T)), &full[s]);
                     }
@@ -367,14 +373,16 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             const bool active = ok && e0 < tlen;
             const int nvalid = tlen - e0 < 4 ? tlen - e0 : 4;
             float4 xr[8], br[8];                      // Eq. 2 results, written after a barrier
+            int nr = 0;                               // Eq. 2 results held
             if (active) {
                 float4 sh = make_float4(0.f, 0.f, 0.f, 0.f);   // G = 1: worker 0's new x (set at i = 0)
-                int nr = 0;
                 for (int i = g; i < n; i += G) {
                     float2 acc01 = x2::splat(0.f), acc23 = acc01;
-                    const int dg = tp->deg[i];
+                    int dg = tp->deg[i];
+                    if (!span_ok(dg, dg + 1, kMaxWorkers, a.err)) dg = -1;
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
+                        if (!span_ok(j, j + 1, n, a.err)) continue;
                         const float2 w = x2::splat(tp->w[i][q]);
                         const float4 sj = E::load4_smem(cp(0, j));
                         float2 s01 = x2::lo(sj), s23 = x2::hi(sj);
@@ -421,6 +429,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                         ce_terms(x2::hi(xn4), x2::hi(sh), s1b, s2b);
                     }
                     if (MODE == kOutEq2) {
+                        if (!span_ok(nr, nr + 1, 8, a.err)) break;
                         xr[nr] = xn4;
                         br[nr] = bn4;
                         ++nr;
@@ -437,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                 consumer_barrier();
                 if (active) {
                     int r = 0;
-                    for (int i = g; i < n; i += G, ++r) {
+                    for (int i = g; i < n && r < nr; i += G, ++r) {
                         E::store4_smem(cp(1, i), xr[r]);
                         E::store4_smem(cp(2, i), br[r]);
                     }

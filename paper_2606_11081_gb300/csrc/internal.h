@@ -63,6 +63,7 @@ struct InitArgs {
     int32_t per_worker_h;
     uint64_t seed;
     int32_t storage;
+    int32_t *err;          // device error word (checked build)
 };
 
 // Step counters of the replicas, resident on the device so that a round can
@@ -102,6 +103,8 @@ struct AdamwArgs {
     uint32_t from_x_mask;                 // bit i: worker i starts from x
     int32_t worker[kMaxWorkers];
     float decay, beta1, beta2, omb1, omb2, eps, sigma;
+    int32_t n_workers;                    // rows of every per-worker array
+    int32_t *err;                         // device error word (checked build)
 };
 
 struct GossipArgs {
@@ -135,6 +138,7 @@ struct CeArgs {
     double *partials;
     unsigned int *ticket;
     double *ce_out;
+    int32_t *err;          // device error word (checked build)
 };
 
 // Launchers (return cudaGetLastError()).
@@ -154,7 +158,12 @@ struct GossipShape {
 GossipShape gossip_shape(int n, int mode, int storage);
 cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s);
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
-                           int32_t n_workers, int32_t storage, float *dst, int grid, cudaStream_t s);
+                           int32_t n_workers, int32_t storage, float *dst, int64_t n_params, int32_t *err,
+                           int grid, cudaStream_t s);
+// 1 if this library was built with the index checks, else 0; the self-test
+// evaluates one failing row check (no memory access) on the device.
+int checked_build();
+cudaError_t launch_check_selftest(int32_t *err, cudaStream_t s);
 cudaError_t launch_gather(const TensorDesc *tens, int32_t ntens, int32_t storage, int32_t which,
                           int32_t worker, const int64_t *idx, int64_t n, float *out, int32_t *err,
                           cudaStream_t s);

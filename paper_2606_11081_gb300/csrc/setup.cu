@@ -3,6 +3,7 @@
 // Algorithm 1) and an index gather used for sampled checks.
 #include <cuda_runtime.h>
 
+#include "check.cuh"
 #include "elem.cuh"
 #include "internal.h"
 #include "ptx.cuh"
@@ -43,6 +44,7 @@ __global__ void init_kernel(const InitArgs a) {
             const uint64_t k = static_cast<uint64_t>(d.goff + off);
             const float x0 = __fmul_rn(x0std, normal_std(a.seed, kTagX0, 0, k));
             for (int i = 0; i < a.n_workers; ++i) {
+                if (!row_ok(i, a.n_workers, off, 1, d.wstride, a.err)) continue;
                 const int64_t o = i * d.wstride + off;
                 E::store1(X + o, x0);
                 E::store1(Y + o, x0);
@@ -50,7 +52,8 @@ __global__ void init_kernel(const InitArgs a) {
             }
             const int nh = a.per_worker_h ? a.n_workers : 1;
             for (int i = 0; i < nh; ++i)
-                E::store1(Hh + i * d.hstride + off, curvature(a.seed, static_cast<uint64_t>(i), k));
+                if (row_ok(i, nh, off, 1, a.per_worker_h ? d.hstride : d.wstride, a.err))
+                    E::store1(Hh + i * d.hstride + off, curvature(a.seed, static_cast<uint64_t>(i), k));
         }
     }
 }
@@ -208,7 +211,7 @@ __global__ void prep_kernel(const PrepArgs a) {
 // allows (tensor offsets in a list layout can be odd), else element by element.
 template <typename T>
 __global__ void __launch_bounds__(256) average_kernel(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
-                                                      int32_t n, float *dst) {
+                                                      int32_t n, float *dst, int64_t n_params, int32_t *err) {
     using E = Elem<T>;
     const float inv_n = static_cast<float>(1.0 / n);
     const int e0 = 4 * threadIdx.x;
@@ -225,7 +228,9 @@ __global__ void __launch_bounds__(256) average_kernel(const TensorDesc *tens, co
             typename E::Raw xv[U];
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                if (i0 + u < n) xv[u] = E::load_raw(X + (i0 + u) * d.wstride + off);
+                if (i0 + u < n)
+                    xv[u] = row_ok(i0 + u, n, off, 4, d.wstride, err) ? E::load_raw(X + (i0 + u) * d.wstride + off)
+                                                                     : typename E::Raw{};
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 if (i0 + u >= n) continue;
@@ -236,6 +241,7 @@ __global__ void __launch_bounds__(256) average_kernel(const TensorDesc *tens, co
                 s[3] = __fadd_rn(s[3], v.w);
             }
         }
+        if (!span_ok(d.goff + off, d.goff + off + nvalid, n_params, err)) continue;
         float *o = dst + d.goff + off;
         const float4 r = make_float4(__fmul_rn(s[0], inv_n), __fmul_rn(s[1], inv_n), __fmul_rn(s[2], inv_n),
                                      __fmul_rn(s[3], inv_n));
@@ -295,6 +301,15 @@ __global__ void widen_kernel(const bf16 *src, float *dst, int64_t n) {
         dst[k] = __bfloat162float(src[k]);
 }
 
+// Evaluates one row check that fails (row n of an n-row buffer) without
+// touching memory: in the checked build it must record kDevBadIndex.
+__global__ void check_selftest_kernel(int32_t *err) {
+    if (threadIdx.x == 0) {
+        const int64_t rows = 4, stride = 64;
+        (void)row_ok(rows, rows, 0, 4, stride, err);
+    }
+}
+
 // A wait on an mbarrier that nothing ever completes, through the bounded-wait
 // routine the pipeline kernels use: it must give up after limit_ns, record
 // kDevWaitTimeout and return.
@@ -336,11 +351,18 @@ cudaError_t launch_prep(const PrepArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles, int32_t n,
-                           int32_t storage, float *dst, int grid, cudaStream_t s) {
+                           int32_t storage, float *dst, int64_t n_params, int32_t *err, int grid, cudaStream_t s) {
     if (storage == kStoreBF16)
-        average_kernel<bf16><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
+        average_kernel<bf16><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst, n_params, err);
     else
-        average_kernel<float><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst);
+        average_kernel<float><<<grid, 256, 0, s>>>(tens, tiles, ntiles, n, dst, n_params, err);
+    return cudaGetLastError();
+}
+
+int checked_build() { return kChecked ? 1 : 0; }
+
+cudaError_t launch_check_selftest(int32_t *err, cudaStream_t s) {
+    check_selftest_kernel<<<1, 32, 0, s>>>(err);
     return cudaGetLastError();
 }
 
