@@ -4,7 +4,8 @@ offset tested before the access (a failed test skips the access and is
 reported as GASLOC_EDEVICE).  Its self-test must see a failing check, and the
 GPU parity suites run against it must pass -- no kernel addressed anything
 outside its buffers on any of their cases (ragged tails, tensor lists, odd
-sizes, random graphs, per-worker steps, bf16)."""
+sizes, random graphs, per-worker steps, bf16, every workload at full size and
+the largest replica the ABI accepts)."""
 import os
 import subprocess
 import sys
@@ -60,7 +61,7 @@ def test_checked_build_reports_a_failing_check(checked_lib):
 
 def test_parity_suites_under_index_checks(checked_lib):
     suites = ["tests/test_gpu_parity.py", "tests/test_gpu_bf16.py", "tests/test_gpu_run.py",
-              "tests/test_gpu_failure.py", "tests/test_gpu_properties.py"]
+              "tests/test_gpu_failure.py", "tests/test_gpu_properties.py", "tests/test_gpu_fullsize.py"]
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-m", "gpu", "-p", "no:cacheprovider"] + suites,
                        env=_env(checked_lib), cwd=ROOT, capture_output=True, text=True, timeout=1200)
     assert r.returncode == 0, r.stdout[-4000:] + r.stderr[-2000:]
