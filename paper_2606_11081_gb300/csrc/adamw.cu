@@ -39,6 +39,12 @@ namespace {
 
 constexpr int kBlock = 256;   // threads; a tile is 4 * kBlock elements
 
+// Cache policies of the global accesses.  Caching in L2 (.cg) rather than
+// marking the lines evict-first measured 4% faster on the 8-worker GPT-2-small
+// workload (1.008 against 0.966 of the copy peak) and 2% on the 16-worker one.
+constexpr Cache kLdIterate = Cache::kL2, kLdMoments = Cache::kL2, kLdCentre = Cache::kL2, kLdCurv = Cache::kL2;
+constexpr Cache kSt = Cache::kL2;
+
 // Per-step constants, each in both halves of a register pair.
 struct Consts {
     float2 decay, b1, b2, omb1, omb2, eps, sigma;
@@ -103,7 +109,7 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
         const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
         const uint32_t k0 = static_cast<uint32_t>(d.goff + off);
         float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::load4(Hh + off);
+        if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::template load4<kLdCurv>(Hh + off);
 
         for (int a0 = 0; a0 < a.n_active; a0 += U) {
             // every load of the batch is issued before any arithmetic; the
@@ -117,11 +123,11 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const int i = a.worker[a0 + u];
                     const int64_t o = i * d.wstride + off;
                     const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
-                    Y[u] = E::load_raw(src + o);
-                    M[u] = E::load_raw(Mw + o);
-                    V[u] = E::load_raw(Vw + o);
-                    Cc[u] = E::load_raw(C + o);
-                    if (PER_WORKER_H) Hw[u] = E::load_raw(Hh + i * d.hstride + off);
+                    Y[u] = E::template load_raw<kLdIterate>(src + o);
+                    M[u] = E::template load_raw<kLdMoments>(Mw + o);
+                    V[u] = E::template load_raw<kLdMoments>(Vw + o);
+                    Cc[u] = E::template load_raw<kLdCentre>(C + o);
+                    if (PER_WORKER_H) Hw[u] = E::template load_raw<kLdCurv>(Hh + i * d.hstride + off);
                 }
             }
 #pragma unroll
@@ -142,9 +148,9 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
-                        E::store4(Yw + o, yo);
-                        E::store4(Mw + o, mo);
-                        E::store4(Vw + o, vo);
+                        E::template store4<kSt>(Yw + o, yo);
+                        E::template store4<kSt>(Mw + o, mo);
+                        E::template store4<kSt>(Vw + o, vo);
                     } else {
                         const float ya[4] = {yo.x, yo.y, yo.z, yo.w};
                         const float ma[4] = {mo.x, mo.y, mo.z, mo.w};

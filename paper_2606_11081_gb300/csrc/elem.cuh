@@ -4,7 +4,7 @@
 // Widening bf16 -> fp32 is exact (the bf16 bits are the top half of the
 // fp32); narrowing rounds to nearest, ties to even (__float2bfloat16_rn).
 // Vector accesses move 4 consecutive elements (16 bytes of fp32, 8 bytes of
-// bf16) with streaming (evict-first) cache hints.
+// bf16) with the cache policy the calling kernel names (default evict-first).
 #pragma once
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -15,6 +15,28 @@ namespace gasloc {
 
 using bf16 = __nv_bfloat16;
 
+// Cache policy of a global access: kStream marks the lines evict-first
+// (ld/st.global.cs), kL2 caches them in L2 only (ld/st.global.cg), kLast
+// marks a load as the last use of its line (ld.global.lu).
+enum class Cache { kStream, kL2, kLast };
+
+template <Cache C, typename V>
+__device__ __forceinline__ V ld_global(const V *p) {
+    if constexpr (C == Cache::kL2)
+        return __ldcg(p);
+    else if constexpr (C == Cache::kLast)
+        return __ldlu(p);
+    else
+        return __ldcs(p);
+}
+template <Cache C, typename V>
+__device__ __forceinline__ void st_global(V *p, V v) {
+    if constexpr (C == Cache::kL2)
+        __stcg(p, v);
+    else
+        __stcs(p, v);
+}
+
 template <typename T>
 struct Elem;
 
@@ -23,15 +45,18 @@ struct Elem<float> {
     static constexpr int kBytes = 4;
     // 4 elements as loaded (kept in registers until used)
     using Raw = float4;
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ Raw load_raw(const float *p) {
-        return __ldcs(reinterpret_cast<const float4 *>(p));
+        return ld_global<C>(reinterpret_cast<const float4 *>(p));
     }
     static __device__ __forceinline__ float4 unpack(Raw r) { return r; }
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ float4 load4(const float *p) {
-        return __ldcs(reinterpret_cast<const float4 *>(p));
+        return ld_global<C>(reinterpret_cast<const float4 *>(p));
     }
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ void store4(float *p, float4 v) {
-        __stcs(reinterpret_cast<float4 *>(p), v);
+        st_global<C>(reinterpret_cast<float4 *>(p), v);
     }
     static __device__ __forceinline__ float4 load4_smem(const float *p) {
         return *reinterpret_cast<const float4 *>(p);
@@ -58,18 +83,20 @@ template <>
 struct Elem<bf16> {
     static constexpr int kBytes = 2;
     using Raw = uint2;
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ Raw load_raw(const bf16 *p) {
-        return __ldcs(reinterpret_cast<const uint2 *>(p));
+        return ld_global<C>(reinterpret_cast<const uint2 *>(p));
     }
     static __device__ __forceinline__ float4 unpack(Raw u) {
         return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
     }
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ float4 load4(const bf16 *p) {
-        const uint2 u = __ldcs(reinterpret_cast<const uint2 *>(p));
-        return make_float4(bf_lo(u.x), bf_hi(u.x), bf_lo(u.y), bf_hi(u.y));
+        return unpack(ld_global<C>(reinterpret_cast<const uint2 *>(p)));
     }
+    template <Cache C = Cache::kStream>
     static __device__ __forceinline__ void store4(bf16 *p, float4 v) {
-        __stcs(reinterpret_cast<uint2 *>(p), make_uint2(bf_pack(v.x, v.y), bf_pack(v.z, v.w)));
+        st_global<C>(reinterpret_cast<uint2 *>(p), make_uint2(bf_pack(v.x, v.y), bf_pack(v.z, v.w)));
     }
     static __device__ __forceinline__ float4 load4_smem(const bf16 *p) {
         const uint2 u = *reinterpret_cast<const uint2 *>(p);
