@@ -157,6 +157,48 @@ __device__ __forceinline__ void tma_store_2d(const void *tmap, int32_t c0, int32
                  "r"(c1), "r"(ptx::smem_addr(src_smem))
                  : "memory");
 }
+// L2 policies of the TMA copies: 0 = no hint, 1 = evict first, 2 = evict
+// last, 3 = evict normal (createpolicy, the whole line range).  Measured on
+// the 8-worker GPT-2-small workload: evict-last loads and stores 0.987 of the
+// copy peak, no hint 0.972, evict-first 0.963 (the 16- and 32-worker
+// workloads: equal or slightly better with evict-last).
+constexpr int kLoadPolicy = 2, kStorePolicy = 2;
+template <int P>
+__device__ __forceinline__ uint64_t l2_policy() {
+    uint64_t pol = 0;
+    if constexpr (P == 1)
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    else if constexpr (P == 2)
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+    else if constexpr (P == 3)
+        asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+template <int P>
+__device__ __forceinline__ void tma_load_2d_p(void *dst_smem, const void *tmap, int32_t c0, int32_t c1, uint64_t *bar,
+                                              uint64_t pol) {
+    if constexpr (P == 0) {
+        tma_load_2d(dst_smem, tmap, c0, c1, bar);
+    } else {
+        asm volatile(
+            "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+            " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(ptx::smem_addr(dst_smem)),
+            "l"(tmap), "r"(c0), "r"(c1), "r"(ptx::smem_addr(bar)), "l"(pol)
+            : "memory");
+    }
+}
+template <int P>
+__device__ __forceinline__ void tma_store_2d_p(const void *tmap, int32_t c0, int32_t c1, const void *src_smem,
+                                               uint64_t pol) {
+    if constexpr (P == 0) {
+        tma_store_2d(tmap, c0, c1, src_smem);
+    } else {
+        asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint [%0, {%1, %2}], [%3], %4;" ::"l"(
+                         tmap),
+                     "r"(c0), "r"(c1), "r"(ptx::smem_addr(src_smem)), "l"(pol)
+                     : "memory");
+    }
+}
 __device__ __forceinline__ void tmap_acquire(const void *tmap) {
     asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(tmap) : "memory");
 }
@@ -232,6 +274,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         // (some workers took no local step this round) go as one 1-D bulk
         // copy per worker and sub-box instead.  Waits and abort decisions are
         // warp-uniform.
+        const uint64_t ld_pol = l2_policy<kLoadPolicy>(), st_pol = l2_policy<kStorePolicy>();
         const uint32_t all_mask = n >= 32 ? 0xffffffffu : ((1u << n) - 1u);
         const bool all_fresh = (a.fresh_mask & all_mask) == all_mask;
         const bool none_fresh = (a.fresh_mask & all_mask) == 0u;
@@ -262,7 +305,8 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                 const int k = 1 + o / nq, q = o % nq;
                 const int arr = k == 1 ? 0 : 2;
                 if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
-                tma_store_2d(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * kBox), 0, blk(st, k, q));
+                tma_store_2d_p<kStorePolicy>(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * kBox), 0,
+                                             blk(st, k, q), st_pol);
             }
             bulk_commit();
         };
@@ -307,8 +351,8 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                 const int k = o / nq, q = o % nq;
                 if (k == kvar && !uniform) continue;
                 if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
-                tma_load_2d(blk(st, k, q), tmap(tl.tensor, arr_of(k)), static_cast<int32_t>(tl.start + q * kBox), 0,
-                            &full[s]);
+                tma_load_2d_p<kLoadPolicy>(blk(st, k, q), tmap(tl.tensor, arr_of(k)),
+                                           static_cast<int32_t>(tl.start + q * kBox), 0, &full[s], ld_pol);
             }
             if (!uniform) {   // per-worker source: y if the worker is fresh, else x
                 for (int j = lane; j < n; j += 32) {
