@@ -12,7 +12,8 @@
 // g = h (y - c) + sigma xi is formed in registers; xi comes from a 32-bit
 // counter hash of the element index and the step key, so the gradient costs
 // no memory traffic.  The step's per-worker scalars (bias corrections, noise
-// keys) come from the step table the prep kernel wrote.
+// keys) come from the step table; the launch's last CTA to copy it advances
+// the step counters and writes the next step's scalars.
 //
 // Per element, in fp32 with one IEEE rounding per operation (the oracle's
 // order; pairs of lanes share f32x2 instructions, which round each lane as
@@ -32,6 +33,7 @@
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
+#include "step.cuh"
 
 namespace gasloc {
 
@@ -86,11 +88,29 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     using E = Elem<T>;
     const Consts kc{x2::splat(a.decay), x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1),
                     x2::splat(a.omb2), x2::splat(a.eps), x2::splat(a.sigma)};
-    // this step's per-worker scalars (written by the prep kernel) -> shared
+    // this step's per-worker scalars -> shared
     __shared__ StepTable tab;
+    __shared__ int last_copy;
     for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += blockDim.x)
         reinterpret_cast<uint32_t *>(&tab)[q] = reinterpret_cast<const uint32_t *>(a.table)[q];
     __syncthreads();
+    // The last CTA to have copied the scalars (atomic ticket; nothing waits)
+    // advances the stepped workers' counters and writes the scalars of their
+    // next step, while the other CTAs already work on their tiles.
+    if (threadIdx.x == 0) last_copy = atomicAdd(a.ticket, 1u) == gridDim.x - 1u;
+    __syncthreads();
+    if (last_copy && threadIdx.x < 32) {
+        const int i = threadIdx.x;
+        if (i < a.n_workers && ((a.active_mask >> i) & 1u)) {
+            const int64_t n = a.state->nsteps[i] + 1;
+            const double p1 = __dmul_rn(a.state->p1[i], a.beta1d), p2 = __dmul_rn(a.state->p2[i], a.beta2d);
+            a.state->nsteps[i] = n;
+            a.state->p1[i] = p1;
+            a.state->p2[i] = p2;
+            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d), a.lr, a.seed);
+        }
+        if (i == 0) *a.ticket = 0u;
+    }
     int32_t cur = -1;
     TensorDesc d{};
     for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {

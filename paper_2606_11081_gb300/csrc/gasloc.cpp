@@ -127,7 +127,8 @@ struct gasloc_ctx {
     double *ce_d = nullptr;          // [0] standalone reduction result
     double *ce_ring = nullptr;       // consensus error of round t at [t % kCeRing]
     DevState *state_d = nullptr;     // device-resident step counters
-    StepTable *table_d = nullptr;    // scalars of the current local step
+    StepTable *table_d = nullptr;    // scalars of each worker's next local step
+    int64_t table_gen = -1;          // gen at which table_d was last refreshed
     cudaStream_t cap_stream = nullptr;
     cudaGraphExec_t graph = nullptr; // one round, captured by gasloc_run
     int32_t graph_H = 0;
@@ -617,11 +618,26 @@ int gasloc_get_local_steps(const gasloc_ctx *c, int32_t *H) {
 
 namespace {
 
+// Rewrites the step table from the device counters (every worker's next
+// step) when the hyperparameters or the counters changed since it was last
+// written by the device: after a start, gasloc_set_hparams or gasloc_load.
+int refresh_step_table(gasloc_ctx *c, cudaStream_t s) {
+    if (c->table_gen == c->gen) return GASLOC_OK;
+    const gasloc_hparams &hp = c->hp;
+    PrepArgs pa{c->state_d, c->table_d, c->n, hp.lr, hp.beta1, hp.beta2, c->seed};
+    const int rc = launch_checked(c, launch_prep(pa, s), "step-scalar kernel");
+    if (!rc) c->table_gen = c->gen;
+    return rc;
+}
+
 // Enqueues the local steps of one call on stream s and advances the host
-// mirrors (step counts, which workers are fresh).  Every step is a prep
-// launch (the step's scalars, from the device counters) and an AdamW launch.
+// mirrors (step counts, which workers are fresh).  Every step is one AdamW
+// launch: it reads the step's scalars from the table, and its last CTA to
+// read them advances the device counters and writes the next step's.
 int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     const gasloc_hparams &hp = c->hp;
+    int rc0 = refresh_step_table(c, s);
+    if (rc0) return rc0;
     int32_t hmax = H;
     if (H < 0) hmax = *std::max_element(c->Hi.begin(), c->Hi.end());
     AdamwArgs a{};
@@ -631,6 +647,12 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.n_workers = c->n;
     a.err = c->err_d;
     a.table = c->table_d;
+    a.state = c->state_d;
+    a.ticket = c->ticket + 1;   // slot 0: the gossip and consensus-error reductions
+    a.lr = hp.lr;
+    a.beta1d = hp.beta1;
+    a.beta2d = hp.beta2;
+    a.seed = c->seed;
     a.per_worker_h = hp.per_worker_h;
     a.storage = hp.storage;
     a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
@@ -640,7 +662,6 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.omb2 = static_cast<float>(1.0 - hp.beta2);
     a.eps = static_cast<float>(hp.eps);
     a.sigma = static_cast<float>(hp.noise_sigma);
-    PrepArgs pa{c->state_d, c->table_d, 0u, c->n, hp.lr, hp.beta1, hp.beta2, c->seed};
     for (int32_t st = 0; st < hmax; ++st) {
         int na = 0;
         uint32_t mask = 0;
@@ -650,12 +671,10 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
             mask |= 1u << i;
         }
         if (na == 0) continue;
-        pa.active_mask = mask;
-        int rc = launch_checked(c, launch_prep(pa, s), "step-scalar kernel");
-        if (rc) return rc;
+        a.active_mask = mask;
         a.n_active = na;
         a.from_x_mask = ~c->fresh_mask;
-        rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, s), "adamw kernel");
+        const int rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, s), "adamw kernel");
         if (rc) return rc;
         for (int q = 0; q < na; ++q) c->nsteps[a.worker[q]] += 1;
         c->fresh_mask |= mask;
@@ -753,7 +772,10 @@ int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) 
             cudaGetLastError();
             return fail(GASLOC_ECUDA, "creating the capture stream failed");
         }
-        // a static neighbour table is built once, outside the graph
+        // the step table is refreshed and a static neighbour table built
+        // outside the graph (the replayed round holds AdamW and gossip only)
+        rc = refresh_step_table(c, c->stream);
+        if (rc) return rc;
         if (c->topo_static && !c->topo_ready) {
             rc = build_topology(c, c->round, nullptr, c->topo_d, c->stream);
             if (rc) return rc;

@@ -591,8 +591,10 @@ GossipShape gossip_shape(int n, int mode, int storage) {
     // fp32 streams best with two (more warps per byte in flight, 97% of
     // the copy peak against 91% with one); bf16, whose tile is half the
     // bytes, is issue-bound and loses the extra consensus-error pass (65%
-    // against 70%).  From 9 to 16 workers two threads per column, above four.
-    sh.groups = n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : 4);
+    // against 70%).  Up to 4 workers one thread per column (the 4-worker
+    // ring: 0.51 of the copy peak against 0.48 with two, 0.36 with four).
+    // From 9 to 16 workers two threads per column, above four.
+    sh.groups = n <= 4 ? 1 : (n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : 4));
     sh.tile = 4 * (kConsumers / sh.groups);
     sh.block = kThreads;
     const size_t esize = storage == kStoreBF16 ? 2 : 4;

@@ -75,7 +75,9 @@ struct DevState {
     double p2[kMaxWorkers];           // beta2^n
 };
 
-// Per-worker scalars of the current local step (written by the prep kernel).
+// Per-worker scalars of each worker's next local step (written by the prep
+// kernel after a start, a hyperparameter change or a checkpoint load, and by
+// every AdamW launch for the workers it stepped).
 struct StepTable {
     float step[kMaxWorkers];          // fl32(lr / (1 - beta1^n))
     float isb[kMaxWorkers];           // fl32(1 / sqrt(1 - beta2^n))
@@ -84,9 +86,8 @@ struct StepTable {
 };
 
 struct PrepArgs {
-    DevState *state;
+    const DevState *state;
     StepTable *table;
-    uint32_t active_mask;             // workers taking this step
     int32_t n_workers;
     double lr, beta1, beta2;
     uint64_t seed;
@@ -96,7 +97,12 @@ struct AdamwArgs {
     const TensorDesc *tens;
     const Tile *tiles;
     int64_t ntiles;
-    const StepTable *table;
+    StepTable *table;                     // this step's scalars; the next step's on return
+    DevState *state;                      // step counters, advanced for the active workers
+    unsigned int *ticket;                 // CTAs that copied the table (returns to 0)
+    uint32_t active_mask;                 // bit i: worker i takes this step
+    double lr, beta1d, beta2d;            // for the next step's scalars
+    uint64_t seed;
     int32_t n_active;
     int32_t per_worker_h;
     int32_t storage;

@@ -8,6 +8,7 @@
 #include "internal.h"
 #include "ptx.cuh"
 #include "rng.cuh"
+#include "step.cuh"
 
 namespace gasloc {
 
@@ -183,25 +184,16 @@ __global__ void topo_kernel(const TopoSpec spec, const int64_t round_arg, const 
     }
 }
 
-// Scalars of one local step for every active worker, from the device-resident
-// counters (one warp; lane i = worker i).  Each operation is a single IEEE
-// double rounding, as the host formulas: p <- p * beta; bc = 1 - p;
-// step = fl32(lr / bc1); isb = fl32(1 / sqrt(bc2)); key = hash(seed, 4, i, n).
+// Scalars of every worker's next local step (step n_i + 1) from the
+// device-resident counters, without advancing them (one warp; lane i =
+// worker i).  Run after a start, a hyperparameter change or a checkpoint
+// load; from then on every AdamW launch advances the counters of the workers
+// it stepped and writes their next scalars itself.
 __global__ void prep_kernel(const PrepArgs a) {
     const int i = threadIdx.x;
-    if (i >= a.n_workers || !((a.active_mask >> i) & 1u)) return;
-    const int64_t n = a.state->nsteps[i] + 1;
-    const double p1 = __dmul_rn(a.state->p1[i], a.beta1);
-    const double p2 = __dmul_rn(a.state->p2[i], a.beta2);
-    const double bc1 = __dsub_rn(1.0, p1), bc2 = __dsub_rn(1.0, p2);
-    a.table->step[i] = __double2float_rn(__ddiv_rn(a.lr, bc1));
-    a.table->isb[i] = __double2float_rn(__ddiv_rn(1.0, __dsqrt_rn(bc2)));
-    const uint64_t key = hash4(a.seed, kTagNoise, static_cast<uint64_t>(i), static_cast<uint64_t>(n));
-    a.table->key_lo[i] = static_cast<uint32_t>(key);
-    a.table->key_hi[i] = static_cast<uint32_t>(key >> 32);
-    a.state->nsteps[i] = n;
-    a.state->p1[i] = p1;
-    a.state->p2[i] = p2;
+    if (i >= a.n_workers) return;
+    write_step_scalars(a.table, i, a.state->nsteps[i] + 1, __dmul_rn(a.state->p1[i], a.beta1),
+                       __dmul_rn(a.state->p2[i], a.beta2), a.lr, a.seed);
 }
 
 // Loads of the average marked as the last use of their lines (ld.global.lu):

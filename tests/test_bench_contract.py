@@ -43,7 +43,7 @@ def test_main_arm_line():
     for k in ("bound", "achieved", "peak", "unit", "frac", "traffic"):
         assert k in rf, k
     assert rf["bound"] == "hbm" and 0 < rf["frac"] < 1.2
-    assert d["gpu_launches"] == 5 * 3        # prep + AdamW + gossip per round
+    assert d["gpu_launches"] == 5 * 2        # AdamW + gossip per round
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     assert d["cpu_baseline"]["cores"] >= 1
