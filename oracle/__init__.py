@@ -110,6 +110,7 @@ class Oracle:
             "oc_create": (ctypes.c_void_p, [ctypes.POINTER(Problem), _I64P, i64]),
             "oc_destroy": (None, [ctypes.c_void_p]),
             "oc_local_steps": (ctypes.c_int, [ctypes.c_void_p, i32, _I32P]),
+            "oc_set_hparams": (None, [ctypes.c_void_p, ctypes.POINTER(Problem)]),
             "oc_gossip_round": (ctypes.c_int, [ctypes.c_void_p]),
             "oc_consensus_error": (dbl, [ctypes.c_void_p]),
             "oc_average": (None, [ctypes.c_void_p, _F64P]),
@@ -214,6 +215,11 @@ class OracleState:
             hp = _ptr(self._hi, _I32P)
         if self.orc.lib.oc_local_steps(self.h, H, hp) != 0:
             raise ValueError("oc_local_steps failed")
+
+    def set_hparams(self, pb: Problem) -> None:
+        """New optimizer hyperparameters and mixing weights for the next steps
+        (sizes, graph, seed and storage stay as created)."""
+        self.orc.lib.oc_set_hparams(self.h, ctypes.byref(pb))
 
     def gossip_round(self) -> None:
         rc = self.orc.lib.oc_gossip_round(self.h)

@@ -440,6 +440,31 @@ static void adamw_step_worker(oc_state *st, int32_t i)
     st->fresh[i] = 1;
 }
 
+/* Replaces the hyperparameters of a running state (the inner AdamW and the
+ * outer optimizer of Algorithm 1 / Eq. 2, and the mixing weights and edge
+ * probability of the sampled neighbourhoods); sizes, graph, seed, curvature
+ * layout and storage stay as created.  The next step uses the new values:
+ * its bias corrections 1 - beta^n are formed from the current betas, as
+ * every step's are. */
+void oc_set_hparams(oc_state *st, const oc_problem *pb)
+{
+    oc_problem *q = &st->pb;
+    q->weights = pb->weights;
+    q->outer_mode = pb->outer_mode;
+    q->edge_prob = pb->edge_prob;
+    q->lr = pb->lr;
+    q->beta1 = pb->beta1;
+    q->beta2 = pb->beta2;
+    q->eps = pb->eps;
+    q->weight_decay = pb->weight_decay;
+    q->noise_sigma = pb->noise_sigma;
+    q->outer_lr = pb->outer_lr;
+    q->outer_momentum = pb->outer_momentum;
+    q->eta = pb->eta;
+    q->alpha = pb->alpha;
+    q->gamma = pb->gamma;
+}
+
 /* Runs a block of local steps.  H > 0: every worker takes H steps.  H <= 0:
  * worker i takes Hi[i] steps (heterogeneous H_i, Sec. 3.2). */
 int oc_local_steps(oc_state *st, int32_t H, const int32_t *Hi)

@@ -275,6 +275,30 @@ int sync_and_check(gasloc_ctx *c) {
     return GASLOC_OK;
 }
 
+// Writes the device step counters from the host mirrors (round, step counts)
+// with beta^n formed as n successive products from 1 with the current betas,
+// as the device forms them step by step.  Waits for the stream first.
+int restore_step_counters(gasloc_ctx *c) {
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    DevState ds{};
+    ds.round = c->round;
+    for (int32_t i = 0; i < kMaxWorkers; ++i) {
+        double a = 1.0, b = 1.0;
+        const int64_t ns = i < c->n ? c->nsteps[i] : 0;
+        for (int64_t t = 0; t < ns; ++t) {
+            a *= c->hp.beta1;
+            b *= c->hp.beta2;
+        }
+        ds.nsteps[i] = ns;
+        ds.p1[i] = a;
+        ds.p2[i] = b;
+    }
+    if (cudaMemcpy(c->state_d, &ds, sizeof ds, cudaMemcpyHostToDevice) != cudaSuccess)
+        return fail(GASLOC_ECUDA, "restoring the step counters failed");
+    return GASLOC_OK;
+}
+
 int launch_checked(gasloc_ctx *c, cudaError_t e, const char *what) {
     if (e != cudaSuccess) return cuda_fail(e, what);
     ++c->launches;
@@ -393,9 +417,13 @@ int gasloc_set_hparams(gasloc_ctx *c, const gasloc_hparams *hp) {
     if (rc) return rc;
     if (c->started && (hp->per_worker_h != c->hp.per_worker_h || hp->storage != c->hp.storage))
         return fail(GASLOC_ESTATE, "per_worker_h and storage cannot change after gasloc_start");
+    const bool new_betas = c->started && (hp->beta1 != c->hp.beta1 || hp->beta2 != c->hp.beta2);
     c->hp = *hp;
     c->gen += 1;
     refresh_spec(c);
+    // bias corrections are 1 - beta^n with the current betas: re-form the
+    // device products beta^n from the step counts
+    if (new_betas) return restore_step_counters(c);
     return GASLOC_OK;
 }
 
@@ -1221,22 +1249,8 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     c->has_Hi = h.has_Hi != 0;
     c->Hi = Hi;
     c->nsteps = nsteps;
-    // device counters: beta^n by n successive products from 1, as the device does
-    DevState ds{};
-    ds.round = h.round;
-    for (int32_t i = 0; i < kMaxWorkers; ++i) {
-        double a = 1.0, b = 1.0;
-        const int64_t ns = i < c->n ? nsteps[i] : 0;
-        for (int64_t t = 0; t < ns; ++t) {
-            a *= hp.beta1;
-            b *= hp.beta2;
-        }
-        ds.nsteps[i] = ns;
-        ds.p1[i] = a;
-        ds.p2[i] = b;
-    }
-    if (cudaMemcpy(c->state_d, &ds, sizeof ds, cudaMemcpyHostToDevice) != cudaSuccess)
-        return fail(GASLOC_ECUDA, "restoring the step counters failed");
+    rc = restore_step_counters(c);
+    if (rc) return rc;
     c->gen += 1;
     c->ce_valid = false;
     refresh_spec(c);

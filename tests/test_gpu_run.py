@@ -120,3 +120,29 @@ def test_async_consensus_error_reads():
         got = host.numpy().tolist()
     assert got == want
     assert want[R] == pytest.approx(st.consensus_error(), rel=1e-5)
+
+
+def test_hparam_change_matches_oracle():
+    """lr, both betas and the outer optimizer changed between rounds: the
+    device's step scalars (the refreshed step table, the re-formed beta^n)
+    and outer update follow the oracle's bit for bit."""
+    from _pairs import oracle_problem
+    N, P = 8, 3001
+    ctx, st = make_pair(N, P, "exp", seed=17, hp=dict(lr=1e-3))
+    with ctx:
+        for _ in range(2):
+            ctx.local_steps(2)
+            ctx.gossip_round()
+            st.local_steps(2)
+            st.gossip_round()
+        full2 = dict(wl.COMMON_HP, lr=4e-3, beta1=0.8, beta2=0.99, outer="sgdm", outer_momentum=0.5)
+        ctx.set_hparams(g.make_hparams(**full2))
+        st.set_hparams(oracle_problem(N, P, "exp", 17, full2))
+        for _ in range(3):
+            ctx.local_steps(3)
+            ctx.gossip_round()
+            st.local_steps(3)
+            st.gossip_round()
+        for w in ("x", "y", "m", "v", "b"):
+            np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)
+        assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)

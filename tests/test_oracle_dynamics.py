@@ -73,6 +73,41 @@ def test_adamw_state_persists_across_rounds(orc64):
         np.testing.assert_allclose(st.get("x", i), ref, rtol=1e-10, atol=1e-14)
 
 
+def test_hparam_change_follows_torch_adamw(orc64):
+    # No edges and an SGD outer step of 1 (x <- y each round): R rounds of H
+    # steps are R*H AdamW steps.  Changing lr and both betas after the first
+    # rounds matches torch.optim.AdamW with its parameter group changed at the
+    # same step (bias corrections 1 - beta^n from the current betas).
+    N, P, H, R1, R2 = 2, 16, 2, 2, 3
+    kw = dict(seed=SEED + 5, lr=2e-3, noise_sigma=0.02, outer="sgd", outer_lr=1.0, outer_momentum=0.0)
+    pb = oracle.make_problem(N, P, "none", **kw)
+    pb2 = oracle.make_problem(N, P, "none", **dict(kw, lr=5e-3, beta1=0.8, beta2=0.99))
+    st = orc64.state(pb)
+    x0, c, h = st.get("x", 0), st.get_all("c"), st.get("h", 0)
+    for _ in range(R1):
+        st.local_steps(H)
+        st.gossip_round()
+    st.set_hparams(pb2)
+    for _ in range(R2):
+        st.local_steps(H)
+        st.gossip_round()
+    for i in range(N):
+        p = torch.tensor(x0, dtype=torch.float64, requires_grad=True)
+        opt = torch.optim.AdamW([p], lr=pb.lr, betas=(pb.beta1, pb.beta2), eps=pb.eps,
+                                weight_decay=pb.weight_decay)
+        ct = torch.tensor(c[i], dtype=torch.float64)
+        ht = torch.tensor(h, dtype=torch.float64)
+        for n in range(1, (R1 + R2) * H + 1):
+            if n == R1 * H + 1:
+                opt.param_groups[0]["lr"] = pb2.lr
+                opt.param_groups[0]["betas"] = (pb2.beta1, pb2.beta2)
+            xi = torch.tensor([orc64.noise(pb.seed, i, n, k) for k in range(P)], dtype=torch.float64)
+            with torch.no_grad():
+                p.grad = ht * (p - ct) + pb.noise_sigma * xi
+            opt.step()
+        np.testing.assert_allclose(st.get("x", i), p.detach().numpy(), rtol=1e-10, atol=1e-14)
+
+
 def test_adamw_first_step_closed_form(orc64):
     # n = 1: m_hat = g, v_hat = g^2, so y1 = y0 (1 - lr wd) - lr g / (|g| + eps)
     N, P = 2, 64
