@@ -192,7 +192,7 @@ def cpu_baseline(w, seconds: float):
         st.consensus_error()
         rounds += 1
         el = time.perf_counter() - t0
-        if el >= seconds or rounds >= 1000:
+        if el >= seconds or rounds >= 100000:
             break
     value = w.n_workers * slice_p * rounds / el
     return {"value": value, "unit": UNIT, "cores": orc.lib.oc_num_threads(), "kind": "oracle",
