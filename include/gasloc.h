@@ -25,8 +25,9 @@
  *  - Work is enqueued asynchronously on the context's stream (default: the
  *    CUDA legacy default stream; see gasloc_set_stream).  Calls documented as
  *    "synchronising" wait for that stream before returning.
- *  - Floating-point parameters are fp32 on the device; host-side scalars of a
- *    step (bias corrections etc.) are computed in double and rounded once.
+ *  - Parameters are fp32 on the device (bf16 with GASLOC_STORAGE_BF16, fp32
+ *    arithmetic); the scalars of a step (bias corrections etc.) are computed
+ *    in double from device-resident step counters and rounded once.
  *  - A context is not thread-safe.  Distinct contexts are independent.
  */
 #ifndef GASLOC_H
@@ -128,10 +129,13 @@ void gasloc_default_hparams(gasloc_hparams *hp);
 int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint64_t seed,
                 gasloc_ctx **out);
 
-/* Sets the hyperparameters (copied).  Before gasloc_start any field may
- * change; afterwards per_worker_h and storage may not (ESTATE).  EINVAL if lr < 0,
- * beta not in [0,1), eps <= 0, edge_prob not in [0,1], an unknown mode or
- * weight rule, or eta/alpha/gamma/outer_lr negative. */
+/* Sets the hyperparameters (copied); the next step uses them.  Before
+ * gasloc_start any field may change; afterwards per_worker_h and storage may
+ * not (ESTATE).  Bias corrections use the betas current at each step (1 -
+ * beta^n, App. B's AdamW), so new betas on a started context re-form the
+ * device products beta^n from the step counts (this waits for the stream).
+ * EINVAL if lr < 0, beta not in [0,1), eps <= 0, edge_prob not in [0,1], an
+ * unknown mode or weight rule, or eta/alpha/gamma/outer_lr negative. */
 int gasloc_set_hparams(gasloc_ctx *ctx, const gasloc_hparams *hp);
 int gasloc_get_hparams(const gasloc_ctx *ctx, gasloc_hparams *hp);
 
