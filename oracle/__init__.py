@@ -57,6 +57,8 @@ class Problem(ctypes.Structure):
         ("outer_lr", ctypes.c_double), ("outer_momentum", ctypes.c_double),
         ("eta", ctypes.c_double), ("alpha", ctypes.c_double), ("gamma", ctypes.c_double),
         ("per_worker_h", ctypes.c_int32), ("storage", ctypes.c_int32),
+        ("lr_total_steps", ctypes.c_int64), ("lr_warmup_frac", ctypes.c_double),
+        ("lr_warmup_start", ctypes.c_double), ("lr_final_frac", ctypes.c_double),
     ]
 
 
@@ -67,14 +69,17 @@ def make_problem(n_workers: int, n_params: int, topology: str = "ring", seed: in
                  weight_decay: float = 0.1, noise_sigma: float = 0.01,
                  outer_lr: float = 0.7, outer_momentum: float = 0.9, eta: float = 1.0,
                  alpha: float = 1.0, gamma: float = 0.0, per_worker_h: bool = False,
-                 storage: str = "f32") -> Problem:
+                 storage: str = "f32", lr_total_steps: int = 0, lr_warmup_frac: float = 0.1,
+                 lr_warmup_start: float = 0.01, lr_final_frac: float = 0.0) -> Problem:
     return Problem(n_workers=n_workers, topology=TOPO[topology], n_params=n_params,
                    torus_rows=torus[0], torus_cols=torus[1], weights=WEIGHTS[weights],
                    outer_mode=OUTER[outer], seed=seed, edge_prob=edge_prob, lr=lr,
                    beta1=beta1, beta2=beta2, eps=eps, weight_decay=weight_decay,
                    noise_sigma=noise_sigma, outer_lr=outer_lr, outer_momentum=outer_momentum,
                    eta=eta, alpha=alpha, gamma=gamma, per_worker_h=int(per_worker_h),
-                   storage=STORAGE[storage])
+                   storage=STORAGE[storage], lr_total_steps=lr_total_steps,
+                   lr_warmup_frac=lr_warmup_frac, lr_warmup_start=lr_warmup_start,
+                   lr_final_frac=lr_final_frac)
 
 
 _I64P = ctypes.POINTER(ctypes.c_int64)
@@ -111,6 +116,7 @@ class Oracle:
             "oc_destroy": (None, [ctypes.c_void_p]),
             "oc_local_steps": (ctypes.c_int, [ctypes.c_void_p, i32, _I32P]),
             "oc_set_hparams": (None, [ctypes.c_void_p, ctypes.POINTER(Problem)]),
+            "oc_sched_lr": (ctypes.c_double, [ctypes.POINTER(Problem), i64]),
             "oc_gossip_round": (ctypes.c_int, [ctypes.c_void_p]),
             "oc_consensus_error": (dbl, [ctypes.c_void_p]),
             "oc_average": (None, [ctypes.c_void_p, _F64P]),
@@ -143,6 +149,10 @@ class Oracle:
 
     def noise(self, seed, i, n, k) -> float:
         return self.lib.oc_noise(seed, i, n, k)
+
+    def sched_lr(self, pb: Problem, n: int) -> float:
+        """Learning rate of a worker's n-th local step under pb's schedule."""
+        return self.lib.oc_sched_lr(ctypes.byref(pb), n)
 
     def bf16_round(self, v: float) -> float:
         return self.lib.oc_bf16_round(v)

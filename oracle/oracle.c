@@ -398,6 +398,30 @@ oc_state *oc_create(const oc_problem *pb, const int64_t *kidx, int64_t nk)
  *   den = fma(sqrt(v), isb, eps)
  *   y = fma(-step, m/den, y)
  * The first step of a round starts from x_i (x_i^{(t,0)} = x_i^{(t)}). */
+/* Learning rate of a worker's n-th local step (n >= 1).  App. B: a warm-up
+ * over the first 10% of the schedule that starts at 1% of the peak rate, then
+ * cosine decay.  Reading: with T = lr_total_steps and W = round(frac * T)
+ * warm-up steps, the rate rises linearly from warmup_start * lr at n = 1
+ * towards lr, reaches lr at n = W + 1, then follows
+ *   lr * (f + (1 - f) * (1 + cos(pi * q)) / 2),  q = (n - W - 1) / (T - W - 1),
+ * q clamped to [0, 1], so it is f * lr from n = T on.  T = 0: constant lr. */
+double oc_sched_lr(const oc_problem *pb, int64_t n)
+{
+    const int64_t T = pb->lr_total_steps;
+    if (T <= 0) return pb->lr;
+    const int64_t W = (int64_t)llround(pb->lr_warmup_frac * (double)T);
+    if (n <= W) {
+        const double s0 = pb->lr_warmup_start;
+        return pb->lr * (s0 + (1.0 - s0) * ((double)(n - 1) / (double)W));
+    }
+    const int64_t span = T - W - 1;
+    double q = span > 0 ? (double)(n - W - 1) / (double)span : 1.0;
+    if (q > 1.0) q = 1.0;
+    const double f = pb->lr_final_frac;
+    const double pi = 3.14159265358979323846;
+    return pb->lr * (f + (1.0 - f) * (0.5 * (1.0 + cos(pi * q))));
+}
+
 static void adamw_step_worker(oc_state *st, int32_t i)
 {
     const oc_problem *pb = &st->pb;
@@ -406,9 +430,10 @@ static void adamw_step_worker(oc_state *st, int32_t i)
     double p1 = 1.0, p2 = 1.0;
     for (int64_t s = 0; s < n; ++s) { p1 *= pb->beta1; p2 *= pb->beta2; }
     const double bc1 = 1.0 - p1, bc2 = 1.0 - p2;
-    const REAL step = (REAL)(pb->lr / bc1);
+    const double lr = oc_sched_lr(pb, n);
+    const REAL step = (REAL)(lr / bc1);
     const REAL isb = (REAL)(1.0 / sqrt(bc2));
-    const REAL decay = (REAL)(1.0 - pb->lr * pb->weight_decay);
+    const REAL decay = (REAL)(1.0 - lr * pb->weight_decay);
     const REAL b1 = (REAL)pb->beta1, b2 = (REAL)pb->beta2;
     const REAL omb1 = (REAL)(1.0 - pb->beta1), omb2 = (REAL)(1.0 - pb->beta2);
     const REAL eps = (REAL)pb->eps, sigma = (REAL)pb->noise_sigma;
@@ -463,6 +488,10 @@ void oc_set_hparams(oc_state *st, const oc_problem *pb)
     q->eta = pb->eta;
     q->alpha = pb->alpha;
     q->gamma = pb->gamma;
+    q->lr_total_steps = pb->lr_total_steps;
+    q->lr_warmup_frac = pb->lr_warmup_frac;
+    q->lr_warmup_start = pb->lr_warmup_start;
+    q->lr_final_frac = pb->lr_final_frac;
 }
 
 /* Runs a block of local steps.  H > 0: every worker takes H steps.  H <= 0:

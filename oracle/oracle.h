@@ -59,6 +59,11 @@ typedef struct {
     int32_t  storage;         /* OC_STORE_F32, or OC_STORE_BF16: every stored
                                  value is rounded to bfloat16 (nearest, ties
                                  to even) */
+    /* learning-rate schedule of App. B over a worker's local steps:
+     * lr_total_steps T (0: constant lr), warm-up over a fraction of T from
+     * lr_warmup_start * lr, then cosine decay to lr_final_frac * lr */
+    int64_t  lr_total_steps;
+    double   lr_warmup_frac, lr_warmup_start, lr_final_frac;
 } oc_problem;
 
 enum { OC_STORE_F32 = 0, OC_STORE_BF16 = 1 };

@@ -108,6 +108,58 @@ def test_hparam_change_follows_torch_adamw(orc64):
         np.testing.assert_allclose(st.get("x", i), p.detach().numpy(), rtol=1e-10, atol=1e-14)
 
 
+@pytest.mark.parametrize("T,frac,s0,f", [(100, 0.1, 0.01, 0.0), (37, 0.1, 0.01, 0.1), (20, 0.25, 0.05, 0.2)])
+def test_lr_schedule_shape(orc64, T, frac, s0, f):
+    # App. B: warm-up over the first 10% of the schedule starting at 1% of
+    # the peak, then cosine decay.  Values the statement fixes: the first
+    # step's rate, the peak after the warm-up, the final rate, the cosine's
+    # midpoint, monotone warm-up and decay.
+    lr = 3e-3
+    pb = oracle.make_problem(2, 8, "none", lr=lr, lr_total_steps=T, lr_warmup_frac=frac,
+                             lr_warmup_start=s0, lr_final_frac=f)
+    W = int(round(frac * T))
+    r = [orc64.sched_lr(pb, n) for n in range(1, T + 6)]
+    assert r[0] == pytest.approx(s0 * lr, rel=1e-15)
+    assert r[W] == pytest.approx(lr, rel=1e-15)                  # step W + 1
+    assert all(b > a for a, b in zip(r[:W], r[1:W + 1]))       # warm-up rises
+    assert all(b <= a for a, b in zip(r[W:], r[W + 1:]))       # then never rises
+    for n in range(T, T + 6):
+        assert r[n - 1] == pytest.approx(f * lr, rel=1e-12, abs=1e-18)
+    if (T - W - 1) % 2 == 0:                                    # cosine midpoint
+        n_mid = W + 1 + (T - W - 1) // 2
+        assert r[n_mid - 1] == pytest.approx(lr * (1 + f) / 2, rel=1e-14)
+    off = oracle.make_problem(2, 8, "none", lr=lr)              # T = 0: constant
+    assert [orc64.sched_lr(off, n) for n in (1, 5, 1000)] == [lr, lr, lr]
+
+
+def test_lr_schedule_enters_adamw_like_torch(orc64):
+    # No edges and an SGD outer step of 1: the rounds are one AdamW trajectory.
+    # torch.optim.AdamW with its group's lr set to each step's scheduled rate
+    # (step size and decoupled weight decay both scale with it) must match.
+    N, P, H, R, T = 2, 12, 3, 6, 14
+    kw = dict(seed=SEED + 9, lr=4e-3, noise_sigma=0.02, outer="sgd", outer_lr=1.0, outer_momentum=0.0,
+              lr_total_steps=T, lr_warmup_frac=0.2, lr_final_frac=0.1)
+    pb = oracle.make_problem(N, P, "none", **kw)
+    st = orc64.state(pb)
+    x0, c, h = st.get("x", 0), st.get_all("c"), st.get("h", 0)
+    for _ in range(R):
+        st.local_steps(H)
+        st.gossip_round()
+    for i in range(N):
+        p = torch.tensor(x0, dtype=torch.float64, requires_grad=True)
+        opt = torch.optim.AdamW([p], lr=pb.lr, betas=(pb.beta1, pb.beta2), eps=pb.eps,
+                                weight_decay=pb.weight_decay)
+        ct = torch.tensor(c[i], dtype=torch.float64)
+        ht = torch.tensor(h, dtype=torch.float64)
+        for n in range(1, R * H + 1):
+            opt.param_groups[0]["lr"] = orc64.sched_lr(pb, n)
+            xi = torch.tensor([orc64.noise(pb.seed, i, n, k) for k in range(P)], dtype=torch.float64)
+            with torch.no_grad():
+                p.grad = ht * (p - ct) + pb.noise_sigma * xi
+            opt.step()
+        np.testing.assert_allclose(st.get("x", i), p.detach().numpy(), rtol=1e-10, atol=1e-14)
+
+
 def test_adamw_first_step_closed_form(orc64):
     # n = 1: m_hat = g, v_hat = g^2, so y1 = y0 (1 - lr wd) - lr g / (|g| + eps)
     N, P = 2, 64
