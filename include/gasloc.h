@@ -99,6 +99,16 @@ typedef struct gasloc_hparams {
     int32_t weights;        /* GASLOC_W_*     */
     int32_t per_worker_h;   /* 1: one curvature vector per worker */
     int32_t storage;        /* GASLOC_STORAGE_F32 or GASLOC_STORAGE_BF16 */
+    /* Learning-rate schedule of the inner AdamW (App. B), applied per worker
+     * to its own local step count n: over lr_total_steps = T steps, a warm-up
+     * of round(lr_warmup_frac * T) = W steps rising linearly from
+     * lr_warmup_start * lr (n = 1) to lr (n = W + 1), then cosine decay
+     *   lr * (f + (1 - f) (1 + cos(pi q)) / 2),  q = (n - W - 1) / (T - W - 1),
+     * to f * lr = lr_final_frac * lr at n = T, held after.  The decoupled
+     * weight decay scales with the step's rate.  T = 0: constant lr.
+     * T <= 16,777,216; the fractions in [0, 1]. */
+    int64_t lr_total_steps;
+    double lr_warmup_frac, lr_warmup_start, lr_final_frac;
 } gasloc_hparams;
 
 /* Element type of the replica store (every array: x, y, m, v, b, c, h).  All
@@ -115,7 +125,9 @@ typedef void (*gasloc_free_fn)(void *ptr, void *stream, void *user);
 
 /* Fills *hp with the defaults: AdamW lr 3e-4, betas (0.9, 0.95), eps 1e-8,
  * weight decay 0.1 (App. B); sigma 0.01; Nesterov with eta_out 0.7, mu 0.9;
- * eta = alpha = 1, gamma = 0; edge_prob 1; uniform weights; shared h. */
+ * eta = alpha = 1, gamma = 0; edge_prob 1; uniform weights; shared h;
+ * constant lr (lr_total_steps 0; warm-up fraction 0.1 from 1% of the peak and
+ * a final fraction of 0 when a schedule length is set, as App. B states). */
 void gasloc_default_hparams(gasloc_hparams *hp);
 
 /* Creates a context for n_workers (1..32) replicas of n_params (>= 1) fp32

@@ -44,7 +44,9 @@ class Hparams(ctypes.Structure):
                 ("alpha", ctypes.c_double), ("gamma", ctypes.c_double),
                 ("edge_prob", ctypes.c_double), ("outer_mode", ctypes.c_int32),
                 ("weights", ctypes.c_int32), ("per_worker_h", ctypes.c_int32),
-                ("storage", ctypes.c_int32)]
+                ("storage", ctypes.c_int32), ("lr_total_steps", ctypes.c_int64),
+                ("lr_warmup_frac", ctypes.c_double), ("lr_warmup_start", ctypes.c_double),
+                ("lr_final_frac", ctypes.c_double)]
 
 
 ALLOC_FN = ctypes.CFUNCTYPE(ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_void_p)

@@ -49,18 +49,18 @@ constexpr Cache kSt = Cache::kL2;
 
 // Per-step constants, each in both halves of a register pair.
 struct Consts {
-    float2 decay, b1, b2, omb1, omb2, eps, sigma;
+    float2 b1, b2, omb1, omb2, eps, sigma;
 };
 
 // Two lanes of the step; each paired operation rounds each lane exactly as
 // the scalar operation does (f32x2.cuh), so the sequence is the one above.
 __device__ __forceinline__ float2 adamw_pair(float2 y, float2 m_in, float2 v_in, float2 c, float2 h, float2 xi,
-                                             float2 nstep, float2 isb, const Consts &k, float2 &m_out,
-                                             float2 &v_out) {
+                                             float2 nstep, float2 isb, float2 decay, const Consts &k,
+                                             float2 &m_out, float2 &v_out) {
     const float2 d = x2::sub(y, c);
     const float2 t = x2::mul(h, d);
     const float2 g = x2::fma(k.sigma, xi, t);
-    y = x2::mul(y, k.decay);
+    y = x2::mul(y, decay);
     const float2 m = x2::fma(k.b1, m_in, x2::mul(k.omb1, g));
     const float2 v = x2::fma(k.b2, v_in, x2::mul(k.omb2, x2::mul(g, g)));
     const float2 den = x2::fma(make_float2(__fsqrt_rn(v.x), __fsqrt_rn(v.y)), isb, k.eps);
@@ -83,11 +83,14 @@ __device__ __forceinline__ float2 noise_pair(uint32_t k, uint32_t klo, uint32_t 
     return x2::mul(make_float2(noise_int(k, klo, khi), noise_int(k + 1, klo, khi)), x2::splat(scale));
 }
 
-template <int U, bool PER_WORKER_H, typename T>
+// SCHED: the learning rate follows a schedule, so the weight-decay factor
+// differs between workers and comes from the step table; otherwise it is the
+// launch-wide fl32(1 - lr * weight_decay).
+template <int U, bool PER_WORKER_H, bool SCHED, typename T>
 __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     using E = Elem<T>;
-    const Consts kc{x2::splat(a.decay), x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1),
-                    x2::splat(a.omb2), x2::splat(a.eps), x2::splat(a.sigma)};
+    const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
+                    x2::splat(a.eps), x2::splat(a.sigma)};
     // this step's per-worker scalars -> shared
     __shared__ StepTable tab;
     __shared__ int last_copy;
@@ -107,7 +110,8 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
             a.state->nsteps[i] = n;
             a.state->p1[i] = p1;
             a.state->p2[i] = p2;
-            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d), a.lr, a.seed);
+            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d),
+                               lr_of_step(n + 1, a.lr_sched, a.lr_steps, a.lr_after), a.wd, a.seed);
         }
         if (i == 0) *a.ticket = 0u;
     }
@@ -156,15 +160,16 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const int i = a.worker[a0 + u];
                     const float2 nstep = x2::splat(-tab.step[i]);
                     const float2 isb = x2::splat(tab.isb[i]);
+                    const float2 dec = SCHED ? x2::splat(tab.decay[i]) : x2::splat(a.decay);
                     const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
                     const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
                     const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
                                  Cu = E::unpack(Cc[u]);
                     float2 m01, v01, m23, v23;
                     const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
-                                                  noise_pair(k0, klo, khi), nstep, isb, kc, m01, v01);
+                                                  noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
                     const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
-                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, kc, m23, v23);
+                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
                     const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
@@ -197,18 +202,26 @@ int blocks_per_sm(int block, bool per_worker_h) {
     int nb = 0;
     const cudaError_t e =
         per_worker_h
-            ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kPerWorkerH, true, T>, block, 0)
-            : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kShared, false, T>, block, 0);
+            ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kPerWorkerH, true, false, T>,
+                                                            block, 0)
+            : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kShared, false, false, T>,
+                                                            block, 0);
     if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
 }
 
 template <typename T>
 void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
-    if (a.per_worker_h)
-        adamw_kernel<Batch<T>::kPerWorkerH, true, T><<<grid, kBlock, 0, s>>>(a);   // 5 loads per worker
+    constexpr int UP = Batch<T>::kPerWorkerH, US = Batch<T>::kShared;   // per-worker h: 5 loads per worker
+    const bool sched = a.lr_steps > 0;
+    if (a.per_worker_h && sched)
+        adamw_kernel<UP, true, true, T><<<grid, kBlock, 0, s>>>(a);
+    else if (a.per_worker_h)
+        adamw_kernel<UP, true, false, T><<<grid, kBlock, 0, s>>>(a);
+    else if (sched)
+        adamw_kernel<US, false, true, T><<<grid, kBlock, 0, s>>>(a);
     else
-        adamw_kernel<Batch<T>::kShared, false, T><<<grid, kBlock, 0, s>>>(a);
+        adamw_kernel<US, false, false, T><<<grid, kBlock, 0, s>>>(a);
 }
 
 }  // namespace

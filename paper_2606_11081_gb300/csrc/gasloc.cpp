@@ -46,6 +46,7 @@ constexpr int64_t kPadFloats = 64;
 constexpr int kTileA = 1024;          // init / adamw / ce / average tiles (4 x 256 threads)
 constexpr int kMaxLocalSteps = 1024;
 constexpr int kCeRing = 4096;
+constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -127,6 +128,9 @@ struct gasloc_ctx {
     double *ce_d = nullptr;          // [0] standalone reduction result
     double *ce_ring = nullptr;       // consensus error of round t at [t % kCeRing]
     DevState *state_d = nullptr;     // device-resident step counters
+    double *lr_sched_d = nullptr;    // lr of local steps 1..lr_steps (schedule of App. B)
+    int64_t lr_sched_cap = 0, lr_steps = 0;
+    double lr_after = 0.0;           // lr of every later step (the constant lr without a schedule)
     StepTable *table_d = nullptr;    // scalars of each worker's next local step
     int64_t table_gen = -1;          // gen at which table_d was last refreshed
     cudaStream_t cap_stream = nullptr;
@@ -241,6 +245,11 @@ int check_hparams(const gasloc_hparams *hp) {
     if (hp->per_worker_h != 0 && hp->per_worker_h != 1) return fail(GASLOC_EINVAL, "per_worker_h must be 0 or 1");
     if (hp->storage != GASLOC_STORAGE_F32 && hp->storage != GASLOC_STORAGE_BF16)
         return fail(GASLOC_EINVAL, "unknown storage type %d", hp->storage);
+    if (hp->lr_total_steps < 0 || hp->lr_total_steps > kMaxScheduleSteps)
+        return fail(GASLOC_EINVAL, "lr_total_steps must be in [0, %lld]", (long long)kMaxScheduleSteps);
+    auto frac = [](double v) { return v >= 0.0 && v <= 1.0; };
+    if (!frac(hp->lr_warmup_frac) || !frac(hp->lr_warmup_start) || !frac(hp->lr_final_frac))
+        return fail(GASLOC_EINVAL, "schedule fractions must be in [0, 1]");
     return GASLOC_OK;
 }
 
@@ -296,6 +305,50 @@ int restore_step_counters(gasloc_ctx *c) {
     }
     if (cudaMemcpy(c->state_d, &ds, sizeof ds, cudaMemcpyHostToDevice) != cudaSuccess)
         return fail(GASLOC_ECUDA, "restoring the step counters failed");
+    return GASLOC_OK;
+}
+
+// Learning rate of a worker's n-th local step under the schedule of App. B
+// (see gasloc_hparams): warm-up from lr_warmup_start * lr over W =
+// round(lr_warmup_frac * T) steps, then cosine decay to lr_final_frac * lr at
+// step T, held after; T = 0: constant.  Double, one rounding per operation.
+double sched_lr(const gasloc_hparams &hp, int64_t n) {
+    const int64_t T = hp.lr_total_steps;
+    if (T <= 0) return hp.lr;
+    const int64_t W = static_cast<int64_t>(std::llround(hp.lr_warmup_frac * static_cast<double>(T)));
+    if (n <= W) {
+        const double s0 = hp.lr_warmup_start;
+        return hp.lr * (s0 + (1.0 - s0) * (static_cast<double>(n - 1) / static_cast<double>(W)));
+    }
+    const int64_t span = T - W - 1;
+    double q = span > 0 ? static_cast<double>(n - W - 1) / static_cast<double>(span) : 1.0;
+    if (q > 1.0) q = 1.0;
+    const double f = hp.lr_final_frac;
+    const double pi = 3.14159265358979323846;
+    return hp.lr * (f + (1.0 - f) * (0.5 * (1.0 + std::cos(pi * q))));
+}
+
+// Puts the rates of local steps 1..T of the current schedule on the device
+// (the kernels index them by each worker's step count; later steps use
+// lr_after).  Waits for the stream.
+int upload_schedule(gasloc_ctx *c) {
+    const int64_t T = c->hp.lr_total_steps;
+    c->lr_after = sched_lr(c->hp, T + 1);
+    c->lr_steps = 0;
+    if (T == 0) return GASLOC_OK;
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    if (T > c->lr_sched_cap) {
+        c->dfree(c->lr_sched_d);
+        c->lr_sched_d = static_cast<double *>(c->dalloc(static_cast<size_t>(T) * sizeof(double)));
+        c->lr_sched_cap = c->lr_sched_d ? T : 0;
+        if (!c->lr_sched_d) return fail(GASLOC_ENOMEM, "device allocation failed (lr schedule)");
+    }
+    std::vector<double> v(static_cast<size_t>(T));
+    for (int64_t n = 1; n <= T; ++n) v[static_cast<size_t>(n - 1)] = sched_lr(c->hp, n);
+    e = cudaMemcpy(c->lr_sched_d, v.data(), v.size() * sizeof(double), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "uploading the lr schedule");
+    c->lr_steps = T;
     return GASLOC_OK;
 }
 
@@ -379,6 +432,10 @@ void gasloc_default_hparams(gasloc_hparams *hp) {
     hp->alpha = 1.0;
     hp->gamma = 0.0;
     hp->edge_prob = 1.0;
+    hp->lr_total_steps = 0;
+    hp->lr_warmup_frac = 0.1;
+    hp->lr_warmup_start = 0.01;
+    hp->lr_final_frac = 0.0;
     hp->outer_mode = GASLOC_OUTER_NESTEROV;
     hp->weights = GASLOC_W_UNIFORM;
     hp->per_worker_h = 0;
@@ -423,6 +480,10 @@ int gasloc_set_hparams(gasloc_ctx *c, const gasloc_hparams *hp) {
     refresh_spec(c);
     // bias corrections are 1 - beta^n with the current betas: re-form the
     // device products beta^n from the step counts
+    if (c->started) {
+        const int rc = upload_schedule(c);
+        if (rc) return rc;
+    }
     if (new_betas) return restore_step_counters(c);
     return GASLOC_OK;
 }
@@ -597,8 +658,10 @@ int gasloc_start(gasloc_ctx *c) {
     }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
 
+    int rc = upload_schedule(c);
+    if (rc) { c->release_all(); return rc; }
     InitArgs ia{c->tens_d, c->tiles_a, c->ntiles_a, n, c->hp.per_worker_h, c->seed, c->hp.storage, c->err_d};
-    int rc = launch_checked(c, launch_init(ia, c->sms * 8, c->stream), "init kernel");
+    rc = launch_checked(c, launch_init(ia, c->sms * 8, c->stream), "init kernel");
     if (rc) { c->release_all(); return rc; }
     c->started = true;
     c->round = 0;
@@ -652,7 +715,8 @@ namespace {
 int refresh_step_table(gasloc_ctx *c, cudaStream_t s) {
     if (c->table_gen == c->gen) return GASLOC_OK;
     const gasloc_hparams &hp = c->hp;
-    PrepArgs pa{c->state_d, c->table_d, c->n, hp.lr, hp.beta1, hp.beta2, c->seed};
+    PrepArgs pa{c->state_d, c->table_d, c->n, hp.beta1, hp.beta2, hp.weight_decay, c->lr_sched_d, c->lr_steps,
+                c->lr_after, c->seed};
     const int rc = launch_checked(c, launch_prep(pa, s), "step-scalar kernel");
     if (!rc) c->table_gen = c->gen;
     return rc;
@@ -677,13 +741,16 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.table = c->table_d;
     a.state = c->state_d;
     a.ticket = c->ticket + 1;   // slot 0: the gossip and consensus-error reductions
-    a.lr = hp.lr;
+    a.lr_sched = c->lr_sched_d;
+    a.lr_steps = c->lr_steps;
+    a.lr_after = c->lr_after;
+    a.wd = hp.weight_decay;
+    a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
     a.beta1d = hp.beta1;
     a.beta2d = hp.beta2;
     a.seed = c->seed;
     a.per_worker_h = hp.per_worker_h;
     a.storage = hp.storage;
-    a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
     a.beta1 = static_cast<float>(hp.beta1);
     a.beta2 = static_cast<float>(hp.beta2);
     a.omb1 = static_cast<float>(1.0 - hp.beta1);
@@ -1153,8 +1220,8 @@ int gasloc_save(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "wb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s' for writing", path);
     CkptHeader h{};
-    std::memcpy(h.magic, "GASLOCK2", 8);
-    h.version = 2;
+    std::memcpy(h.magic, "GASLOCK3", 8);
+    h.version = 3;
     h.n = c->n;
     h.P = c->P;
     h.n_tensors = static_cast<int64_t>(c->numels.size());
@@ -1202,7 +1269,7 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "rb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s'", path);
     CkptHeader h{};
-    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK2", 8) == 0 && h.version == 2;
+    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK3", 8) == 0 && h.version == 3;
     if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "'%s' is not a checkpoint", path); }
     if (h.n != c->n || h.P != c->P || h.n_tensors != static_cast<int64_t>(c->numels.size()) || h.seed != c->seed ||
         h.kind != c->spec.kind || h.rows != c->spec.rows || h.cols != c->spec.cols ||

@@ -79,17 +79,21 @@ struct DevState {
 // kernel after a start, a hyperparameter change or a checkpoint load, and by
 // every AdamW launch for the workers it stepped).
 struct StepTable {
-    float step[kMaxWorkers];          // fl32(lr / (1 - beta1^n))
+    float step[kMaxWorkers];          // fl32(lr_n / (1 - beta1^n)), lr_n the step's scheduled rate
     float isb[kMaxWorkers];           // fl32(1 / sqrt(1 - beta2^n))
     uint32_t key_lo[kMaxWorkers];     // noise key hash(seed, 4, i, n)
     uint32_t key_hi[kMaxWorkers];
+    float decay[kMaxWorkers];         // fl32(1 - lr_n * weight_decay)
 };
 
 struct PrepArgs {
     const DevState *state;
     StepTable *table;
     int32_t n_workers;
-    double lr, beta1, beta2;
+    double beta1, beta2, wd;
+    const double *lr_sched;               // lr of local steps 1..lr_steps
+    int64_t lr_steps;
+    double lr_after;                      // lr of later steps
     uint64_t seed;
 };
 
@@ -101,14 +105,18 @@ struct AdamwArgs {
     DevState *state;                      // step counters, advanced for the active workers
     unsigned int *ticket;                 // CTAs that copied the table (returns to 0)
     uint32_t active_mask;                 // bit i: worker i takes this step
-    double lr, beta1d, beta2d;            // for the next step's scalars
+    double beta1d, beta2d, wd;            // for the next step's scalars
+    const double *lr_sched;               // lr of local steps 1..lr_steps
+    int64_t lr_steps;
+    double lr_after;                      // lr of later steps
     uint64_t seed;
     int32_t n_active;
     int32_t per_worker_h;
     int32_t storage;
     uint32_t from_x_mask;                 // bit i: worker i starts from x
     int32_t worker[kMaxWorkers];
-    float decay, beta1, beta2, omb1, omb2, eps, sigma;
+    float decay;                          // fl32(1 - lr * weight_decay) without a schedule
+    float beta1, beta2, omb1, omb2, eps, sigma;
     int32_t n_workers;                    // rows of every per-worker array
     int32_t *err;                         // device error word (checked build)
 };

@@ -192,8 +192,9 @@ __global__ void topo_kernel(const TopoSpec spec, const int64_t round_arg, const 
 __global__ void prep_kernel(const PrepArgs a) {
     const int i = threadIdx.x;
     if (i >= a.n_workers) return;
-    write_step_scalars(a.table, i, a.state->nsteps[i] + 1, __dmul_rn(a.state->p1[i], a.beta1),
-                       __dmul_rn(a.state->p2[i], a.beta2), a.lr, a.seed);
+    const int64_t n = a.state->nsteps[i] + 1;
+    write_step_scalars(a.table, i, n, __dmul_rn(a.state->p1[i], a.beta1), __dmul_rn(a.state->p2[i], a.beta2),
+                       lr_of_step(n, a.lr_sched, a.lr_steps, a.lr_after), a.wd, a.seed);
 }
 
 // Loads of the average marked as the last use of their lines (ld.global.lu):

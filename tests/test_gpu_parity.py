@@ -266,3 +266,22 @@ def test_gather_rejects_bad_index():
         assert e.value.code == g.EINVAL
         np.testing.assert_array_equal(ctx.gather("x", 1, np.array([0, 99, 42])),
                                       ctx.read("x", 1)[[0, 99, 42]])
+
+
+@pytest.mark.parametrize("storage", ["f32", "bf16"])
+def test_lr_schedule_matches_oracle(storage):
+    # App. B's warm-up + cosine schedule runs over each worker's own local
+    # steps: with different H_i the workers sit at different points of it, and
+    # the busiest one passes the warm-up, the decay and the held final rate.
+    N, P, R = 6, 2 * 1024 + 9, 5
+    Hi = np.array([1, 3, 2, 4, 1, 2], np.int32)
+    hp = dict(lr=4e-3, storage=storage, lr_total_steps=9, lr_warmup_frac=0.25, lr_final_frac=0.1)
+    ctx, st = make_pair(N, P, "ring", seed=31, hp=hp, Hi=Hi)
+    with ctx:
+        for _ in range(R):
+            ctx.local_steps(g.PER_WORKER_STEPS)
+            ctx.gossip_round()
+            st.local_steps(0, Hi)
+            st.gossip_round()
+        for w in ("x", "y", "m", "v", "b"):
+            np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)

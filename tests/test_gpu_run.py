@@ -146,3 +146,16 @@ def test_hparam_change_matches_oracle():
         for w in ("x", "y", "m", "v", "b"):
             np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)
         assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)
+
+
+def test_run_with_lr_schedule_matches_stepwise():
+    hp = dict(lr=3e-3, lr_total_steps=12, lr_final_frac=0.05)
+    a, _ = make_pair(8, 4099, "matching", seed=23, hp=hp)
+    b, _ = make_pair(8, 4099, "matching", seed=23, hp=hp)
+    with a, b:
+        a.run(6, 3)
+        for _ in range(6):
+            b.local_steps(3)
+            b.gossip_round()
+        for w in ("x", "y", "m", "v", "b"):
+            np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
