@@ -1316,6 +1316,8 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     c->has_Hi = h.has_Hi != 0;
     c->Hi = Hi;
     c->nsteps = nsteps;
+    rc = upload_schedule(c);   // the checkpoint's learning-rate schedule
+    if (rc) return rc;
     rc = restore_step_counters(c);
     if (rc) return rc;
     c->gen += 1;

@@ -233,8 +233,11 @@ def test_tensor_list_equals_flat():
         np.testing.assert_array_equal(v.cpu().numpy(), b.read_all("x")[:, 1003:1003 + 4097])
 
 
-def test_resume_is_exact(tmp_path):
-    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True)
+@pytest.mark.parametrize("sched", [0, 8])
+def test_resume_is_exact(tmp_path, sched):
+    # the resumed context starts with other hyperparameters (no lr schedule):
+    # the checkpoint's, schedule included, take over
+    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True, lr_total_steps=sched)
     a, _ = make_pair(6, 3000, "exp", seed=21, hp=hp, Hi=[1, 2, 3, 1, 2, 3])
     with a:
         for _ in range(3):
@@ -247,7 +250,7 @@ def test_resume_is_exact(tmp_path):
             a.gossip_round()
         xa = a.read_all("x")
         ce_a = a.consensus_error()
-    b, _ = make_pair(6, 3000, "exp", seed=21, hp=hp, Hi=[1, 1, 1, 1, 1, 1])
+    b, _ = make_pair(6, 3000, "exp", seed=21, hp=dict(hp, lr_total_steps=0), Hi=[1, 1, 1, 1, 1, 1])
     with b:
         b.load(path)
         assert b.round == 3
