@@ -654,7 +654,7 @@ int gasloc_start(gasloc_ctx *c) {
     c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0, c->hp.storage);
     for (int m = 0; m < 6; ++m) {
         const GossipShape sm = gossip_shape(n, m, c->hp.storage);
-        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm.smem));
+        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm.smem, sm.dense != 0));
     }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
 
@@ -802,6 +802,7 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     a.tile = gs.tile;
     a.groups = gs.groups;
     a.stages = gs.stages;
+    a.dense = gs.dense;
     a.eta_out = static_cast<float>(hp.outer_lr);
     a.mu = static_cast<float>(hp.outer_momentum);
     a.eta = static_cast<float>(hp.eta);

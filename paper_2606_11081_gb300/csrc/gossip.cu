@@ -44,6 +44,7 @@
 #include <cuda_runtime.h>
 
 #include <cstddef>
+#include <type_traits>
 
 #include "check.cuh"
 #include "elem.cuh"
@@ -209,7 +210,17 @@ __device__ __forceinline__ void consumer_barrier() {
     asm volatile("barrier.sync 1, %0;" ::"r"(kConsumers) : "memory");
 }
 
-template <int MODE, typename T>
+// DENSE (bf16, one thread per column, n <= 8, not Eq. 2): the thread widens the n
+// mixed rows of its column once and forms each worker's mix over all j < n
+// in ascending order with a dense weight row (zero off the neighbourhood),
+// built from the round's table in the prologue.  For finite rows a
+// zero-weight term adds an exact zero, so the sums are those of the neighbour
+// lists; a non-finite row (a diverged replica) reaches every worker of its
+// column as NaN (0 * inf) where the lists would confine it to its neighbours.
+constexpr int kDenseMax = 8;
+constexpr int kDenseRow = 8;   // dense row i lives in tp->w[kDenseRow + i] (rows >= n are free)
+
+template <int MODE, typename T, bool DENSE>
 __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kernel(const GossipArgs a) {
     using R = ModeRows<MODE>;
     using E = Elem<T>;
@@ -243,6 +254,19 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         for (int q = threadIdx.x; q < 2 * rows + (kAll - kDeg); q += blockDim.x) {
             const int at = q < rows ? q : (q < 2 * rows ? kW + q - rows : kDeg + q - 2 * rows);
             dst[at] = src[at];
+        }
+    }
+    if constexpr (DENSE) {   // dense weights of the round, from the table in global memory
+        const int t = threadIdx.x;
+        if (t < kDenseMax * kDenseMax) {
+            const int i = t / kDenseMax, j = t % kDenseMax;
+            if (i < n && j < n) {
+                float wij = 0.f;
+                const int dg = a.topo->deg[i];
+                for (int q = 0; q <= dg && q < kMaxWorkers; ++q)
+                    if (a.topo->nbr[i][q] == j) wij = a.topo->w[i][q];
+                tp->w[kDenseRow + i][j] = wij;
+            }
         }
     }
     if (threadIdx.x == 0) {
@@ -420,10 +444,30 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             int nr = 0;                               // Eq. 2 results held
             if (active) {
                 float4 sh = make_float4(0.f, 0.f, 0.f, 0.f);   // G = 1: worker 0's new x (set at i = 0)
+                float4 sall[DENSE ? kDenseMax : 1];           // DENSE: the column's mixed rows, widened once
+                if constexpr (DENSE) {
+#pragma unroll
+                    for (int j = 0; j < kDenseMax; ++j)
+                        if (j < n) sall[j] = E::load4_smem(cp(0, j));
+                }
                 for (int i = g; i < n; i += G) {
                     float2 acc01 = x2::splat(0.f), acc23 = acc01;
-                    int dg = tp->deg[i];
-                    if (!span_ok(dg, dg + 1, kMaxWorkers, a.err)) dg = -1;
+                    if constexpr (DENSE) {
+                        const float *wr = &tp->w[kDenseRow + i][0];
+#pragma unroll
+                        for (int j = 0; j < kDenseMax; ++j) {
+                            if (j < n) {
+                                const float2 w = x2::splat(wr[j]);
+                                acc01 = x2::fma(w, x2::lo(sall[j]), acc01);
+                                acc23 = x2::fma(w, x2::hi(sall[j]), acc23);
+                            }
+                        }
+                    }
+                    int dg = -1;   // DENSE: every neighbour was taken above
+                    if constexpr (!DENSE) {
+                        dg = tp->deg[i];
+                        if (!span_ok(dg, dg + 1, kMaxWorkers, a.err)) dg = -1;
+                    }
                     for (int q = 0; q <= dg; ++q) {
                         const int j = tp->nbr[i][q];
                         if (!span_ok(j, j + 1, n, a.err)) continue;
@@ -553,34 +597,47 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
 }
 
 template <int MODE>
-void *kernel_ptr(int storage) {
-    return storage == kStoreBF16 ? reinterpret_cast<void *>(gossip_kernel<MODE, bf16>)
-                                 : reinterpret_cast<void *>(gossip_kernel<MODE, float>);
+void *kernel_ptr(int storage, bool dense) {
+    // dense mixing exists for bf16 only, and not for Eq. 2
+    constexpr bool kCanDense = MODE != kOutEq2;
+    if (storage != kStoreBF16) return reinterpret_cast<void *>(gossip_kernel<MODE, float, false>);
+    if (dense && kCanDense) return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, kCanDense>);
+    return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, false>);
 }
 
-void *mode_kernel(int mode, int storage) {
+void *mode_kernel(int mode, int storage, bool dense) {
     switch (mode) {
-    case kOutSgd: return kernel_ptr<kOutSgd>(storage);
-    case kOutSgdm: return kernel_ptr<kOutSgdm>(storage);
-    case kOutNesterov: return kernel_ptr<kOutNesterov>(storage);
-    case kOutEq2: return kernel_ptr<kOutEq2>(storage);
-    case kOutDadam: return kernel_ptr<kOutDadam>(storage);
-    default: return kernel_ptr<kOutLocalDadam>(storage);
+    case kOutSgd: return kernel_ptr<kOutSgd>(storage, dense);
+    case kOutSgdm: return kernel_ptr<kOutSgdm>(storage, dense);
+    case kOutNesterov: return kernel_ptr<kOutNesterov>(storage, dense);
+    case kOutEq2: return kernel_ptr<kOutEq2>(storage, false);
+    case kOutDadam: return kernel_ptr<kOutDadam>(storage, dense);
+    default: return kernel_ptr<kOutLocalDadam>(storage, dense);
     }
 }
 
 int mode_rows(int mode) { return (mode == kOutSgd || mode == kOutDadam) ? 2 : 3; }
 
+template <typename T, bool D>
+void launch_td(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
+    switch (a.mode) {
+    case kOutSgd: gossip_kernel<kOutSgd, T, D><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutSgdm: gossip_kernel<kOutSgdm, T, D><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutNesterov: gossip_kernel<kOutNesterov, T, D><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutEq2: gossip_kernel<kOutEq2, T, false><<<grid, kThreads, smem, s>>>(a); break;
+    case kOutDadam: gossip_kernel<kOutDadam, T, D><<<grid, kThreads, smem, s>>>(a); break;
+    default: gossip_kernel<kOutLocalDadam, T, D><<<grid, kThreads, smem, s>>>(a); break;
+    }
+}
 template <typename T>
 void launch_t(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
-    switch (a.mode) {
-    case kOutSgd: gossip_kernel<kOutSgd, T><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutSgdm: gossip_kernel<kOutSgdm, T><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutNesterov: gossip_kernel<kOutNesterov, T><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutEq2: gossip_kernel<kOutEq2, T><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutDadam: gossip_kernel<kOutDadam, T><<<grid, kThreads, smem, s>>>(a); break;
-    default: gossip_kernel<kOutLocalDadam, T><<<grid, kThreads, smem, s>>>(a); break;
+    if constexpr (std::is_same<T, bf16>::value) {
+        if (a.dense) {
+            launch_td<T, true>(a, grid, smem, s);
+            return;
+        }
     }
+    launch_td<T, false>(a, grid, smem, s);
 }
 
 }  // namespace
@@ -595,6 +652,13 @@ GossipShape gossip_shape(int n, int mode, int storage) {
     // ring: 0.51 of the copy peak against 0.48 with two, 0.36 with four).
     // From 9 to 16 workers two threads per column, above four.
     sh.groups = n <= 4 ? 1 : (n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : 4));
+    // Dense mixing (every row of the column widened once, then w_ij * s_j
+    // over all j with w_ij = 0 off the graph) for bf16 with one thread per
+    // column: the 8-worker exponential graph's gossip went from 0.885 to 1.006
+    // of the copy peak.  fp32 keeps the neighbour lists (the 4-worker ring
+    // was 2% slower dense), and so does Eq. 2, whose mixed rows are formed
+    // per neighbour.
+    sh.dense = (storage == kStoreBF16 && sh.groups == 1 && n <= kDenseMax && mode != kOutEq2) ? 1 : 0;
     sh.tile = 4 * (kConsumers / sh.groups);
     sh.block = kThreads;
     const size_t esize = storage == kStoreBF16 ? 2 : 4;
@@ -616,19 +680,20 @@ GossipShape gossip_shape(int n, int mode, int storage) {
 
 cudaError_t gossip_set_smem(size_t smem) {
     for (int st = 0; st <= kStoreBF16; ++st)
-        for (int m = 0; m <= kOutLocalDadam; ++m) {
-            const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m, st),
-                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                       static_cast<int>(smem));
-            if (e != cudaSuccess) return e;
-        }
+        for (int m = 0; m <= kOutLocalDadam; ++m)
+            for (int d = 0; d < 2; ++d) {
+                const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m, st, d != 0),
+                                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                           static_cast<int>(smem));
+                if (e != cudaSuccess) return e;
+            }
     return cudaSuccess;
 }
 
-int gossip_blocks_per_sm(int mode, int storage, size_t smem) {
+int gossip_blocks_per_sm(int mode, int storage, size_t smem, bool dense) {
     int nb = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, reinterpret_cast<const void *>(mode_kernel(mode, storage)),
-                                                      kThreads, smem) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+            &nb, reinterpret_cast<const void *>(mode_kernel(mode, storage, dense)), kThreads, smem) != cudaSuccess)
         return 1;
     return nb > 0 ? nb : 1;
 }

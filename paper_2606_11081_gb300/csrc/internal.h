@@ -135,6 +135,7 @@ struct GossipArgs {
     int32_t tile;          // elements per tile (4 x 256 / groups)
     int32_t groups;        // consumer threads per 16-byte column
     int32_t stages;
+    int32_t dense;         // dense mixing variant (GossipShape::dense)
     float eta_out, mu, eta, alpha, oma, gamma;
     double *partials;      // [gridDim] per-CTA consensus-error partials
     unsigned int *ticket;  // last-CTA-done counter (returns to 0)
@@ -167,6 +168,7 @@ cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream
 // Launch shape of the gossip kernel for n workers and an outer mode.
 struct GossipShape {
     int groups, tile, block, stages;
+    int dense;   // one thread per column mixing with a dense weight row (n <= 8, not Eq. 2)
     size_t smem;
 };
 GossipShape gossip_shape(int n, int mode, int storage);
@@ -188,7 +190,7 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s
 
 // Occupancy-derived persistent grid sizes.
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage);
-int gossip_blocks_per_sm(int mode, int storage, size_t smem);
+int gossip_blocks_per_sm(int mode, int storage, size_t smem, bool dense);
 int ce_blocks_per_sm(int block, int storage);
 cudaError_t gossip_set_smem(size_t smem);
 

@@ -60,6 +60,27 @@ def test_bf16_trajectory(mode, N, topo, kw):
         same(ctx, st, ("x", "b", "m", "v"))
 
 
+@pytest.mark.parametrize("mode", ["sgd", "sgdm", "nesterov", "dadam", "local_dadam"])
+@pytest.mark.parametrize("N,topo,kw", [(2, "ring", {}), (3, "complete", {}), (5, "2peer", {}),
+                                       (8, "matching", {}), (7, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
+                                       (6, "torus:2x3", {"weights": "lazy"})])
+def test_bf16_dense_mixing(mode, N, topo, kw):
+    """Up to 8 workers a bf16 column is mixed densely (zero weight off the
+    graph): bit-exact against the neighbour-list sums for every outer mode,
+    and on graphs drawn afresh each round (1-Peer, 2-Peer, dropped edges)."""
+    P, R, H = 3 * 1024 + 7, 4, 1
+    hp = dict(kw, **BF, outer=mode, lr=2e-3, eta=0.9, alpha=0.8, gamma=0.3, noise_sigma=0.02)
+    ctx, st = make_pair(N, P, topo, seed=900 + N, hp=hp)
+    with ctx:
+        for _ in range(R):
+            ctx.local_steps(H)
+            st.local_steps(H)
+            ctx.gossip_round()
+            st.gossip_round()
+            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+        same(ctx, st, ("x", "b", "m", "v", "y"))
+
+
 def test_bf16_heterogeneous_and_graph_rounds():
     Hi = np.array([0, 2, 1, 3], np.int32)
     ctx, st = make_pair(4, 3001, "complete", seed=8, hp=dict(BF, lr=1e-3), Hi=Hi)
