@@ -106,7 +106,7 @@ class Oracle:
             "oc_fmix32": (ctypes.c_uint32, [ctypes.c_uint32]),
             "oc_normal": (dbl, [u64, u64, u64, u64]),
             "oc_uniform": (dbl, [u64, u64, u64, u64, dbl, dbl]),
-            "oc_noise": (dbl, [u64, u64, u64, u64]),
+            "oc_noise": (dbl, [u64, u64, u64, u64, i32]),
             "oc_real_size": (ctypes.c_int, []), "oc_num_threads": (ctypes.c_int, []),
             "oc_bf16_round": (dbl, [dbl]),
             "oc_permutation": (None, [u64, i64, i32, _I32P]),
@@ -147,8 +147,8 @@ class Oracle:
     def uniform(self, seed, tag, i, k, lo, span) -> float:
         return self.lib.oc_uniform(seed, tag, i, k, lo, span)
 
-    def noise(self, seed, i, n, k) -> float:
-        return self.lib.oc_noise(seed, i, n, k)
+    def noise(self, seed, i, n, k, storage: str = "f32") -> float:
+        return self.lib.oc_noise(seed, i, n, k, STORAGE[storage])
 
     def sched_lr(self, pb: Problem, n: int) -> float:
         """Learning rate of a worker's n-th local step under pb's schedule."""

@@ -107,15 +107,36 @@ static REAL uniform_lo_span(uint64_t seed, uint64_t tag, uint64_t i, uint64_t k,
 }
 
 /* Gradient noise xi(i, n, k): uniform on [-sqrt3, sqrt3), unit variance.
- * K = hash(seed, 4, i, n) is the key of worker i's n-th (1-based) local step,
- * u = fmix32(fmix32(k ^ lo32(K)) ^ hi32(K)), xi = (u>>8 * 2^-23 - 1) * sqrt3. */
-static REAL noise_xi(uint64_t key, uint64_t k)
+ * K = hash(seed, 4, i, n) is the key of worker i's n-th (1-based) local step
+ * and W(a) = fmix32(fmix32(a ^ lo32(K)) ^ hi32(K)), a taken modulo 2^32.
+ *   fp32 storage, a grid of 2^24 points, one word per element:
+ *     u = W(k),  xi = ((u >> 8) * 2^-23 - 1) * sqrt3.
+ *   bf16 storage, a grid of 2^16 points, one word per pair of elements:
+ *     element 2j takes the low 16 bits of W(j), element 2j+1 the high 16
+ *     bits; with q = half - 2^15 (an integer in [-2^15, 2^15)),
+ *     xi = q * (sqrt3 * 2^-15), one rounding (q and the power-of-two scaling
+ *     of sqrt3 are exact).  A bf16 store keeps 8 significand bits, so the
+ *     finer grid of the fp32 form would buy it nothing. */
+static uint32_t noise_word(uint64_t key, uint64_t a)
 {
+    return oc_fmix32(oc_fmix32((uint32_t)a ^ lo32(key)) ^ hi32(key));
+}
+
+static REAL noise_xi(uint64_t key, uint64_t k, int storage)
+{
+    const REAL sqrt3 = (REAL)1.7320508075688772;
+    if (storage == OC_STORE_BF16) {
+        const REAL two_m15 = (REAL)3.0517578125e-05;
+        const REAL scale = sqrt3 * two_m15;
+        const uint32_t u = noise_word(key, k >> 1);
+        const uint32_t half = (k & 1u) ? (u >> 16) : (u & 0xFFFFu);
+        const REAL q = (REAL)((int32_t)half - 32768);
+        return q * scale;
+    }
     const REAL two_m23 = (REAL)1.1920928955078125e-07;
     const REAL one = (REAL)1;
-    const REAL sqrt3 = (REAL)1.7320508075688772;
-    uint32_t u = oc_fmix32(oc_fmix32((uint32_t)k ^ lo32(key)) ^ hi32(key));
-    REAL a = (REAL)(u >> 8) * two_m23;
+    const uint32_t u = noise_word(key, k);
+    const REAL a = (REAL)(u >> 8) * two_m23;
     return (a - one) * sqrt3;
 }
 
@@ -154,8 +175,8 @@ double oc_normal(uint64_t seed, uint64_t tag, uint64_t i, uint64_t k)
 { return (double)normal01(seed, tag, i, k); }
 double oc_uniform(uint64_t seed, uint64_t tag, uint64_t i, uint64_t k, double lo, double span)
 { return (double)uniform_lo_span(seed, tag, i, k, (REAL)lo, (REAL)span); }
-double oc_noise(uint64_t seed, uint64_t i, uint64_t n, uint64_t k)
-{ return (double)noise_xi(oc_hash(seed, 4, i, n), k); }
+double oc_noise(uint64_t seed, uint64_t i, uint64_t n, uint64_t k, int32_t storage)
+{ return (double)noise_xi(oc_hash(seed, 4, i, n), k, storage); }
 int oc_real_size(void) { return (int)sizeof(REAL); }
 int oc_num_threads(void)
 {
@@ -450,7 +471,7 @@ static void adamw_step_worker(oc_state *st, int32_t i)
     #pragma omp parallel for schedule(static)
     for (int64_t e = 0; e < nk; ++e) {
         REAL yy = first ? x[e] : y[e];
-        const REAL xi = noise_xi(key, (uint64_t)st->kidx[e]);
+        const REAL xi = noise_xi(key, (uint64_t)st->kidx[e], sto);
         const REAL d = yy - c[e];
         const REAL t = h[e] * d;
         const REAL g = fma(sigma, xi, t);

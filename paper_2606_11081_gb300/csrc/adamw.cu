@@ -10,8 +10,8 @@
 // 6), issuing all of their loads before any arithmetic so that about 256
 // bytes of requests per thread stay in flight.  The synthetic gradient
 // g = h (y - c) + sigma xi is formed in registers; xi comes from a 32-bit
-// counter hash of the element index and the step key, so the gradient costs
-// no memory traffic.  The step's per-worker scalars (bias corrections, noise
+// counter hash of the element index and the step key (of the index of the
+// element pair with bf16 storage), so the gradient costs no memory traffic.  The step's per-worker scalars (bias corrections, noise
 // keys) come from the step table; the launch's last CTA to copy it advances
 // the step counters and writes the next step's scalars.
 //
@@ -26,6 +26,8 @@
 //   den = fma(sqrt(v), isb, eps)
 //   y = fma(-step, m / den, y)
 #include <cuda_runtime.h>
+
+#include <type_traits>
 
 #include "check.cuh"
 #include "elem.cuh"
@@ -70,17 +72,48 @@ __device__ __forceinline__ float2 adamw_pair(float2 y, float2 m_in, float2 v_in,
     return y;
 }
 
-// xi = ((u >> 8) * 2^-23 - 1) * sqrt3: uniform on [-sqrt3, sqrt3), unit
-// variance.  (u >> 8) * 2^-23 - 1 = ((u >> 8) - 2^23) * 2^-23 exactly, and
-// sqrt3 * 2^-23 is exact, so xi = fl(((u >> 8) - 2^23) * (sqrt3 * 2^-23)):
-// the same real product rounded once.
+// Gradient noise, uniform on [-sqrt3, sqrt3) with unit variance.
+// fp32 storage, 24 bits per element: u = word(k) and
+// xi = ((u >> 8) * 2^-23 - 1) * sqrt3.  (u >> 8) * 2^-23 - 1 equals
+// ((u >> 8) - 2^23) * 2^-23 exactly and sqrt3 * 2^-23 is exact, so
+// xi = fl(((u >> 8) - 2^23) * (sqrt3 * 2^-23)): the same real product rounded
+// once, from one integer conversion.
 __device__ __forceinline__ float noise_int(uint32_t k, uint32_t klo, uint32_t khi) {
-    const uint32_t u = noise_bits(k, klo, khi);
+    const uint32_t u = noise_word(k, klo, khi);
     return __int2float_rn(static_cast<int32_t>(u >> 8) - (1 << 23));
 }
 __device__ __forceinline__ float2 noise_pair(uint32_t k, uint32_t klo, uint32_t khi) {
     const float scale = static_cast<float>(1.7320508075688772) * 0x1p-23f;
     return x2::mul(make_float2(noise_int(k, klo, khi), noise_int(k + 1, klo, khi)), x2::splat(scale));
+}
+
+// bf16 storage, 16 bits per element: element 2j takes the low half of
+// word(j), element 2j + 1 the high half, and xi = q * (sqrt3 * 2^-15) with
+// q = half - 2^15.  A byte permute puts a half h in the mantissa of 2^23 (the
+// float 2^23 + h, exact); subtracting 2^23 + 2^15 leaves q exactly, and the
+// product is the one rounding.  One hash serves two elements, which matters
+// where the arithmetic, not the memory, sets the pace.  Columns start at even
+// k unless a tensor starts at an odd global index; then the 4 elements span 3
+// words.
+__device__ __forceinline__ float biased_half(uint32_t w, bool high) {
+    return __uint_as_float(__byte_perm(w, 0x4B000000u, high ? 0x7632u : 0x7610u));
+}
+__device__ __forceinline__ void noise4_pairs(uint32_t k, uint32_t klo, uint32_t khi, float2 &xi01, float2 &xi23) {
+    const uint32_t j = k >> 1;
+    const uint32_t w0 = noise_word(j, klo, khi), w1 = noise_word(j + 1u, klo, khi);
+    float2 b01, b23;
+    if ((k & 1u) == 0) {
+        b01 = make_float2(biased_half(w0, false), biased_half(w0, true));
+        b23 = make_float2(biased_half(w1, false), biased_half(w1, true));
+    } else {
+        const uint32_t w2 = noise_word(j + 2u, klo, khi);
+        b01 = make_float2(biased_half(w0, true), biased_half(w1, false));
+        b23 = make_float2(biased_half(w1, true), biased_half(w2, false));
+    }
+    const float2 bias = x2::splat(8421376.0f);   // 2^23 + 2^15
+    const float2 scale = x2::splat(static_cast<float>(1.7320508075688772) * 0x1p-15f);
+    xi01 = x2::mul(x2::sub(b01, bias), scale);
+    xi23 = x2::mul(x2::sub(b23, bias), scale);
 }
 
 // SCHED: the learning rate follows a schedule, so the weight-decay factor
@@ -131,7 +164,7 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
         T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
         const int64_t off = tl.start + e0;
         const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-        const uint32_t k0 = static_cast<uint32_t>(d.goff + off);
+        const uint32_t k0 = static_cast<uint32_t>(d.goff + off);   // global index of the column's first element
         float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
         if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::template load4<kLdCurv>(Hh + off);
 
@@ -165,11 +198,20 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
                     const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
                                  Cu = E::unpack(Cc[u]);
-                    float2 m01, v01, m23, v23;
-                    const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
-                                                  noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
-                    const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
-                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
+                    float2 m01, v01, m23, v23, y01, y23;
+                    if constexpr (std::is_same<T, bf16>::value) {
+                        float2 xi01, xi23;
+                        noise4_pairs(k0, klo, khi, xi01, xi23);
+                        y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4), xi01, nstep, isb,
+                                         dec, kc, m01, v01);
+                        y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4), xi23, nstep, isb,
+                                         dec, kc, m23, v23);
+                    } else {
+                        y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
+                                         noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
+                        y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
+                                         noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
+                    }
                     const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {

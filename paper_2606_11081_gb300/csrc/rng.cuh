@@ -7,8 +7,9 @@
 //   hash(seed, tag, a, b) = mix64(mix64(mix64(mix64(seed) ^ tag) ^ a) ^ b)
 //             tags: 1 x0, 2 centre, 3 curvature, 4 noise key, 5 permutation,
 //                   6 edge activation, 7 local step counts.
-//   fmix32:   MurmurHash3's 32-bit finalizer (Appleby), used per element for
-//             the gradient noise so that the per-element cost stays in 32-bit
+//   fmix32:   MurmurHash3's 32-bit finalizer (Appleby), applied twice per
+//             element (fp32 storage) or per pair of elements (bf16 storage)
+//             for the gradient noise, so that its cost stays in 32-bit
 //             integer arithmetic.
 #pragma once
 #include <cstdint>
@@ -47,9 +48,11 @@ GL_HD uint32_t fmix32(uint32_t h) {
 // 24-bit integer uniform in [0, 2^24) from the top bits of a hash.
 GL_HD uint32_t top24(uint64_t h) { return static_cast<uint32_t>(h >> 40); }
 
-// Per-element noise bits of step key (klo, khi) at global index k.
-GL_HD uint32_t noise_bits(uint32_t k, uint32_t klo, uint32_t khi) {
-    return fmix32(fmix32(k ^ klo) ^ khi);
+// Noise word a of step key (klo, khi): with fp32 storage the word of global
+// element a; with bf16 storage its 16-bit halves belong to elements 2a (low)
+// and 2a + 1 (high).
+GL_HD uint32_t noise_word(uint32_t a, uint32_t klo, uint32_t khi) {
+    return fmix32(fmix32(a ^ klo) ^ khi);
 }
 
 }  // namespace gasloc

@@ -46,17 +46,23 @@ def test_bf16_run_stores_bf16_values(orc32):
 
 def test_bf16_run_tracks_f32_run(orc32):
     N, P, R = 8, 2000, 5
-    common = dict(seed=11, lr=3e-4, noise_sigma=0.01)
-    a = orc32.state(oracle.make_problem(N, P, "exp", storage="bf16", **common))
-    b = orc32.state(oracle.make_problem(N, P, "exp", storage="f32", **common))
-    for _ in range(R):
-        for s in (a, b):
+
+    def run(storage, sigma):
+        s = orc32.state(oracle.make_problem(N, P, "exp", storage=storage, seed=11, lr=3e-4, noise_sigma=sigma))
+        for _ in range(R):
             s.local_steps(1)
             s.gossip_round()
+        return s
+
+    # Without noise both stores solve the same problem: bf16 keeps 8
+    # significant bits, so after R rounds the replicas agree to a few bf16
+    # steps of the largest value.
+    a, b = run("bf16", 0.0), run("f32", 0.0)
     xa, xb = a.get_all("x"), b.get_all("x")
-    # bf16 keeps 8 significant bits: after R rounds the replicas agree to a
-    # few bf16 steps of the largest value
     assert np.abs(xa - xb).max() <= R * 2 ** -8 * np.abs(xb).max()
-    # the disagreement between replicas (~1e-4 per element here) is of the
-    # order of one bf16 step, so the consensus error agrees only roughly
+    # With noise the stores draw it on different grids (16 and 24 bits), so
+    # only the statistics agree: the disagreement between replicas (~1e-4 per
+    # element here) is of the order of one bf16 step, and the consensus errors
+    # agree roughly.
+    a, b = run("bf16", 0.01), run("f32", 0.01)
     assert 0.5 < a.consensus_error() / b.consensus_error() < 2.0

@@ -120,6 +120,57 @@ def test_noise_unit_variance_uniform(orc64):
     assert abs(np.corrcoef(xi, xi3)[0, 1]) < 0.03
 
 
+def test_noise_grid_and_words_f32(orc64):
+    # fp32 storage: xi = ((u >> 8) 2^-23 - 1) sqrt3 with u = fmix32 twice over
+    # the element index k with the step key's halves: (xi / sqrt3 + 1) 2^23
+    # is the integer u >> 8.
+    seed, i, n = 29, 1, 3
+    key = orc64.hash(seed, 4, i, n)
+    lo, hi = key & 0xFFFFFFFF, key >> 32
+    for k in [0, 1, 2, 3, 1001, 2 ** 26 + 5]:
+        x = orc64.noise(seed, i, n, k)
+        r = (x / math.sqrt(3) + 1) * 2 ** 23
+        assert abs(r - round(r)) < 1e-6
+        assert round(r) == orc64.fmix32(orc64.fmix32(k ^ lo) ^ hi) >> 8
+
+
+def test_noise_grid_and_pair_words_bf16(orc32, orc64):
+    # bf16 storage: every xi is q * (sqrt3 * 2^-15) for an integer q in [-2^15, 2^15),
+    # rounded once in the build's precision (the f32 build scales fl32(sqrt3));
+    # the two elements of a pair (2j, 2j+1) are the low and high halves of one
+    # 32-bit word, fmix32 twice over j with the step key's halves (fmix32 and
+    # hash are pinned above).
+    s = math.sqrt(3) * 2.0 ** -15
+    s32 = np.float32(np.float32(math.sqrt(3)) * np.float32(2.0 ** -15))
+    seed, i, n = 17, 3, 9
+    key = orc64.hash(seed, 4, i, n)
+    lo, hi = key & 0xFFFFFFFF, key >> 32
+    for j in [0, 1, 2, 1000, 2 ** 20 + 7, 2 ** 29 - 1]:
+        q = []
+        for k in (2 * j, 2 * j + 1):
+            x = orc64.noise(seed, i, n, k, "bf16")
+            r = round(x / s)
+            assert abs(x - r * s) <= 1e-15 and -2 ** 15 <= r < 2 ** 15
+            assert orc32.noise(seed, i, n, k, "bf16") == np.float32(np.float32(r) * s32)
+            q.append(int(r))
+        word = (q[0] + 2 ** 15) | ((q[1] + 2 ** 15) << 16)
+        assert word == orc32.fmix32(orc32.fmix32(j ^ lo) ^ hi)
+
+
+def test_noise_halves_uniform_and_uncorrelated_bf16(orc64):
+    # bf16 storage: the 2^16-point grid is hit uniformly (chi-square over 64
+    # bins), with unit variance, and the two halves of a word are uncorrelated.
+    n = 2 ** 15
+    xi = np.array([orc64.noise(23, 1, 4, k, "bf16") for k in range(2 * n)])
+    assert xi.min() >= -math.sqrt(3) and xi.max() < math.sqrt(3)
+    assert abs(xi.var() - 1) < 0.03
+    cnt = np.histogram(xi, bins=64, range=(-math.sqrt(3), math.sqrt(3)))[0]
+    exp = 2 * n / 64
+    chi2 = ((cnt - exp) ** 2 / exp).sum()
+    assert chi2 < 120          # 63 degrees of freedom: p < 1e-5 above 120
+    assert abs(np.corrcoef(xi[0::2], xi[1::2])[0, 1]) < 0.03
+
+
 def test_permutation_is_uniform(orc32):
     # every permutation of 4 elements appears with frequency 1/24
     from collections import Counter
