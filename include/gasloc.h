@@ -119,7 +119,9 @@ typedef struct gasloc_hparams {
 enum { GASLOC_STORAGE_F32 = 0, GASLOC_STORAGE_BF16 = 1 };
 
 /* Device allocator hooks: alloc returns a device pointer (NULL on failure) of
- * at least `bytes` bytes, 256-byte aligned, usable on `stream`. */
+ * at least `bytes` bytes, 256-byte aligned, usable on `stream`.  A block off
+ * that boundary is handed back to free (the kernels' bulk copies need aligned
+ * rows) and gasloc_start fails with GASLOC_EINVAL. */
 typedef void *(*gasloc_alloc_fn)(size_t bytes, void *stream, void *user);
 typedef void (*gasloc_free_fn)(void *ptr, void *stream, void *user);
 

@@ -1,19 +1,25 @@
 // adamw.cu -- K_adamw: one inner AdamW step (Algorithm 1, inner loop; App. B
 // settings) for every active worker, all replicas in one launch.
 //
-// Memory-bound streaming kernel: per active worker and element it reads the
+// Memory-bound streaming kernels: per active worker and element they read the
 // iterate (x on the first step of a round, else y), m, v and the centre c and
-// writes y, m, v -- 28 bytes in fp32 storage, 14 in bf16 -- plus the shared
+// write y, m, v -- 28 bytes in fp32 storage, 14 in bf16 -- plus the shared
 // curvature h per element (h is per worker in the heterogeneous workload).
-// One thread owns a column of 4 consecutive elements of a tile and walks the
-// active workers U at a time (fp32: U = 4, or 3 with per-worker h; bf16: 8 or
-// 6), issuing all of their loads before any arithmetic so that about 256
-// bytes of requests per thread stay in flight.  The synthetic gradient
-// g = h (y - c) + sigma xi is formed in registers; xi comes from a 32-bit
-// counter hash of the element index and the step key (of the index of the
-// element pair with bf16 storage), so the gradient costs no memory traffic.  The step's per-worker scalars (bias corrections, noise
+// The synthetic gradient g = h (y - c) + sigma xi is formed in registers; xi
+// comes from a 32-bit counter hash of the element index and the step key (of
+// the index of the element pair with bf16 storage), so the gradient costs no
+// memory traffic.  The step's per-worker scalars (bias corrections, noise
 // keys) come from the step table; the launch's last CTA to copy it advances
 // the step counters and writes the next step's scalars.
+//
+// fp32 storage (adamw_kernel): one thread owns a column of 4 consecutive
+// elements of a tile and walks the active workers U at a time (U = 4, or 3
+// with per-worker h), issuing all of their loads before any arithmetic so
+// that about 256 bytes of requests per thread stay in flight.
+// bf16 storage (adamw_staged_kernel): a producer warp stages the rows in
+// shared memory with bulk copies while 256 consumer threads compute (see
+// there); with half the bytes per element the arithmetic sets the pace, and
+// the consumers must not wait on their own loads.
 //
 // Per element, in fp32 with one IEEE rounding per operation (the oracle's
 // order; pairs of lanes share f32x2 instructions, which round each lane as
@@ -121,6 +127,7 @@ __device__ __forceinline__ void noise4_pairs(uint32_t k, uint32_t klo, uint32_t 
 // launch-wide fl32(1 - lr * weight_decay).
 template <int U, bool PER_WORKER_H, bool SCHED, typename T>
 __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
+    static_assert(std::is_same<T, float>::value, "bf16 storage runs adamw_staged_kernel");
     using E = Elem<T>;
     const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
                     x2::splat(a.eps), x2::splat(a.sigma)};
@@ -198,20 +205,11 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
                     const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
                     const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
                                  Cu = E::unpack(Cc[u]);
-                    float2 m01, v01, m23, v23, y01, y23;
-                    if constexpr (std::is_same<T, bf16>::value) {
-                        float2 xi01, xi23;
-                        noise4_pairs(k0, klo, khi, xi01, xi23);
-                        y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4), xi01, nstep, isb,
-                                         dec, kc, m01, v01);
-                        y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4), xi23, nstep, isb,
-                                         dec, kc, m23, v23);
-                    } else {
-                        y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
-                                         noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
-                        y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
-                                         noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
-                    }
+                    float2 m01, v01, m23, v23;
+                    const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
+                                                  noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
+                    const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
+                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
                     const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
                     const int64_t o = i * d.wstride + off;
                     if (nvalid == 4) {
@@ -234,10 +232,231 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     }
 }
 
-// Workers per load batch: 16 (fp32) or 8 (bf16) bytes per load, so that a
-// thread keeps about 256 bytes of loads in flight in both storage types.
+// ---------------------------------------------------------------------------
+// Staged variant, used with bf16 storage.  With half the bytes per element
+// the arithmetic, not the memory, sets the pace, and a thread that waits on
+// its own loads (as above) leaves no loads in flight while it computes.  Here
+// a producer warp keeps the HBM busy: for each unit of work (a tile of 1024
+// elements for a group of G workers) its lanes issue one 1-D bulk copy per
+// row -- the iterate (y, or x on the worker's first step of the round), m, v,
+// c, and h (the tile's shared row, or each worker's own) -- into a ring of
+// kStages shared-memory stages, completing on the stage's `full` mbarrier.
+// The 256 consumer threads (a column of 4 elements each) read their rows from
+// shared memory, take the step exactly as above and store y, m, v straight to
+// global memory, then release the stage on its `empty` mbarrier.  Every wait
+// is bounded: on a timeout the CTA records kDevWaitTimeout, stops computing
+// but keeps releasing stages, and the producer stops issuing and waits
+// (bounded) for the copies it has in flight before it leaves.
+constexpr int kStagedConsumers = 256;
+constexpr int kStagedThreads = kStagedConsumers + 32;
+constexpr int kStagedTile = 4 * kStagedConsumers;   // elements per tile (the host's tile size)
+constexpr uint64_t kStagedWaitNs = 2000000000ull;
+
+template <bool PER_WORKER_H>
+struct StagedShape {
+    // Measured on the 8-worker GPT-2-small bf16 workload (fraction of the copy
+    // peak): groups of 4 workers, 2 stages, 3 CTAs per SM 0.931; 3 stages and
+    // 2 CTAs 0.842; groups of 2 with 3 or 4 stages and 3 CTAs 0.853 / 0.856;
+    // single workers, 4 stages, 4 CTAs 0.725.
+    static constexpr int kGroup = PER_WORKER_H ? 3 : 4;           // workers per unit
+    static constexpr int kStages = 2;                             // ring depth
+    static constexpr int kMinBlocks = 3;                          // CTAs per SM
+    static constexpr int kArrs = PER_WORKER_H ? 5 : 4;            // rows per worker
+    static constexpr int kSegs = kArrs * kGroup + (PER_WORKER_H ? 0 : 1);
+    static constexpr size_t kStageBytes = static_cast<size_t>(kSegs) * kStagedTile * sizeof(bf16);
+    static constexpr size_t kBarOffset = kStages * kStageBytes;
+    static constexpr size_t kSmem = kBarOffset + 2 * kStages * sizeof(uint64_t);
+};
+
+__device__ __forceinline__ void mbar_release(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
+}
+
+template <bool PER_WORKER_H, bool SCHED>
+__global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMinBlocks)
+    adamw_staged_kernel(const AdamwArgs a) {
+    using T = bf16;
+    using E = Elem<T>;
+    using SS = StagedShape<PER_WORKER_H>;
+    constexpr int G = SS::kGroup;
+    constexpr int kStages = SS::kStages;
+    extern __shared__ __align__(128) unsigned char smem[];
+    T *stages = reinterpret_cast<T *>(smem);
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + SS::kBarOffset);
+    uint64_t *empty = full + kStages;
+    __shared__ StepTable tab;
+    __shared__ int last_copy;
+    __shared__ int abort_flag;
+
+    for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += blockDim.x)
+        reinterpret_cast<uint32_t *>(&tab)[q] = reinterpret_cast<const uint32_t *>(a.table)[q];
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], kStagedConsumers / 32);
+        }
+        ptx::fence_mbar_init();
+        abort_flag = 0;
+    }
+    __syncthreads();
+    // the last CTA to have copied the scalars advances the counters and
+    // writes the next step's scalars (as in adamw_kernel)
+    if (threadIdx.x == 0) last_copy = atomicAdd(a.ticket, 1u) == gridDim.x - 1u;
+    __syncthreads();
+    if (last_copy && threadIdx.x < 32) {
+        const int i = threadIdx.x;
+        if (i < a.n_workers && ((a.active_mask >> i) & 1u)) {
+            const int64_t n = a.state->nsteps[i] + 1;
+            const double p1 = __dmul_rn(a.state->p1[i], a.beta1d), p2 = __dmul_rn(a.state->p2[i], a.beta2d);
+            a.state->nsteps[i] = n;
+            a.state->p1[i] = p1;
+            a.state->p2[i] = p2;
+            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d),
+                               lr_of_step(n + 1, a.lr_sched, a.lr_steps, a.lr_after), a.wd, a.seed);
+        }
+        if (i == 0) *a.ticket = 0u;
+    }
+
+    // units of this CTA: its tiles (grid stride) x the groups of G active workers
+    const int ngroups = (a.n_active + G - 1) / G;
+    const int64_t my_tiles = a.ntiles > blockIdx.x ? (a.ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+    const int64_t my_n = my_tiles * ngroups;
+    const int lane = threadIdx.x & 31;
+    auto seg = [&](int s, int k) {   // row k of stage s
+        return stages + (static_cast<size_t>(s) * SS::kSegs + k) * kStagedTile;
+    };
+
+    if (threadIdx.x >= kStagedConsumers) {
+        // ---------------------------------------------------------- producer ---
+        int64_t issued = 0;
+        bool aborted = false;
+        for (int64_t it = 0; it < my_n; ++it) {
+            const int s = static_cast<int>(it % kStages);
+            if (it >= kStages) {
+                const int64_t j = it - kStages;
+                const bool ok = ptx::mbar_wait_bounded(&empty[s], static_cast<uint32_t>((j / kStages) & 1),
+                                                       kStagedWaitNs);
+                if (!__all_sync(0xffffffffu, ok)) {
+                    aborted = true;
+                    break;
+                }
+            }
+            if (__any_sync(0xffffffffu, abort_flag != 0)) {
+                aborted = true;
+                break;
+            }
+            const int64_t ti = blockIdx.x + (it / ngroups) * gridDim.x;
+            const int a0 = static_cast<int>(it % ngroups) * G;
+            const Tile tl = a.tiles[ti];
+            const TensorDesc &d = a.tens[tl.tensor];
+            const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
+            const int lenr = (tl.len + 7) & ~7;   // whole 16-byte pieces (the row padding is allocated)
+            const uint32_t bytes = static_cast<uint32_t>(lenr) * sizeof(T);
+            const int nsegs = SS::kArrs * nw + (PER_WORKER_H ? 0 : 1);
+            if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsegs) * bytes);
+            __syncwarp();
+            if (lane < nsegs && span_ok(0, lenr, kStagedTile, a.err) &&
+                aligned16_ok((tl.start) * static_cast<int64_t>(sizeof(T)), a.err)) {
+                const T *src = nullptr;
+                int k = lane;
+                if (!PER_WORKER_H && lane == SS::kArrs * nw) {   // the tile's shared curvature row
+                    if (row_ok(0, 1, tl.start, lenr, d.wstride, a.err)) src = as<T>(static_cast<const void *>(d.h)) + tl.start;
+                    k = SS::kArrs * G;
+                } else {
+                    const int w = lane / SS::kArrs, arr = lane % SS::kArrs;
+                    const int i = a.worker[a0 + w];
+                    if (row_ok(i, a.n_workers, tl.start, lenr, d.wstride, a.err)) {
+                        const int64_t o = i * d.wstride + tl.start;
+                        const void *base = arr == 0 ? (((a.from_x_mask >> i) & 1u) ? d.x : d.y)
+                                         : arr == 1 ? d.m : arr == 2 ? d.v : arr == 3 ? d.c : d.h;
+                        src = as<T>(base) + (arr == 4 ? i * d.hstride + tl.start : o);
+                    }
+                }
+                if (src) ptx::bulk_g2s(seg(s, k), src, bytes, &full[s]);
+            }
+            issued = it + 1;
+        }
+        if (aborted) {
+            if (lane == 0) {
+                abort_flag = 1;
+                atomicCAS(a.err, static_cast<int32_t>(kDevOk), static_cast<int32_t>(kDevWaitTimeout));
+            }
+            // copies still in flight land before the CTA leaves (bounded)
+            for (int64_t j = issued - kStages > 0 ? issued - kStages : 0; j < issued; ++j)
+                ptx::mbar_wait_bounded(&full[j % kStages], static_cast<uint32_t>((j / kStages) & 1), kStagedWaitNs);
+        }
+        return;
+    }
+
+    // ------------------------------------------------------------ consumers ---
+    const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
+                    x2::splat(a.eps), x2::splat(a.sigma)};
+    const int e0 = 4 * threadIdx.x;
+    for (int64_t it = 0; it < my_n; ++it) {
+        const int s = static_cast<int>(it % kStages);
+        bool ok = abort_flag == 0;
+        if (ok && !ptx::mbar_wait_bounded(&full[s], static_cast<uint32_t>((it / kStages) & 1), kStagedWaitNs)) {
+            ok = false;
+            abort_flag = 1;
+            atomicCAS(a.err, static_cast<int32_t>(kDevOk), static_cast<int32_t>(kDevWaitTimeout));
+        }
+        const int64_t ti = blockIdx.x + (it / ngroups) * gridDim.x;
+        const int a0 = static_cast<int>(it % ngroups) * G;
+        const Tile tl = a.tiles[ti];
+        if (ok && e0 < tl.len) {
+            const TensorDesc &d = a.tens[tl.tensor];
+            T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
+            const int64_t off = tl.start + e0;
+            const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
+            const uint32_t k0 = static_cast<uint32_t>(d.goff + off);   // global index of the column's first element
+            const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
+            float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (!PER_WORKER_H) hs = E::unpack(*reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * G) + e0));
+#pragma unroll
+            for (int w = 0; w < G; ++w) {
+                if (w >= nw) break;
+                const int i = a.worker[a0 + w];
+                if (!row_ok(i, a.n_workers, off, 4, d.wstride, a.err)) continue;
+                const uint2 *rw = reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * w) + e0);
+                constexpr int kSegStep = kStagedTile / 4;   // uint2 words per row
+                const float4 Yu = E::unpack(rw[0]), Mu = E::unpack(rw[kSegStep]), Vu = E::unpack(rw[2 * kSegStep]),
+                             Cu = E::unpack(rw[3 * kSegStep]);
+                const float4 h4 = PER_WORKER_H ? E::unpack(rw[4 * kSegStep]) : hs;
+                const float2 nstep = x2::splat(-tab.step[i]);
+                const float2 isb = x2::splat(tab.isb[i]);
+                const float2 dec = SCHED ? x2::splat(tab.decay[i]) : x2::splat(a.decay);
+                float2 m01, v01, m23, v23, xi01, xi23;
+                noise4_pairs(k0, tab.key_lo[i], tab.key_hi[i], xi01, xi23);
+                const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4), xi01, nstep,
+                                              isb, dec, kc, m01, v01);
+                const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4), xi23, nstep,
+                                              isb, dec, kc, m23, v23);
+                const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
+                const int64_t o = i * d.wstride + off;
+                if (nvalid == 4) {
+                    E::template store4<kSt>(Yw + o, yo);
+                    E::template store4<kSt>(Mw + o, mo);
+                    E::template store4<kSt>(Vw + o, vo);
+                } else {
+                    const float ya[4] = {yo.x, yo.y, yo.z, yo.w};
+                    const float ma[4] = {mo.x, mo.y, mo.z, mo.w};
+                    const float va[4] = {vo.x, vo.y, vo.z, vo.w};
+                    for (int l = 0; l < nvalid; ++l) {
+                        E::store1(Yw + o + l, ya[l]);
+                        E::store1(Mw + o + l, ma[l]);
+                        E::store1(Vw + o + l, va[l]);
+                    }
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_release(&empty[s]);
+    }
+}
+
+// Workers per load batch of adamw_kernel: 16-byte loads, so that a thread
+// keeps about 256 bytes of loads in flight.
 template <typename T> struct Batch { static constexpr int kShared = 4, kPerWorkerH = 3; };
-template <> struct Batch<bf16> { static constexpr int kShared = 8, kPerWorkerH = 6; };
 
 template <typename T>
 int blocks_per_sm(int block, bool per_worker_h) {
@@ -250,6 +469,43 @@ int blocks_per_sm(int block, bool per_worker_h) {
                                                             block, 0);
     if (e != cudaSuccess) return 1;
     return nb > 0 ? nb : 1;
+}
+
+template <bool P, bool S>
+const void *staged_ptr() {
+    return reinterpret_cast<const void *>(adamw_staged_kernel<P, S>);
+}
+
+// Occupancy of the staged kernel with its shared memory (the attribute is set
+// here, before the first launch).
+int staged_blocks_per_sm(bool per_worker_h) {
+    const size_t smem = per_worker_h ? StagedShape<true>::kSmem : StagedShape<false>::kSmem;
+    const void *k[2] = {per_worker_h ? staged_ptr<true, false>() : staged_ptr<false, false>(),
+                        per_worker_h ? staged_ptr<true, true>() : staged_ptr<false, true>()};
+    for (const void *f : k)
+        if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+            cudaSuccess)
+            return 1;
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k[0], kStagedThreads, smem) != cudaSuccess) return 1;
+    return nb > 0 ? nb : 1;
+}
+
+void launch_staged(const AdamwArgs &a, int grid, cudaStream_t s) {
+    const bool sched = a.lr_steps > 0;
+    if (a.per_worker_h) {
+        constexpr size_t m = StagedShape<true>::kSmem;
+        if (sched)
+            adamw_staged_kernel<true, true><<<grid, kStagedThreads, m, s>>>(a);
+        else
+            adamw_staged_kernel<true, false><<<grid, kStagedThreads, m, s>>>(a);
+    } else {
+        constexpr size_t m = StagedShape<false>::kSmem;
+        if (sched)
+            adamw_staged_kernel<false, true><<<grid, kStagedThreads, m, s>>>(a);
+        else
+            adamw_staged_kernel<false, false><<<grid, kStagedThreads, m, s>>>(a);
+    }
 }
 
 template <typename T>
@@ -269,14 +525,13 @@ void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
 }  // namespace
 
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage) {
-    return storage == kStoreBF16 ? blocks_per_sm<bf16>(block, per_worker_h)
-                                 : blocks_per_sm<float>(block, per_worker_h);
+    return storage == kStoreBF16 ? staged_blocks_per_sm(per_worker_h) : blocks_per_sm<float>(block, per_worker_h);
 }
 
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s) {
     (void)block;
     if (a.storage == kStoreBF16)
-        launch<bf16>(a, grid, s);
+        launch_staged(a, grid, s);
     else
         launch<float>(a, grid, s);
     return cudaGetLastError();

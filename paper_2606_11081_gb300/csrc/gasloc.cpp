@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdint>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -152,6 +153,7 @@ struct gasloc_ctx {
     bool topo_static = false, topo_ready = false;
     int64_t launches = 0;
 
+    bool misaligned = false;   // an allocator hook returned a block off a 256-byte boundary
     void *dalloc(size_t bytes) {
         bytes = static_cast<size_t>(round_up(static_cast<int64_t>(bytes ? bytes : 1), 256));
         void *p = nullptr;
@@ -160,6 +162,14 @@ struct gasloc_ctx {
         } else if (cudaMalloc(&p, bytes) != cudaSuccess) {
             cudaGetLastError();
             p = nullptr;
+        }
+        if (p && (reinterpret_cast<uintptr_t>(p) & 255u) != 0) {
+            // the bulk and tensor-map copies address rows at 16-byte
+            // boundaries: hand the block back rather than fault on it
+            if (free_fn) free_fn(p, stream, alloc_user);
+            else if (!alloc) cudaFree(p);
+            misaligned = true;
+            return nullptr;
         }
         if (p) allocs.emplace_back(p, bytes);
         return p;
@@ -559,6 +569,8 @@ int gasloc_start(gasloc_ctx *c) {
     auto oom = [&](const char *what) {
         c->release_all();
         c->tens_h.clear();
+        if (c->misaligned)
+            return fail(GASLOC_EINVAL, "the allocator returned a block that is not 256-byte aligned (%s)", what);
         return fail(GASLOC_ENOMEM, "device allocation failed (%s)", what);
     };
 

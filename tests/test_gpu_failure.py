@@ -44,3 +44,34 @@ def test_bounded_wait_expires_and_context_survives():
         np.testing.assert_array_equal(ctx.read_all("x"), st.get_all("x").astype(np.float32))
         with pytest.raises(g.GaslocError):
             g._check(g.gasloc_selftest_bounded_wait(ctx.h, 0))      # limit out of range
+
+
+def test_misaligned_allocator_block_is_refused():
+    # An allocator hook that returns blocks 16 bytes past a 256-byte boundary:
+    # gasloc_start hands each block back and fails with EINVAL before any
+    # kernel could address it.
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    gbuild.build()
+    dev = torch.cuda.current_device()
+    live = {}
+
+    def _alloc(nbytes, stream, user):
+        base = torch.cuda.caching_allocator_alloc(int(nbytes) + 256, dev, stream if stream else 0)
+        live[base + 16] = base
+        return base + 16
+
+    def _free(ptr, stream, user):
+        torch.cuda.caching_allocator_delete(live.pop(ptr))
+
+    af, ff = g.ALLOC_FN(_alloc), g.FREE_FN(_free)
+    h = g.gasloc_init(4, 5000, "ring", 1)
+    try:
+        g.gasloc_set_allocator(h, af, ff, None)
+        with pytest.raises(g.GaslocError) as ei:
+            g.gasloc_start(h)
+        assert ei.value.code == g.EINVAL and "256-byte aligned" in str(ei.value)
+        assert not live                       # every block went back
+    finally:
+        g.gasloc_destroy(h)

@@ -271,14 +271,15 @@ def test_gather_rejects_bad_index():
                                       ctx.read("x", 1)[[0, 99, 42]])
 
 
-@pytest.mark.parametrize("storage", ["f32", "bf16"])
-def test_lr_schedule_matches_oracle(storage):
+@pytest.mark.parametrize("storage,per_h", [("f32", False), ("bf16", False), ("bf16", True)])
+def test_lr_schedule_matches_oracle(storage, per_h):
     # App. B's warm-up + cosine schedule runs over each worker's own local
     # steps: with different H_i the workers sit at different points of it, and
     # the busiest one passes the warm-up, the decay and the held final rate.
     N, P, R = 6, 2 * 1024 + 9, 5
     Hi = np.array([1, 3, 2, 4, 1, 2], np.int32)
-    hp = dict(lr=4e-3, storage=storage, lr_total_steps=9, lr_warmup_frac=0.25, lr_final_frac=0.1)
+    hp = dict(lr=4e-3, storage=storage, lr_total_steps=9, lr_warmup_frac=0.25, lr_final_frac=0.1,
+              per_worker_h=per_h)
     ctx, st = make_pair(N, P, "ring", seed=31, hp=hp, Hi=Hi)
     with ctx:
         for _ in range(R):
