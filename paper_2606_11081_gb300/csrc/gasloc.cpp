@@ -133,7 +133,7 @@ struct gasloc_ctx {
     int64_t lr_sched_cap = 0, lr_steps = 0;
     double lr_after = 0.0;           // lr of every later step (the constant lr without a schedule)
     StepTable *table_d = nullptr;    // scalars of each worker's next local step
-    int64_t table_gen = -1;          // gen at which table_d was last refreshed
+    uint64_t table_gen = 0;          // gen at which table_d was last refreshed (0: never; gen starts at 1)
     cudaStream_t cap_stream = nullptr;
     cudaGraphExec_t graph = nullptr; // one round, captured by gasloc_run
     int32_t graph_H = 0;
