@@ -170,7 +170,10 @@ int gasloc_set_stream(gasloc_ctx *ctx, void *cuda_stream);
 /* Allocates the replica store and initialises it on the device: identical
  * x_i = x_0 ~ N(0, 0.02^2) on every worker (Prop. 2 assumes equal initial
  * replicas), y_i = x_i, centres c_i ~ N(0,1), curvature h ~ U(0.1, 1), and
- * m = v = b = 0.  Asynchronous.  ENOMEM if an allocation fails. */
+ * m = v = b = 0.  Besides the store (x, y, m, v, b, c per worker and h) it
+ * allocates the round tables and one array of n_params floats for the
+ * average's way to host memory.  Asynchronous.  ENOMEM if an allocation
+ * fails, EINVAL if an allocator hook returns a misaligned block. */
 int gasloc_start(gasloc_ctx *ctx);
 
 /* Per-worker local step counts H_i (Sec. 3.2, heterogeneous local steps),
@@ -257,7 +260,9 @@ int gasloc_get_topology(gasloc_ctx *ctx, int64_t round, int32_t *nbr, float *w, 
 /* Output of Algorithm 1: xbar = (1/n) sum_i x_i into dst (n_params fp32,
  * device memory; concatenation order).  Asynchronous. */
 int gasloc_average(gasloc_ctx *ctx, float *dst_device);
-/* Same into host memory (pinned or pageable).  Synchronising. */
+/* Same into host memory (pinned or pageable), through a device buffer of
+ * n_params floats that the context allocates in gasloc_start.
+ * Synchronising. */
 int gasloc_average_host(gasloc_ctx *ctx, float *dst_host);
 
 /* Device pointer of buffer `which` for tensor `tensor`: worker i's slice

@@ -133,6 +133,7 @@ struct gasloc_ctx {
     int64_t lr_sched_cap = 0, lr_steps = 0;
     double lr_after = 0.0;           // lr of every later step (the constant lr without a schedule)
     StepTable *table_d = nullptr;    // scalars of each worker's next local step
+    float *avg_d = nullptr;          // n_params floats: the average on its way to host memory
     uint64_t table_gen = 0;          // gen at which table_d was last refreshed (0: never; gen starts at 1)
     cudaStream_t cap_stream = nullptr;
     cudaGraphExec_t graph = nullptr; // one round, captured by gasloc_run
@@ -195,6 +196,7 @@ struct gasloc_ctx {
             else cudaFree(pr.first);
         }
         allocs.clear();
+        avg_d = nullptr;
         if (pinned) cudaFreeHost(pinned);
         pinned = nullptr;
     }
@@ -637,8 +639,11 @@ int gasloc_start(gasloc_ctx *c) {
     c->state_d = static_cast<DevState *>(c->dalloc(sizeof(DevState)));
     c->table_d = static_cast<StepTable *>(c->dalloc(sizeof(StepTable)));
     c->err_d = static_cast<int32_t *>(c->dalloc(sizeof(int32_t) * 4));
+    // allocated with the rest, so that reading the average back at the end of
+    // a run costs the kernel and the copy only
+    c->avg_d = static_cast<float *>(c->dalloc(static_cast<size_t>(c->P) * 4));
     if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->maps_d || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
-        !c->ce_d || !c->err_d || !c->ce_ring || !c->state_d || !c->table_d)
+        !c->ce_d || !c->err_d || !c->ce_ring || !c->state_d || !c->table_d || !c->avg_d)
         return oom("tables");
     if (cudaMallocHost(&c->pinned, 64 + sizeof(Topo)) != cudaSuccess) {
         cudaGetLastError();
@@ -1029,16 +1034,13 @@ int gasloc_average_host(gasloc_ctx *c, float *dst) {
     int rc = check_started(c);
     if (rc) return rc;
     if (!dst) return fail(GASLOC_EINVAL, "dst is NULL");
-    float *tmp = static_cast<float *>(c->dalloc(static_cast<size_t>(c->P) * 4));
-    if (!tmp) return fail(GASLOC_ENOMEM, "device allocation failed (average)");
-    rc = gasloc_average(c, tmp);
+    rc = gasloc_average(c, c->avg_d);
     if (!rc) {
-        cudaError_t e = cudaMemcpyAsync(dst, tmp, static_cast<size_t>(c->P) * 4, cudaMemcpyDeviceToHost, c->stream);
+        cudaError_t e = cudaMemcpyAsync(dst, c->avg_d, static_cast<size_t>(c->P) * 4, cudaMemcpyDeviceToHost, c->stream);
         if (e != cudaSuccess) rc = cuda_fail(e, "copying the average");
         else rc = sync_and_check(c);
     }
     cudaStreamSynchronize(c->stream);
-    c->dfree(tmp);
     return rc;
 }
 
