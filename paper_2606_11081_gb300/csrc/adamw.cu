@@ -265,8 +265,18 @@ struct StagedShape {
     static constexpr int kSegs = kArrs * kGroup + (PER_WORKER_H ? 0 : 1);
     static constexpr size_t kStageBytes = static_cast<size_t>(kSegs) * kStagedTile * sizeof(bf16);
     static constexpr size_t kBarOffset = kStages * kStageBytes;
-    static constexpr size_t kSmem = kBarOffset + 2 * kStages * sizeof(uint64_t);
+    static constexpr size_t kDescOffset = kBarOffset + 2 * kStages * sizeof(uint64_t);
+    static constexpr size_t kSmem = kDescOffset + kStages * 64;
 };
+
+// What the consumers need of a unit's tile, written by the producer beside
+// the stage's rows (so that the consumers make no global loads of their own).
+struct UnitDesc {
+    int64_t start, wstride, goff;   // tile start in the tensor, row stride, global index of element 0
+    void *y, *m, *v;
+    int32_t len, pad;
+};
+static_assert(sizeof(UnitDesc) <= 64, "one 64-byte slot per stage");
 
 __device__ __forceinline__ void mbar_release(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
@@ -284,6 +294,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
     T *stages = reinterpret_cast<T *>(smem);
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + SS::kBarOffset);
     uint64_t *empty = full + kStages;
+    UnitDesc *descs = reinterpret_cast<UnitDesc *>(smem + SS::kDescOffset);
     __shared__ StepTable tab;
     __shared__ int last_copy;
     __shared__ int abort_flag;
@@ -353,7 +364,19 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
             const int lenr = (tl.len + 7) & ~7;   // whole 16-byte pieces (the row padding is allocated)
             const uint32_t bytes = static_cast<uint32_t>(lenr) * sizeof(T);
             const int nsegs = SS::kArrs * nw + (PER_WORKER_H ? 0 : 1);
-            if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsegs) * bytes);
+            if (lane == 0) {
+                // the descriptor's stores precede the arrive (release), the
+                // consumers read it after their wait (acquire)
+                UnitDesc &u = descs[s];
+                u.start = tl.start;
+                u.wstride = d.wstride;
+                u.goff = d.goff;
+                u.y = d.y;
+                u.m = d.m;
+                u.v = d.v;
+                u.len = tl.len;
+                ptx::mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsegs) * bytes);
+            }
             __syncwarp();
             if (lane < nsegs && span_ok(0, lenr, kStagedTile, a.err) &&
                 aligned16_ok((tl.start) * static_cast<int64_t>(sizeof(T)), a.err)) {
@@ -400,15 +423,14 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
             abort_flag = 1;
             atomicCAS(a.err, static_cast<int32_t>(kDevOk), static_cast<int32_t>(kDevWaitTimeout));
         }
-        const int64_t ti = blockIdx.x + (it / ngroups) * gridDim.x;
         const int a0 = static_cast<int>(it % ngroups) * G;
-        const Tile tl = a.tiles[ti];
-        if (ok && e0 < tl.len) {
-            const TensorDesc &d = a.tens[tl.tensor];
-            T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
-            const int64_t off = tl.start + e0;
-            const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-            const uint32_t k0 = static_cast<uint32_t>(d.goff + off);   // global index of the column's first element
+        const UnitDesc &u = descs[s];
+        if (ok && e0 < u.len) {
+            T *Yw = as<T>(u.y), *Mw = as<T>(u.m), *Vw = as<T>(u.v);
+            const int64_t wstride = u.wstride;
+            const int64_t off = u.start + e0;
+            const int nvalid = u.len - e0 < 4 ? u.len - e0 : 4;
+            const uint32_t k0 = static_cast<uint32_t>(u.goff + off);   // global index of the column's first element
             const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
             float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
             if (!PER_WORKER_H) hs = E::unpack(*reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * G) + e0));
@@ -416,7 +438,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
             for (int w = 0; w < G; ++w) {
                 if (w >= nw) break;
                 const int i = a.worker[a0 + w];
-                if (!row_ok(i, a.n_workers, off, 4, d.wstride, a.err)) continue;
+                if (!row_ok(i, a.n_workers, off, 4, wstride, a.err)) continue;
                 const uint2 *rw = reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * w) + e0);
                 constexpr int kSegStep = kStagedTile / 4;   // uint2 words per row
                 const float4 Yu = E::unpack(rw[0]), Mu = E::unpack(rw[kSegStep]), Vu = E::unpack(rw[2 * kSegStep]),
@@ -432,7 +454,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
                 const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4), xi23, nstep,
                                               isb, dec, kc, m23, v23);
                 const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
-                const int64_t o = i * d.wstride + off;
+                const int64_t o = i * wstride + off;
                 if (nvalid == 4) {
                     E::template store4<kSt>(Yw + o, yo);
                     E::template store4<kSt>(Mw + o, mo);
