@@ -233,11 +233,11 @@ def test_tensor_list_equals_flat():
         np.testing.assert_array_equal(v.cpu().numpy(), b.read_all("x")[:, 1003:1003 + 4097])
 
 
-@pytest.mark.parametrize("sched", [0, 8])
-def test_resume_is_exact(tmp_path, sched):
+@pytest.mark.parametrize("sched,storage", [(0, "f32"), (8, "f32"), (8, "bf16")])
+def test_resume_is_exact(tmp_path, sched, storage):
     # the resumed context starts with other hyperparameters (no lr schedule):
     # the checkpoint's, schedule included, take over
-    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True, lr_total_steps=sched)
+    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True, lr_total_steps=sched, storage=storage)
     a, _ = make_pair(6, 3000, "exp", seed=21, hp=hp, Hi=[1, 2, 3, 1, 2, 3])
     with a:
         for _ in range(3):
