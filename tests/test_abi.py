@@ -61,7 +61,11 @@ def test_hparams_validation(lib):
     c = g.gasloc_init(4, 100, "ring", 1)
     try:
         for bad in [dict(lr=-1.0), dict(beta1=1.0), dict(beta2=-0.1), dict(eps=0.0),
-                    dict(edge_prob=1.5), dict(outer_lr=-0.1), dict(gamma=float("nan"))]:
+                    dict(edge_prob=1.5), dict(outer_lr=-0.1), dict(gamma=float("nan")),
+                    dict(lr_total_steps=-1), dict(lr_total_steps=2 ** 24 + 1),
+                    dict(lr_total_steps=10, lr_warmup_frac=1.5),
+                    dict(lr_total_steps=10, lr_warmup_start=-0.1),
+                    dict(lr_total_steps=10, lr_final_frac=float("nan"))]:
             with pytest.raises(g.GaslocError) as e:
                 g.gasloc_set_hparams(c, g.make_hparams(**bad))
             assert e.value.code == g.EINVAL
