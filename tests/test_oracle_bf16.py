@@ -66,3 +66,44 @@ def test_bf16_run_tracks_f32_run(orc32):
     # agree roughly.
     a, b = run("bf16", 0.01), run("f32", 0.01)
     assert 0.5 < a.consensus_error() / b.consensus_error() < 2.0
+
+
+def _bf16_of(t):
+    # the oracle's rule for a REAL result: to binary32, then to bfloat16
+    return t.float().to(torch.bfloat16).to(torch.float64)
+
+
+def test_bf16_adamw_matches_torch_with_bf16_rounding(orc64):
+    # H AdamW steps with a bf16 store against torch.optim.AdamW in fp64 whose
+    # parameter and both moment buffers are rounded to bf16 after every step,
+    # with the gradient noise of the bf16 grid.  The two sides order their
+    # fp64 operations differently, so a value that lands on a bf16 rounding
+    # boundary may round the other way: at most one bf16 step apart, rarely.
+    N, P, H = 2, 600, 3
+    pb = oracle.make_problem(N, P, "none", seed=77, lr=3e-3, noise_sigma=0.05, outer="sgd",
+                             outer_lr=1.0, outer_momentum=0.0, storage="bf16")
+    st = orc64.state(pb)
+    x0, c, h = st.get("x", 0), st.get_all("c"), st.get("h", 0)
+    st.local_steps(H)
+    for i in range(N):
+        p = torch.tensor(x0, dtype=torch.float64, requires_grad=True)
+        opt = torch.optim.AdamW([p], lr=pb.lr, betas=(pb.beta1, pb.beta2), eps=pb.eps,
+                                weight_decay=pb.weight_decay)
+        ct, ht = torch.tensor(c[i], dtype=torch.float64), torch.tensor(h, dtype=torch.float64)
+        for n in range(1, H + 1):
+            xi = torch.tensor([orc64.noise(pb.seed, i, n, k, "bf16") for k in range(P)], dtype=torch.float64)
+            with torch.no_grad():
+                p.grad = ht * (p - ct) + pb.noise_sigma * xi
+            opt.step()
+            with torch.no_grad():
+                p.copy_(_bf16_of(p))
+                s = opt.state[p]
+                s["exp_avg"].copy_(_bf16_of(s["exp_avg"]))
+                s["exp_avg_sq"].copy_(_bf16_of(s["exp_avg_sq"]))
+        s = opt.state[p]
+        for name, ref in (("y", p.detach()), ("m", s["exp_avg"]), ("v", s["exp_avg_sq"])):
+            got, ref = st.get(name, i), ref.numpy()
+            diff = got != ref
+            ulp = np.abs(ref) * 2.0 ** -7
+            assert np.all(np.abs(got - ref)[diff] <= ulp[diff] * 1.0001), name
+            assert diff.mean() <= 0.01, (name, diff.mean())
