@@ -44,11 +44,14 @@ NOMINAL_HBM_GBS = 8000.0      # the metric's "vs 8 TB/s" (GB300 HBM3e, nominal)
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed rounds (default: the workload's round count)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gasloc", choices=["gasloc", "reference"])
     ap.add_argument("--workload", default=None)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--extras", default="all",
+                    help="other workloads timed after the main one: 'all', 'none' or a comma list")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     return ap.parse_args()
@@ -256,10 +259,126 @@ def workload_config(w, args):
             "l2": "inputs larger than L2 (%.1f GB replica state per GPU, no flush)" % state_gb}
 
 
+def adamw_bytes_of(w, steps, es):
+    """Algorithmic bytes of every AdamW launch of one round (a launch per
+    sub-step; sub-step s steps the workers with H_i > s)."""
+    per_h = bool(w.hp.get("per_worker_h"))
+    out = []
+    for s in range(max(steps)):
+        act = sum(1 for h in steps if h > s)
+        if act:
+            out.append(((8 * es * act) if per_h else (7 * es * act + es)) * w.n_params)
+    return out
+
+
+def time_rounds(ctx, torch, stream, K, H):
+    """K rounds with CUDA events around the local steps and the gossip round of
+    each; returns (total ms, local-step ms, gossip ms) summed over the rounds."""
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(K):
+        ev[k][0].record(stream)
+        ctx.local_steps(H)
+        ev[k][1].record(stream)
+        ctx.gossip_round()
+        ev[k][2].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    ms = t_start.elapsed_time(t_end)
+    local_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(K))
+    gossip_ms = sum(ev[k][1].elapsed_time(ev[k][2]) for k in range(K))
+    return ms, local_ms, gossip_ms
+
+
+def kernel_entry(bytes_, time_ms, peak, **extra):
+    """Rate of `bytes_` algorithmic bytes moved in `time_ms`, against the peak."""
+    gbs = bytes_ / (time_ms / 1e3) / 1e9
+    d = {"gbs": gbs, "frac": gbs / peak, "frac_of_nominal_8tbs": gbs / NOMINAL_HBM_GBS}
+    d.update(extra)
+    return d
+
+
+def substep_profile(g, ctx, torch, stream, w, Hi, es, peak, reps=3):
+    """AdamW launches of the heterogeneous workload one sub-step at a time:
+    sub-step s steps the workers with H_i > s (the same launch as inside a
+    round); each is timed over `reps` launches with CUDA events."""
+    out = []
+    for s in range(max(Hi)):
+        mask = [1 if h > s else 0 for h in Hi]
+        act = sum(mask)
+        if act == 0:
+            continue
+        g.gasloc_set_local_steps(ctx.h, mask)
+        ctx.local_steps(g.PER_WORKER_STEPS)   # warm-up launch
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            ctx.local_steps(g.PER_WORKER_STEPS)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        b = adamw_bytes_of(w, mask, es)[0]
+        out.append(kernel_entry(b, ms, peak, substep=s + 1, active_workers=act, ms=ms, bytes=b))
+    g.gasloc_set_local_steps(ctx.h, Hi)
+    ctx.gossip_round()   # back to a round boundary
+    torch.cuda.synchronize()
+    return out
+
+
+def measure_workload(g, torch, wl, name, K, warmup, peak):
+    """Per-kernel rates of another workload in the same run (its own context,
+    created and released here): AdamW, gossip and the round, CUDA events on the
+    launch stream, plus the same rounds replayed from a CUDA graph."""
+    w = wl.ALL_WORKLOADS[name]
+    es = 2 if w.hp.get("storage") == "bf16" else 4
+    hp = g.make_hparams(**wl.hparams_of(w))
+    ctx = g.Context(w.n_workers, w.n_params, w.topology, w.seed, hparams=hp, numels=w.numels,
+                    draw_hmax=w.draw_hmax)
+    try:
+        H = w.H if w.H > 0 else g.PER_WORKER_STEPS
+        Hi = g.gasloc_get_local_steps(ctx.h, w.n_workers).tolist() if w.H < 0 else None
+        stream = torch.cuda.current_stream()
+        for _ in range(warmup):
+            ctx.local_steps(H)
+            ctx.gossip_round()
+        torch.cuda.synchronize()
+        ms, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H)
+        steps = [H] * w.n_workers if H > 0 else Hi
+        ab = adamw_bytes_of(w, steps, es)
+        gb = 5 * es * w.n_workers * w.n_params
+        graph_ms = measure_graph(ctx, torch, stream, K, H)
+        units = float(w.n_workers) * w.n_params
+        return {
+            "rounds": K, "ms_per_round": ms / K, "value": units * K / (ms / 1e3),
+            "graph_ms_per_round": graph_ms, "graph_value": units / (graph_ms / 1e3),
+            "adamw": kernel_entry(sum(ab), local_ms / K, peak, ms_per_round=local_ms / K,
+                                  bytes_per_round=sum(ab), launches_per_round=len(ab)),
+            "gossip": kernel_entry(gb, gossip_ms / K, peak, ms_per_round=gossip_ms / K, bytes_per_round=gb),
+            "round": kernel_entry(sum(ab) + gb, ms / K, peak, bytes=sum(ab) + gb),
+            "storage": "bf16" if es == 2 else "f32",
+        }
+    finally:
+        ctx.close()
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+
+
+# Other workloads timed in the same run, after the main one (name: rounds
+# timed).  The 105 MB ring is short enough for launch gaps to count, so it
+# takes more rounds.
+EXTRA_WORKLOADS = {"ring_n4_p1m": 200, "exp_n8_gpt2s": 20, "exp_n8_gpt2s_bf16": 20,
+                   "matching_n16_gpt2s_h8": 5, "torus2x4_n8_gpt2m_h4": 5}
+
+
 def main():
     args = parse_args()
     from paper_2606_11081_gb300 import workloads as wl
     w = wl.ALL_WORKLOADS[args.workload or wl.BENCH_WORKLOAD]
+    if args.steps is None:
+        args.steps = w.rounds
     if args.impl == "reference":
         return run_reference(args, w)
 
@@ -293,7 +412,6 @@ def main():
     torch.cuda.synchronize()
 
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
     clocks = ClockSampler(local)
     if pg:
         pg.barrier()
@@ -301,22 +419,9 @@ def main():
     clocks.start()
     time.sleep(0.3)
     l0 = ctx.launches
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
-    for k in range(K):
-        ev[k][0].record(stream)
-        ctx.local_steps(H)
-        ev[k][1].record(stream)
-        ctx.gossip_round()
-        ev[k][2].record(stream)
-    t_end.record(stream)
-    torch.cuda.synchronize()
+    ms, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H)
     clk = clocks.stop()
     launches = ctx.launches - l0
-    ms = t_start.elapsed_time(t_end)
-    local_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(K))
-    gossip_ms = sum(ev[k][1].elapsed_time(ev[k][2]) for k in range(K))
     units = float(w.n_workers) * w.n_params * K
     ms, value = aggregate(ms, units, pg, torch.device("cuda", local) if pg else None)
     if pg:
@@ -325,14 +430,11 @@ def main():
 
     # algorithmic bytes
     N, P = w.n_workers, w.n_params
-    per_h = bool(w.hp.get("per_worker_h"))
     es = 2 if w.hp.get("storage") == "bf16" else 4      # bytes per stored element
     steps = [H] * N if H > 0 else Hi
-    adamw_launches = max(steps)
-    adamw_bytes = 0
-    for s in range(max(steps)):
-        act = sum(1 for h in steps if h > s)
-        adamw_bytes += (8 * es * act if per_h else 7 * es * act + es) * P
+    adamw_per_launch = adamw_bytes_of(w, steps, es)
+    adamw_launches = len(adamw_per_launch)
+    adamw_bytes = sum(adamw_per_launch)
     gossip_bytes = 5 * es * N * P
     peak, peak_kind = peak_hbm()
     adamw_gbs = adamw_bytes / (local_ms / K / 1e3) / 1e9
@@ -340,6 +442,7 @@ def main():
     dom = "adamw" if local_ms >= gossip_ms else "gossip"
     dom_gbs = adamw_gbs if dom == "adamw" else gossip_gbs
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
+    dom_ms_launch = local_ms / K / adamw_launches if dom == "adamw" else gossip_ms / K
     traffic = kernel_traffic(dom, w.name)
 
     # the same rounds replayed from a CUDA graph (gasloc_run)
@@ -352,17 +455,31 @@ def main():
     ce_ms = measure_ce(ctx, torch, stream, 10)
     ce_bytes = es * N * P
     ce_gbs = ce_bytes / (ce_ms / 1e3) / 1e9
+    # AdamW one sub-step at a time (heterogeneous local steps)
+    substeps = substep_profile(g, ctx, torch, stream, w, Hi, es, peak) if Hi is not None else None
 
     e2e = None
+    ctx.close()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
     if not args.no_e2e:
-        ctx.close()
-        torch.cuda.empty_cache()
         e2e = measure_e2e(g, torch, w, hp, H, K)
         # whole job: every rank's units over the slowest rank's time
         _, e2e["value"] = aggregate(e2e["seconds"] * 1e3, float(w.n_workers) * w.n_params * K, pg,
                                     torch.device("cuda", local) if pg else None)
-    else:
-        ctx.close()
+        torch.cuda.empty_cache()
+
+    extras = None
+    names = [] if args.extras == "none" else (
+        list(EXTRA_WORKLOADS) if args.extras == "all" else args.extras.split(","))
+    names = [n for n in names if n != w.name]
+    if names:
+        extras = {}
+        eclk = ClockSampler(local)
+        eclk.start()
+        for name in names:
+            extras[name] = measure_workload(g, torch, wl, name, EXTRA_WORKLOADS.get(name, 10), 3, peak)
+        extras["clocks"] = eclk.stop()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -377,10 +494,14 @@ def main():
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": dom_gbs, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": dom_gbs / peak,
                          "frac_of_nominal_8tbs": dom_gbs / NOMINAL_HBM_GBS,
-                         "traffic": traffic, "algorithmic_bytes_per_launch": dom_bytes_launch},
+                         "traffic": traffic, "algorithmic_bytes_per_launch": dom_bytes_launch,
+                         "ms_per_launch": dom_ms_launch,
+                         "note": "algorithmic bytes of the kernel's launches over their summed "
+                                 "CUDA-event time (AdamW: one launch per local sub-step)"},
             "kernels": {"adamw": {"gbs": adamw_gbs, "frac": adamw_gbs / peak,
                                   "frac_of_nominal_8tbs": adamw_gbs / NOMINAL_HBM_GBS, "ms_per_round": local_ms / K,
-                                  "bytes_per_round": adamw_bytes, "launches_per_round": adamw_launches},
+                                  "bytes_per_round": adamw_bytes, "launches_per_round": adamw_launches,
+                                  "substeps": substeps},
                         "gossip": {"gbs": gossip_gbs, "frac": gossip_gbs / peak,
                                    "frac_of_nominal_8tbs": gossip_gbs / NOMINAL_HBM_GBS,
                                    "ms_per_round": gossip_ms / K, "bytes_per_round": gossip_bytes},
@@ -405,6 +526,12 @@ def main():
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clk,
             "consensus_error": ce,
         }
+        if extras is not None:
+            line["workloads"] = extras
+            if "exp_n8_gpt2s_bf16" in extras:
+                xb = extras["exp_n8_gpt2s_bf16"]
+                line["kernels_bf16"] = {"workload": "exp_n8_gpt2s_bf16", "adamw": xb["adamw"],
+                                        "gossip": xb["gossip"], "round": xb["round"]}
         print(json.dumps(line), flush=True)
     if pg:
         pg.barrier()

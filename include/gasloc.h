@@ -234,21 +234,30 @@ int gasloc_synchronize(gasloc_ctx *ctx);
  * a latency-critical loop where cudaMalloc/cudaFree would synchronise the
  * device, or a plug-in that is handed pre-allocated buffers only.  The paper
  * has no counterpart; this is a service of the library.
- *   x: device pointer, n_workers rows of worker_stride floats each (row i is
- *      replica i; the caller owns all n_workers * worker_stride floats),
- *      16-byte aligned, worker_stride a multiple of 4 and >= n_params.
+ *   x: device pointer to fp32 values, n_workers rows of worker_stride floats
+ *      each (row i is replica i; the caller owns all n_workers * worker_stride
+ *      floats), 16-byte aligned, worker_stride a multiple of 4 and >=
+ *      n_params.  The values must be fp32: the pointer gasloc_buffer returns
+ *      for a context with a bf16 store is not valid input (its elements would
+ *      be read as floats and the value would be wrong, with no error).
  *   ce_out_device: device pointer to one double that receives
  *      (1/n) sum_i ||x_i - xbar||^2 (same arithmetic as gasloc_consensus_error).
  *   cuda_stream: the stream the work is enqueued on (asynchronous).
  * Nothing is allocated: the reduction's scratch is a fixed 512 KiB + 256 B
  * array compiled into the library, held by every GPU that loads it until the
  * process exits.  n_params above 536,870,912 is rejected (GASLOC_ENOMEM).
- * The first call on a device looks up that array's device address (and the
- * launch shape) for the current device; make that first call before any
- * stream capture.  Every call reuses the same array (its completion counter is
- * cleared at the start of each call): calls whose work overlaps on the GPU
- * race, so serialise them (one stream, or events).  Errors: EINVAL (null or
- * misaligned pointers, bad sizes), ENOMEM (size limit), ECUDA. */
+ * The array's device address belongs to the CUDA context: the first call in
+ * each context (the device's primary context, or a driver context the caller
+ * created and made current) looks it up, with the launch shape, in the
+ * context current on the calling thread and caches it under that context's
+ * process-unique id; make that first call before any stream capture.  A
+ * context that replaces another (after cudaDeviceReset or a primary-context
+ * reset) has a new id, so the address is looked up again.  Every call reuses
+ * the same array (its completion counter is cleared at the start of each
+ * call): calls whose work overlaps on the GPU race, so serialise them (one
+ * stream, or events).  In the index-checked build a failed check makes the
+ * result NaN.  Errors: EINVAL (null or misaligned pointers, bad sizes), ENOMEM
+ * (size limit), ECUDA. */
 int gasloc_consensus_error_noalloc(const float *x, int32_t n_workers, int64_t n_params,
                                    int64_t worker_stride, double *ce_out_device, void *cuda_stream);
 

@@ -16,12 +16,21 @@
 // column, e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with s = x_0k,
 // fp64 across elements.  Partials are written per chunk and added in chunk
 // order by the last CTA to finish, so the result does not depend on the grid.
+//
+// The array's device address belongs to a CUDA context, not to a device: the
+// device's primary context gets a new one after cudaDeviceReset, and a caller
+// that runs its own driver context on the device has another.  The address is
+// therefore looked up in the context current on the calling thread and cached
+// under that context's process-unique id (cuCtxGetId), so a replaced or
+// different context is looked up afresh.
+#include <cuda.h>   // driver types only; the entry points are fetched through the runtime
 #include <cuda_runtime.h>
 
 #include <cstdint>
 #include <mutex>
 
 #include "../../include/gasloc.h"
+#include "check.cuh"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -31,10 +40,11 @@ constexpr int kBlock = 256;
 constexpr int64_t kChunk = 8192;                       // elements per partial
 constexpr int64_t kMaxChunks = 65536;                  // partials in the scratch
 constexpr int64_t kMaxParams = kChunk * kMaxChunks;    // 536,870,912 elements
-constexpr int kHeaderDoubles = 32;                     // ticket lives in the first 256 bytes
-constexpr int kMaxDevices = 64;
+constexpr int kHeaderDoubles = 32;                     // ticket and error word in the first 256 bytes
+constexpr int kMaxContexts = 64;                       // contexts whose address is cached
 
-// 256 bytes of header (completion ticket) + 512 KiB of per-chunk partials.
+// 256 bytes of header (completion ticket at byte 0, the checked build's error
+// word at byte 8) + 512 KiB of per-chunk partials.
 static __device__ __align__(256) double g_ce_scratch[kHeaderDoubles + kMaxChunks];
 
 __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restrict__ x, int32_t n,
@@ -43,6 +53,7 @@ __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restr
     __shared__ double red[kBlock / 32];
     __shared__ int last;
     unsigned int *ticket = reinterpret_cast<unsigned int *>(scratch);
+    int32_t *err = reinterpret_cast<int32_t *>(scratch + 1);   // checked build: a failed index check
     double *partials = scratch + kHeaderDoubles;
     const float inv_n = static_cast<float>(1.0 / n);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -59,8 +70,11 @@ __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restr
             for (int i0 = 0; i0 < n; i0 += U) {
                 float4 X[U];
 #pragma unroll
-                for (int u = 0; u < U; ++u)
-                    if (i0 + u < n) X[u] = gasloc::ptx::ld_stream(x + (i0 + u) * wstride + off);
+                for (int u = 0; u < U; ++u) {
+                    X[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (i0 + u < n && gasloc::row_ok(i0 + u, n, off, 4, wstride, err))
+                        X[u] = gasloc::ptx::ld_stream(x + (i0 + u) * wstride + off);
+                }
 #pragma unroll
                 for (int u = 0; u < U; ++u) {
                     if (i0 + u >= n) continue;
@@ -86,7 +100,7 @@ __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restr
         if (threadIdx.x == 0) {
             double s = 0.0;
             for (int w = 0; w < kBlock / 32; ++w) s += red[w];
-            partials[ch] = s;
+            if (gasloc::span_ok(ch, ch + 1, kMaxChunks, err)) partials[ch] = s;
         }
         __syncthreads();
     }
@@ -103,24 +117,67 @@ __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restr
         for (int64_t b = lane; b < nchunks; b += 32) s += __ldcg(partials + b);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_down_sync(0xffffffffu, s, o);
         if (lane == 0) {
-            *out = s / static_cast<double>(n);
+            // a failed index check (checked build only) makes the result NaN
+            *out = __ldcg(err) != 0 ? __longlong_as_double(0x7ff8000000000000ll) : s / static_cast<double>(n);
             *ticket = 0u;
         }
     }
 }
 
-struct DeviceSetup {
+// Address of the scratch array in one CUDA context, and the launch shape.
+struct ContextSetup {
+    unsigned long long ctx_id = 0;
     void *scratch = nullptr;
     int grid = 0;
-    bool ready = false;
 };
 
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long *);
+
 std::mutex g_mu;
-DeviceSetup g_setup[kMaxDevices];
+ContextSetup g_setup[kMaxContexts];
+int g_nsetup = 0, g_next = 0;
+CtxGetCurrentFn g_get_current = nullptr;
+CtxGetIdFn g_get_id = nullptr;
 
 int fail(int code, const char *msg) {
     gasloc::set_last_error(msg);   // reported by gasloc_last_error()
     return code;
+}
+
+void *driver_entry(const char *name) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion(name, &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    return p;
+}
+
+// Process-unique id of the context current on this thread (binding the
+// device's primary context first if none is current yet).  0 on failure.
+unsigned long long current_context_id() {
+    if (!g_get_current || !g_get_id) {
+        g_get_current = reinterpret_cast<CtxGetCurrentFn>(driver_entry("cuCtxGetCurrent"));
+        g_get_id = reinterpret_cast<CtxGetIdFn>(driver_entry("cuCtxGetId"));
+        if (!g_get_current || !g_get_id) return 0;
+    }
+    CUcontext ctx = nullptr;
+    if (g_get_current(&ctx) != CUDA_SUCCESS) return 0;
+    if (!ctx) {
+        // the runtime binds the primary context on its first call that needs one
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_ce_scratch) != cudaSuccess) {
+            cudaGetLastError();
+            return 0;
+        }
+        if (g_get_current(&ctx) != CUDA_SUCCESS || !ctx) return 0;
+    }
+    unsigned long long id = 0;
+    if (g_get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
 }
 
 }  // namespace
@@ -141,40 +198,42 @@ int gasloc_consensus_error_noalloc(const float *x, int32_t n_workers, int64_t n_
     if (reinterpret_cast<uintptr_t>(ce_out_device) % 8 != 0)
         return fail(GASLOC_EINVAL, "ce_out_device must be 8-byte aligned");
 
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
-        cudaGetLastError();
-        return fail(GASLOC_ECUDA, "no usable current CUDA device");
-    }
-    DeviceSetup setup;
+    ContextSetup setup;
     {
-        // once per device, with that device current: resolve the scratch
-        // array's device address (the host-side name is not a device address)
         std::lock_guard<std::mutex> lock(g_mu);
-        DeviceSetup &s = g_setup[dev];
-        if (!s.ready) {
+        const unsigned long long id = current_context_id();
+        if (id == 0) return fail(GASLOC_ECUDA, "no usable CUDA context on this thread");
+        int hit = -1;
+        for (int q = 0; q < g_nsetup; ++q)
+            if (g_setup[q].ctx_id == id) hit = q;
+        if (hit < 0) {
+            // first call in this context, which is current: resolve the scratch
+            // array's device address here (the host-side name is not one)
             void *p = nullptr;
             if (cudaGetSymbolAddress(&p, g_ce_scratch) != cudaSuccess || !p) {
                 cudaGetLastError();
                 return fail(GASLOC_ECUDA, "cudaGetSymbolAddress of the scratch array failed");
             }
-            int sms = 0, per_sm = 0;
-            if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            int dev = 0, sms = 0, per_sm = 0;
+            if (cudaGetDevice(&dev) != cudaSuccess ||
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
                 cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ce_noalloc_kernel, kBlock, 0) != cudaSuccess) {
                 cudaGetLastError();
                 return fail(GASLOC_ECUDA, "querying the device for the launch shape failed");
             }
-            s.scratch = p;
-            s.grid = sms * (per_sm > 0 ? per_sm : 1);
-            s.ready = true;
+            hit = g_nsetup < kMaxContexts ? g_nsetup++ : (g_next++ % kMaxContexts);
+            g_setup[hit].ctx_id = id;
+            g_setup[hit].scratch = p;
+            g_setup[hit].grid = sms * (per_sm > 0 ? per_sm : 1);
         }
-        setup = s;
+        setup = g_setup[hit];
     }
     const cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
     const int64_t nchunks = (n_params + kChunk - 1) / kChunk;
     const int grid = static_cast<int>(nchunks < setup.grid ? nchunks : setup.grid);
-    // the array keeps the previous call's contents: the ticket must start at 0
-    cudaError_t e = cudaMemsetAsync(setup.scratch, 0, sizeof(unsigned int), stream);
+    // the array keeps the previous call's contents: the ticket and the error
+    // word (bytes 0..15) must start at 0
+    cudaError_t e = cudaMemsetAsync(setup.scratch, 0, 2 * sizeof(double), stream);
     if (e != cudaSuccess) {
         cudaGetLastError();
         return fail(GASLOC_ECUDA, "clearing the completion ticket failed");

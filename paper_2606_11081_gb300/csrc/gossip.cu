@@ -211,14 +211,15 @@ __device__ __forceinline__ void consumer_barrier() {
 }
 
 // DENSE (bf16, one thread per column, n <= 8, not Eq. 2): the thread widens the n
-// mixed rows of its column once and forms each worker's mix over all j < n
-// in ascending order with a dense weight row (zero off the neighbourhood),
-// built from the round's table in the prologue.  For finite rows a
-// zero-weight term adds an exact zero, so the sums are those of the neighbour
-// lists; a non-finite row (a diverged replica) reaches every worker of its
-// column as NaN (0 * inf) where the lists would confine it to its neighbours.
+// mixed rows of its column once and forms each worker's mix over the j < n
+// of its neighbourhood in ascending order, with a dense weight row and a
+// neighbour bitmask built from the round's table in the prologue.  The terms
+// and their order are those of the neighbour lists, so the sums are the same
+// bit for bit, and a non-finite row (a diverged replica) reaches only the
+// workers that mix it.
 constexpr int kDenseMax = 8;
-constexpr int kDenseRow = 8;   // dense row i lives in tp->w[kDenseRow + i] (rows >= n are free)
+constexpr int kDenseRow = 8;   // dense row i lives in tp->w[kDenseRow + i] and its neighbour mask in
+                               // tp->nbr[kDenseRow + i][0] (rows >= n are free)
 
 template <int MODE, typename T, bool DENSE>
 __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kernel(const GossipArgs a) {
@@ -256,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             dst[at] = src[at];
         }
     }
-    if constexpr (DENSE) {   // dense weights of the round, from the table in global memory
+    if constexpr (DENSE) {   // dense weights and neighbour masks of the round, from the table in global memory
         const int t = threadIdx.x;
         if (t < kDenseMax * kDenseMax) {
             const int i = t / kDenseMax, j = t % kDenseMax;
@@ -266,6 +267,17 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                 for (int q = 0; q <= dg && q < kMaxWorkers; ++q)
                     if (a.topo->nbr[i][q] == j) wij = a.topo->w[i][q];
                 tp->w[kDenseRow + i][j] = wij;
+            }
+        } else if (t < kDenseMax * kDenseMax + kDenseMax) {
+            const int i = t - kDenseMax * kDenseMax;
+            if (i < n) {
+                uint32_t mask = 0;
+                const int dg = a.topo->deg[i];
+                for (int q = 0; q <= dg && q < kMaxWorkers; ++q) {
+                    const int j = a.topo->nbr[i][q];
+                    if (span_ok(j, j + 1, kDenseMax, a.err)) mask |= 1u << j;
+                }
+                tp->nbr[kDenseRow + i][0] = static_cast<int32_t>(mask);
             }
         }
     }
@@ -454,9 +466,10 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
                     float2 acc01 = x2::splat(0.f), acc23 = acc01;
                     if constexpr (DENSE) {
                         const float *wr = &tp->w[kDenseRow + i][0];
+                        const uint32_t nm = static_cast<uint32_t>(tp->nbr[kDenseRow + i][0]);
 #pragma unroll
                         for (int j = 0; j < kDenseMax; ++j) {
-                            if (j < n) {
+                            if (j < n && ((nm >> j) & 1u)) {
                                 const float2 w = x2::splat(wr[j]);
                                 acc01 = x2::fma(w, x2::lo(sall[j]), acc01);
                                 acc23 = x2::fma(w, x2::hi(sall[j]), acc23);

@@ -132,7 +132,9 @@ ALL_WORKLOADS = dict(WORKLOADS, **PROFILE_WORKLOADS, **BF16_WORKLOADS)
 COMMON_HP = dict(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-8, weight_decay=0.1,
                  outer="nesterov", outer_lr=0.7, outer_momentum=0.9)
 
-BENCH_WORKLOAD = "exp_n8_gpt2s"
+# The workload bench.py measures by default: the largest one that fits one GPU
+# (112 GB of replica state, about 650 GB moved per round).
+BENCH_WORKLOAD = "hetero_exp_n32_gpt2s"
 
 
 def hparams_of(w: Workload) -> Dict[str, object]:

@@ -28,7 +28,7 @@ def test_reference_arm_line():
         assert k in d, k
     assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
-    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["config"]["workload"] == "exp_n8_gpt2s"
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["config"]["workload"] == "hetero_exp_n32_gpt2s"
 
 
 @pytest.mark.gpu
@@ -36,14 +36,25 @@ def test_main_arm_line():
     import torch
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
-    d = _run(["--workload", "exp_n8_p16m", "--steps", "5", "--warmup", "3", "--cpu-seconds", "1"], 900)
+    d = _run(["--workload", "exp_n32_p4m_hetero", "--steps", "5", "--warmup", "3", "--cpu-seconds", "1",
+              "--extras", "ring_n4_p1m,exp_n8_p16m_bf16"], 900)
     for k in BASE + ["roofline", "e2e", "cpu_baseline", "gpu_launches", "clocks"]:
         assert k in d, k
     rf = d["roofline"]
     for k in ("bound", "achieved", "peak", "unit", "frac", "traffic"):
         assert k in rf, k
     assert rf["bound"] == "hbm" and 0 < rf["frac"] < 1.2
-    assert d["gpu_launches"] == 5 * 2        # AdamW + gossip per round
+    # per round: one AdamW launch per local sub-step (H_i up to 8), the
+    # round's random neighbour table, and gossip
+    subs = d["kernels"]["adamw"]["substeps"]
+    assert d["gpu_launches"] == 5 * (len(subs) + 2)
+    assert [s["substep"] for s in subs] == list(range(1, len(subs) + 1))
+    assert all(0 < s["frac"] < 1.3 for s in subs)
+    assert d["config"]["workload"] == "exp_n32_p4m_hetero"
+    for name in ("ring_n4_p1m", "exp_n8_p16m_bf16"):
+        x = d["workloads"][name]
+        assert x["adamw"]["gbs"] > 0 and x["gossip"]["gbs"] > 0 and x["value"] > 0
+
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     assert d["cpu_baseline"]["cores"] >= 1

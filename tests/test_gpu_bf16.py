@@ -150,3 +150,46 @@ def test_bf16_host_transfer_over_staging_chunks():
         for i in range(2):
             got = ctx.read("c", i)
             np.testing.assert_array_equal(got.view(np.uint32), ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("storage", ["f32", "bf16"])
+@pytest.mark.parametrize("N,topo,kw", [(8, "ring", {}), (8, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
+                                       (6, "2peer", {"weights": "lazy"})])
+def test_nonfinite_replica_reaches_neighbours_only(storage, N, topo, kw):
+    # A diverged replica (inf in some elements of worker j) is mixed only by
+    # the workers whose neighbourhood holds j, as in the oracle's neighbour
+    # lists; the dense bf16 mixing at n <= 8 must not carry it elsewhere.
+    P = 2 * 1024 + 5
+    hp = dict(kw, storage=storage, outer="nesterov")
+    ctx, st = make_pair(N, P, topo, seed=900 + N, hp=hp)
+    with ctx:
+        j = 3
+        bad = ctx.read("x", j)
+        cols = np.array([0, 1, 700, 1031, P - 1])
+        bad[cols[:3]] = np.inf
+        bad[cols[3:]] = -np.inf
+        ctx.write("x", j, bad)
+        st.set("x", j, bad.astype(np.float64))
+        # round 0: no local step, every worker sends x
+        nbr, w, deg = ctx.topology(0)
+        ctx.gossip_round()
+        st.gossip_round()
+        x = ctx.read_all("x")
+        np.testing.assert_array_equal(x, st.get_all("x").astype(np.float32))
+        np.testing.assert_array_equal(ctx.read_all("b"), st.get_all("b").astype(np.float32))
+        mixes_j = [i for i in range(N) if j in nbr[i, :deg[i] + 1]]
+        assert j in mixes_j
+        for i in range(N):
+            if i in mixes_j:
+                assert not np.isfinite(x[i, cols]).any(), i
+            else:
+                assert np.isfinite(x[i]).all(), i
+        # then ordinary rounds: the non-finite values spread along the graph
+        # exactly as in the oracle
+        for _ in range(2):
+            ctx.local_steps(1)
+            st.local_steps(1)
+            ctx.gossip_round()
+            st.gossip_round()
+        np.testing.assert_array_equal(ctx.read_all("x"), st.get_all("x").astype(np.float32))
+        np.testing.assert_array_equal(ctx.read_all("b"), st.get_all("b").astype(np.float32))

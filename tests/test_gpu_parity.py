@@ -190,6 +190,45 @@ def test_consensus_error_closed_form_and_paths():
         assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-6)
 
 
+@pytest.mark.parametrize("N", [8, 32])
+def test_consensus_error_near_consensus_far_from_zero(N):
+    # Replicas a thousand times further from zero than from each other:
+    # x_ik = a_k + 1e-3 (i - (N-1)/2) with a_k in [1000, 2000).  A one-pass
+    # fp32 form without a shift would lose every digit here; the shifted form
+    # subtracts worker 0's value exactly (the values are within a factor of 2
+    # of each other), so only the sums round.  Compared with the exact
+    # consensus error of the stored fp32 values (fp64, two passes), with the
+    # oracle, and with the closed form P 1e-6 (N^2 - 1) / 12 of the unrounded
+    # values (the fp32 rounding of the values moves it by about 1%).
+    P = 3 * 4096 + 77
+    hp = dict(outer="sgd", outer_lr=0.0)        # the gossip round leaves x as it is
+    ctx, st = make_pair(N, P, "exp", seed=21, hp=hp)
+    rng = np.random.default_rng(N)
+    a = 1000.0 + 1000.0 * rng.random(P)
+    x = np.stack([(a + 1e-3 * (i - (N - 1) / 2)).astype(np.float32) for i in range(N)])
+    xd = x.astype(np.float64)
+    exact = ((xd - xd.mean(0)) ** 2).sum() / N
+    # the shifted form's bound for these values: relative (3N + 2) u kappa + u,
+    # kappa = sum_i (x_i - x_0)^2 / sum_i (x_i - xbar)^2 (worker 0's shift)
+    kappa = ((xd - xd[0]) ** 2).sum() / (((xd - xd.mean(0)) ** 2).sum())
+    u = 2.0 ** -24
+    tol = (3 * N + 2) * u * kappa + u
+    with ctx:
+        for i in range(N):
+            ctx.write("x", i, x[i])
+            st.set("x", i, xd[i])
+        now = ctx.consensus_error_now()                 # standalone reduction
+        ctx.gossip_round()                              # fused reduction of the unchanged x
+        np.testing.assert_array_equal(ctx.read_all("x"), x)
+        fused = ctx.consensus_error()
+        st.gossip_round()
+        ref = st.consensus_error()
+        assert ref == pytest.approx(exact, rel=1e-12)
+        assert ref == pytest.approx(P * 1e-6 * (N * N - 1) / 12, rel=0.05)
+        for got in (now, fused):
+            assert got == pytest.approx(exact, rel=tol), (got, exact, tol)
+
+
 @pytest.mark.parametrize("storage", ["f32", "bf16"])
 @pytest.mark.parametrize("numels", [None, [1000, 3, 4097, 64, 1, 2048, 5]])
 def test_average_is_the_fp32_mean_of_the_replicas(storage, numels):
