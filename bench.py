@@ -7,8 +7,11 @@ round's neighbour table where it is random (K_topo), and the gossip round with
 the outer optimizer and the fused consensus-error reduction (K_gossip).
 
 Prints ONE JSON line (rank 0).  `value` is replica-element updates per second
-over the timed rounds (n_workers * n_params * rounds / time, summed over ranks
-that each run their own replica set: multi-GPU runs are independent replicas).
+over the timed rounds (n_workers * n_params * rounds / time).  On several GPUs
+(torchrun) every replica is split by parameter range, one contiguous range per
+GPU (the steps are element-wise in the parameter index), and the one exchange
+per round is an all-reduce of the ranks' consensus-error shares; the job's
+time is the slowest rank's and `value` counts every rank's elements.
 `e2e` repeats the measurement through the public C ABI from host buffers:
 upload of the initial replicas, centres and curvature from pinned host memory,
 every round's consensus error read back to the host, and the network average
@@ -147,9 +150,10 @@ class ClockSampler:
 
 
 def aggregate(ms_local: float, units_local: float, dist_mod=None, device=None):
-    """Whole-job timing for independent replicas (one per GPU): the job's time
-    is the slowest rank's timed region and its throughput is the units all
-    ranks processed over that time.  Returns (ms_max, units_per_second)."""
+    """Whole-job timing over the ranks (one GPU each, each holding a range of
+    the parameters): the job's time is the slowest rank's timed region and its
+    throughput is the units all ranks processed over that time.  Returns
+    (ms_max, units_per_second)."""
     if dist_mod is None:
         return ms_local, units_local / (ms_local / 1e3)
     import torch
@@ -159,6 +163,18 @@ def aggregate(ms_local: float, units_local: float, dist_mod=None, device=None):
     dist_mod.all_reduce(t_sum, op=dist_mod.ReduceOp.SUM)
     ms = float(t_max.item())
     return ms, float(t_sum.item()) / (ms / 1e3)
+
+
+def shard_range(P: int, world: int, rank: int, align: int = 4096):
+    """The part [p0, p1) of the P parameters that `rank` holds when every
+    replica is split over `world` GPUs: contiguous, in multiples of `align`
+    elements (the last part takes the rest)."""
+    units = -(-P // align)                       # blocks of `align` elements, the last one ragged
+    p0 = min(rank * units // world * align, P)
+    p1 = min((rank + 1) * units // world * align, P)
+    if p1 <= p0:
+        raise ValueError("%d parameters do not split over %d ranks in parts of %d" % (P, world, align))
+    return p0, p1
 
 
 def dist_env():
@@ -248,14 +264,25 @@ def run_reference(args, w):
     return 0
 
 
-def workload_config(w, args):
-    state_gb = w.n_workers * w.n_params * 4 * (6 + (1 if w.hp.get("per_worker_h") else 0)) / 1e9
+def ce_exchange(dist_mod, ctx, ce_dev, k):
+    """The one exchange of a round when the replicas are split over GPUs by
+    parameter range: this GPU's consensus-error share is copied to device
+    memory on the round's stream and summed over the ranks (all-reduce)."""
+    ctx.consensus_error_async(ce_dev.data_ptr() + 8 * k)
+    dist_mod.all_reduce(ce_dev[k:k + 1], op=dist_mod.ReduceOp.SUM)
+
+
+def workload_config(w, args, world=1):
+    state_gb = w.n_workers * w.n_params * 4 * (6 + (1 if w.hp.get("per_worker_h") else 0)) / 1e9 / world
     return {"workload": w.name, "n_workers": w.n_workers, "n_params": w.n_params,
             "topology": w.topology, "H": w.H if w.H > 0 else "H_i~U{1..%d}" % w.draw_hmax,
             "layout": "tensor-list(%d)" % len(w.numels) if w.numels else "flat",
             "storage": w.hp.get("storage", "f32"),
             "weights": w.hp.get("weights", "uniform"), "outer": "nesterov(0.7, 0.9)",
-            "seed": w.seed, "parallelism": "replicas x%d" % args.gpus,
+            "seed": w.seed,
+            "parallelism": ("parameter ranges x%d (each GPU holds a contiguous range of every replica; "
+                            "one fp64 all-reduce of the consensus-error shares per round)" % world
+                            if world > 1 else "one GPU"),
             "l2": "inputs larger than L2 (%.1f GB replica state per GPU, no flush)" % state_gb}
 
 
@@ -271,9 +298,10 @@ def adamw_bytes_of(w, steps, es):
     return out
 
 
-def time_rounds(ctx, torch, stream, K, H):
+def time_rounds(ctx, torch, stream, K, H, after_round=None):
     """K rounds with CUDA events around the local steps and the gossip round of
-    each; returns (total ms, local-step ms, gossip ms) summed over the rounds."""
+    each; returns (total ms, local-step ms, gossip ms) summed over the rounds.
+    after_round(k) runs after round k's gossip (the ranks' exchange)."""
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
@@ -284,6 +312,8 @@ def time_rounds(ctx, torch, stream, K, H):
         ev[k][1].record(stream)
         ctx.gossip_round()
         ev[k][2].record(stream)
+        if after_round is not None:
+            after_round(k)
     t_end.record(stream)
     torch.cuda.synchronize()
     ms = t_start.elapsed_time(t_end)
@@ -400,18 +430,26 @@ def main():
         pg.barrier()
 
     hp = g.make_hparams(**wl.hparams_of(w))
+    # more than one GPU: each holds a contiguous range of every replica's
+    # parameters (every step is element-wise in the parameter index); the one
+    # exchange per round is the sum of the ranks' consensus-error shares
+    p_range = shard_range(w.n_params, world, rank) if world > 1 else None
     ctx = g.Context(w.n_workers, w.n_params, w.topology, w.seed, hparams=hp, numels=w.numels,
-                    draw_hmax=w.draw_hmax)
+                    draw_hmax=w.draw_hmax, p_range=p_range)
     H = w.H if w.H > 0 else g.PER_WORKER_STEPS
     Hi = g.gasloc_get_local_steps(ctx.h, w.n_workers).tolist() if w.H < 0 else None
     stream = torch.cuda.current_stream()
+    K = args.steps
+    ce_dev = torch.zeros(max(K, args.warmup, 1), dtype=torch.float64, device="cuda")
+    exchange = (lambda k: ce_exchange(pg, ctx, ce_dev, k)) if pg else None
 
-    for _ in range(args.warmup):
+    for k in range(args.warmup):
         ctx.local_steps(H)
         ctx.gossip_round()
+        if exchange:
+            exchange(k)
     torch.cuda.synchronize()
 
-    K = args.steps
     clocks = ClockSampler(local)
     if pg:
         pg.barrier()
@@ -419,17 +457,19 @@ def main():
     clocks.start()
     time.sleep(0.3)
     l0 = ctx.launches
-    ms, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H)
+    ms, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H, exchange)
     clk = clocks.stop()
     launches = ctx.launches - l0
-    units = float(w.n_workers) * w.n_params * K
+    N, P = w.n_workers, ctx.P        # P: the parameters this GPU holds
+    units = float(N) * P * K
     ms, value = aggregate(ms, units, pg, torch.device("cuda", local) if pg else None)
     if pg:
         pg.barrier()
-    ce = ctx.consensus_error()
+        ce = float(ce_dev[K - 1].item())        # the all-reduced sum of the shares
+    else:
+        ce = ctx.consensus_error()
 
-    # algorithmic bytes
-    N, P = w.n_workers, w.n_params
+    # algorithmic bytes (of this GPU's range)
     es = 2 if w.hp.get("storage") == "bf16" else 4      # bytes per stored element
     steps = [H] * N if H > 0 else Hi
     adamw_per_launch = adamw_bytes_of(w, steps, es)
@@ -463,14 +503,14 @@ def main():
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     if not args.no_e2e:
-        e2e = measure_e2e(g, torch, w, hp, H, K)
+        e2e = measure_e2e(g, torch, w, hp, H, K, p_range, pg)
         # whole job: every rank's units over the slowest rank's time
-        _, e2e["value"] = aggregate(e2e["seconds"] * 1e3, float(w.n_workers) * w.n_params * K, pg,
+        _, e2e["value"] = aggregate(e2e["seconds"] * 1e3, float(N) * P * K, pg,
                                     torch.device("cuda", local) if pg else None)
         torch.cuda.empty_cache()
 
     extras = None
-    names = [] if args.extras == "none" else (
+    names = [] if (args.extras == "none" or world > 1) else (
         list(EXTRA_WORKLOADS) if args.extras == "all" else args.extras.split(","))
     names = [n for n in names if n != w.name]
     if names:
@@ -489,8 +529,8 @@ def main():
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
             "warmup": args.warmup, "ms_per_step": ms / K, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if es == 2 else "f32",
-            "data": "synthetic", "config": workload_config(w, args),
+            "scaling": "strong", "vs_baseline": None, "dtype": "bf16" if es == 2 else "f32",
+            "data": "synthetic", "config": workload_config(w, args, world),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": dom_gbs, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": dom_gbs / peak,
                          "frac_of_nominal_8tbs": dom_gbs / NOMINAL_HBM_GBS,
@@ -588,13 +628,17 @@ def measure_ce(ctx, torch, stream, reps):
     return e0.elapsed_time(e1) / reps
 
 
-def measure_e2e(g, torch, w, hp, H, K):
+def measure_e2e(g, torch, w, hp, H, K, p_range=None, dist_mod=None):
     """Same rounds through the public C ABI from host buffers: upload the
     initial replicas (x_0 broadcast), centres and curvature from pinned memory,
-    read the consensus error back every round, read the average back at the end."""
+    read the consensus error back every round, read the average back at the
+    end.  Split over GPUs, each rank does so for its parameter range, and each
+    round's value read back is the all-reduced sum of the ranks' shares."""
     import numpy as np
-    N, P = w.n_workers, w.n_params
-    ctx = g.Context(N, P, w.topology, w.seed, hparams=hp, numels=w.numels, draw_hmax=w.draw_hmax)
+    N = w.n_workers
+    ctx = g.Context(N, w.n_params, w.topology, w.seed, hparams=hp, numels=w.numels, draw_hmax=w.draw_hmax,
+                    p_range=p_range)
+    P = ctx.P
     per_h = bool(w.hp.get("per_worker_h"))
     nh = N if per_h else 1
     # host inputs (taken from the device initialisation, untimed)
@@ -607,10 +651,14 @@ def measure_e2e(g, torch, w, hp, H, K):
     for i in range(nh):
         g.gasloc_read(ctx.h, "h", i, hs[i].numpy())
     out = torch.empty(P, dtype=torch.float32, pin_memory=True)
+    ces = torch.zeros(K, dtype=torch.float64, pin_memory=True)
+    ce_dev = torch.zeros(K, dtype=torch.float64, device="cuda") if dist_mod else None
     # untimed warm-up of the host-to-device path (one worker's centre row);
     # the timed region below uploads everything again
     g.gasloc_write_ptr(ctx.h, "c", 0, cs[0].data_ptr())
     torch.cuda.synchronize()
+    if dist_mod:
+        dist_mod.barrier()
     t0 = time.perf_counter()
     g.gasloc_write_ptr(ctx.h, "x", -1, x0.data_ptr())
     for i in range(N):
@@ -620,13 +668,17 @@ def measure_e2e(g, torch, w, hp, H, K):
     t1 = time.perf_counter()
     # every round's consensus error is copied to pinned host memory as the
     # round completes; the host waits once, after the last round
-    ces = torch.zeros(K, dtype=torch.float64, pin_memory=True)
     base = ces.data_ptr()
     for k in range(K):
         ctx.local_steps(H)
         ctx.gossip_round()
-        ctx.consensus_error_async(base + 8 * k)
+        if dist_mod:
+            ce_exchange(dist_mod, ctx, ce_dev, k)
+            ces[k:k + 1].copy_(ce_dev[k:k + 1], non_blocking=True)
+        else:
+            ctx.consensus_error_async(base + 8 * k)
     ctx.synchronize()
+    torch.cuda.synchronize()
     t2 = time.perf_counter()
     g.gasloc_average_host(ctx.h, out.numpy())
     el = time.perf_counter() - t0
@@ -635,10 +687,14 @@ def measure_e2e(g, torch, w, hp, H, K):
         raise RuntimeError("a round's consensus error did not arrive on the host")
     # the same rounds with a blocking read after each one, for comparison
     tb = time.perf_counter()
-    for _ in range(K):
+    for k in range(K):
         ctx.local_steps(H)
         ctx.gossip_round()
-        ctx.consensus_error()
+        if dist_mod:
+            ce_exchange(dist_mod, ctx, ce_dev, k)
+            float(ce_dev[k].item())
+        else:
+            ctx.consensus_error()
     tb = time.perf_counter() - tb
     ctx.close()
     h2d = (P + N * P + nh * P) * 4

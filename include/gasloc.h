@@ -160,6 +160,28 @@ int gasloc_get_hparams(const gasloc_ctx *ctx, gasloc_hparams *hp);
  * parameter index used by every generator.  Before gasloc_start only. */
 int gasloc_set_layout(gasloc_ctx *ctx, int32_t n_tensors, const int64_t *numels);
 
+/* Restricts the context to the parameters [p_begin, p_end) of every replica
+ * (0 <= p_begin < p_end <= n_params), before gasloc_start.  Every step of
+ * Algorithm 1 acts on each parameter index separately -- the gradient of the
+ * synthetic quadratic is diagonal and the gossip mixes the workers' values at
+ * one index -- so contexts holding disjoint ranges of the same problem (same
+ * n_workers, n_params, topology, seed, hyperparameters and layout) evolve
+ * exactly as the corresponding parts of one context holding all of it: every
+ * generator is keyed on the global index, and every context builds the same
+ * neighbour tables and H_i.  This is how the replicas are split over several
+ * GPUs (one range per GPU), with no data exchanged between them.  After the
+ * call the context holds n = p_end - p_begin parameters per replica: the
+ * host arrays of gasloc_read / gasloc_write / gasloc_gather /
+ * gasloc_average[_host] and the indices of gasloc_gather count from p_begin,
+ * gasloc_buffer exposes the context's pieces of the tensors (a tensor list is
+ * cut at the range's ends), and gasloc_consensus_error returns the range's
+ * share (1/n_workers) sum_{k in range} sum_i (x_ik - xbar_k)^2, so that the
+ * shares of a partition of [0, n_params) add up to the whole consensus error.
+ * EINVAL for an empty or out-of-bounds range, ESTATE after gasloc_start. */
+int gasloc_set_range(gasloc_ctx *ctx, int64_t p_begin, int64_t p_end);
+/* The context's range and the problem's n_params (default: [0, n_params)). */
+int gasloc_get_range(const gasloc_ctx *ctx, int64_t *p_begin, int64_t *p_end, int64_t *n_params_global);
+
 /* Registers device allocator hooks (before gasloc_start only). */
 int gasloc_set_allocator(gasloc_ctx *ctx, gasloc_alloc_fn alloc, gasloc_free_fn free_fn,
                          void *user);
@@ -216,13 +238,15 @@ int gasloc_consensus_error(gasloc_ctx *ctx, double *out);
  * reduction kernel (ignores the value the last gossip round produced). */
 int gasloc_consensus_error_now(gasloc_ctx *ctx, double *out);
 
-/* The quantity gasloc_consensus_error returns, copied to host_dst (caller
- * memory; page-locked memory keeps the copy asynchronous) on the context's
- * stream without waiting for it: the per-round metric of a training loop
- * can be logged without draining the GPU's queue after every round.
- * *host_dst holds the value once the stream has passed the copy, e.g. after
- * gasloc_synchronize; later rounds do not disturb a copy already enqueued. */
-int gasloc_consensus_error_async(gasloc_ctx *ctx, double *host_dst);
+/* The quantity gasloc_consensus_error returns, copied to dst on the
+ * context's stream without waiting for it: the per-round metric of a training
+ * loop can be logged without draining the GPU's queue after every round.
+ * dst is caller memory, host (page-locked memory keeps the copy asynchronous)
+ * or device (e.g. the operand of an all-reduce that adds the shares of
+ * contexts holding disjoint ranges, see gasloc_set_range).  *dst holds the
+ * value once the stream has passed the copy, e.g. after gasloc_synchronize;
+ * later rounds do not disturb a copy already enqueued. */
+int gasloc_consensus_error_async(gasloc_ctx *ctx, double *dst);
 
 /* Waits until every call enqueued on the context's stream has finished;
  * EDEVICE if a kernel reported an error (the flag is then cleared). */

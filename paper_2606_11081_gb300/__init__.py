@@ -64,6 +64,8 @@ SIGNATURES = {
     "gasloc_set_hparams": (ctypes.c_int, [_P, ctypes.POINTER(Hparams)]),
     "gasloc_get_hparams": (ctypes.c_int, [_P, ctypes.POINTER(Hparams)]),
     "gasloc_set_layout": (ctypes.c_int, [_P, _I32, _I64P]),
+    "gasloc_set_range": (ctypes.c_int, [_P, _I64, _I64]),
+    "gasloc_get_range": (ctypes.c_int, [_P, _I64P, _I64P, _I64P]),
     "gasloc_set_allocator": (ctypes.c_int, [_P, ALLOC_FN, FREE_FN, _P]),
     "gasloc_set_stream": (ctypes.c_int, [_P, _P]),
     "gasloc_start": (ctypes.c_int, [_P]),
@@ -160,6 +162,17 @@ def gasloc_set_layout(ctx, numels: Sequence[int]) -> None:
     _check(_lib.gasloc_set_layout(ctx, int(a.size), _arr(a, _I64P)))
 
 
+def gasloc_set_range(ctx, p_begin: int, p_end: int) -> None:
+    _check(_lib.gasloc_set_range(ctx, p_begin, p_end))
+
+
+def gasloc_get_range(ctx):
+    """(p_begin, p_end, n_params of the whole problem)."""
+    a, b, n = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    _check(_lib.gasloc_get_range(ctx, ctypes.byref(a), ctypes.byref(b), ctypes.byref(n)))
+    return a.value, b.value, n.value
+
+
 def gasloc_set_allocator(ctx, alloc_fn, free_fn, user=None) -> None:
     _check(_lib.gasloc_set_allocator(ctx, alloc_fn, free_fn, user))
 
@@ -221,10 +234,10 @@ def gasloc_consensus_error_now(ctx) -> float:
     return out.value
 
 
-def gasloc_consensus_error_async(ctx, host_ptr: int) -> None:
-    """Enqueues the copy of the consensus error to host address host_ptr
-    (8 bytes; pinned memory keeps it asynchronous)."""
-    _check(_lib.gasloc_consensus_error_async(ctx, ctypes.c_void_p(host_ptr)))
+def gasloc_consensus_error_async(ctx, dst_ptr: int) -> None:
+    """Enqueues the copy of the consensus error to address dst_ptr (8 bytes,
+    host or device; pinned host memory keeps it asynchronous)."""
+    _check(_lib.gasloc_consensus_error_async(ctx, ctypes.c_void_p(dst_ptr)))
 
 
 def gasloc_synchronize(ctx) -> None:
@@ -372,7 +385,10 @@ class Context:
     def __init__(self, n_workers: int, n_params: int, topology: str, seed: int,
                  hparams: Optional[Hparams] = None, numels: Optional[Sequence[int]] = None,
                  local_steps: Optional[Sequence[int]] = None, draw_hmax: Optional[int] = None,
-                 use_torch: bool = True, stream: Optional[int] = None):
+                 use_torch: bool = True, stream: Optional[int] = None,
+                 p_range: Optional[Sequence[int]] = None):
+        """p_range = (p_begin, p_end): hold only those parameters of every
+        replica (gasloc_set_range); self.P is then p_end - p_begin."""
         load_library()
         self.n = n_workers
         self.P = n_params
@@ -383,6 +399,9 @@ class Context:
             gasloc_set_hparams(self.h, hparams)
         if numels is not None:
             gasloc_set_layout(self.h, numels)
+        if p_range is not None:
+            gasloc_set_range(self.h, int(p_range[0]), int(p_range[1]))
+            self.P = int(p_range[1]) - int(p_range[0])
         if use_torch:
             import torch
             self._alloc = _TorchAllocator()

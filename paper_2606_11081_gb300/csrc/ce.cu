@@ -7,7 +7,9 @@
 // loads in flight per batch; with bf16 storage the columns of two tiles are
 // loaded together, so that a thread keeps as many bytes in flight as with
 // fp32).  Per element the shifted one-pass form
-// e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with s = x_0k, in fp32.
+// e_k = sum_i (x_ik - s)^2 - (sum_i (x_ik - s))^2 / n with s = x_0k, in fp32;
+// each e_k is widened and added on its own, so the value of an element does
+// not depend on the column it shares (nor on how a range is cut).
 // Reduction: fp64 per thread, warp shuffles, one partial per CTA, the last
 // CTA adds the partials in CTA order (atomic ticket; nothing waits).  Reads
 // one element per worker-element (4 or 2 bytes).
@@ -95,13 +97,10 @@ __global__ void __launch_bounds__(kBlock, 3) ce_kernel(const CeArgs a) {
             }
         }
 #pragma unroll
-        for (int p = 0; p < TPI; ++p) {
-            float e = 0.f;
+        for (int p = 0; p < TPI; ++p)
 #pragma unroll
-            for (int l = 0; l < 4; ++l)
-                if (l < nvalid[p]) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[p][l], inv_n), s1[p][l], s2[p][l]));
-            acc += static_cast<double>(e);
-        }
+            for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
+                if (l < nvalid[p]) acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1[p][l], inv_n), s1[p][l], s2[p][l]));
     }
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;

@@ -88,11 +88,9 @@ __global__ void __launch_bounds__(kBlock) ce_noalloc_kernel(const float *__restr
                     }
                 }
             }
-            float e = 0.f;
 #pragma unroll
-            for (int l = 0; l < 4; ++l)
-                if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
-            acc += static_cast<double>(e);
+            for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
+                if (l < nvalid) acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
         }
         for (int o = 16; o > 0; o >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, o);
         if (lane == 0) red[warp] = acc;

@@ -99,12 +99,15 @@ void gasloc::set_last_error(const char *msg) { g_err = msg; }
 
 struct gasloc_ctx {
     int32_t n = 0;
-    int64_t P = 0;
+    int64_t P = 0;                   // parameters per replica this context holds (p_end - p_begin)
+    int64_t P_global = 0;            // parameters per replica of the whole problem
+    int64_t p_begin = 0, p_end = 0;  // the global indices [p_begin, p_end) this context holds
+    std::vector<int64_t> layout;     // tensor sizes of the whole problem (gasloc_set_layout)
     TopoSpec spec{};
     uint64_t seed = 0;
     gasloc_hparams hp{};
     std::vector<int64_t> numels;
-    gasloc_alloc_fn alloc = nullptr;
+    gasloc_alloc_fn alloc = nullptr;   // numels: the context's pieces of those tensors (gasloc_start)
     gasloc_free_fn free_fn = nullptr;
     void *alloc_user = nullptr;
     cudaStream_t stream = nullptr;
@@ -469,6 +472,10 @@ int gasloc_init(int32_t n_workers, int64_t n_params, const char *topology, uint6
     if (!c) return fail(GASLOC_ENOMEM, "out of host memory");
     c->n = n_workers;
     c->P = n_params;
+    c->P_global = n_params;
+    c->p_begin = 0;
+    c->p_end = n_params;
+    c->layout.assign(1, n_params);
     c->spec = spec;
     c->seed = seed;
     gasloc_default_hparams(&c->hp);
@@ -515,9 +522,30 @@ int gasloc_set_layout(gasloc_ctx *c, int32_t n_tensors, const int64_t *numels) {
         if (numels[t] < 1) return fail(GASLOC_EINVAL, "tensor %d has %lld elements", t, (long long)numels[t]);
         tot += numels[t];
     }
-    if (tot != c->P) return fail(GASLOC_EINVAL, "tensor sizes sum to %lld, not n_params %lld", (long long)tot,
-                                 (long long)c->P);
-    c->numels.assign(numels, numels + n_tensors);
+    if (tot != c->P_global)
+        return fail(GASLOC_EINVAL, "tensor sizes sum to %lld, not n_params %lld", (long long)tot,
+                    (long long)c->P_global);
+    c->layout.assign(numels, numels + n_tensors);
+    return GASLOC_OK;
+}
+
+int gasloc_set_range(gasloc_ctx *c, int64_t p_begin, int64_t p_end) {
+    if (!c) return fail(GASLOC_EINVAL, "context is NULL");
+    if (c->started) return fail(GASLOC_ESTATE, "the range cannot change after gasloc_start");
+    if (p_begin < 0 || p_end <= p_begin || p_end > c->P_global)
+        return fail(GASLOC_EINVAL, "range [%lld, %lld) is not a non-empty part of [0, %lld)", (long long)p_begin,
+                    (long long)p_end, (long long)c->P_global);
+    c->p_begin = p_begin;
+    c->p_end = p_end;
+    c->P = p_end - p_begin;
+    return GASLOC_OK;
+}
+
+int gasloc_get_range(const gasloc_ctx *c, int64_t *p_begin, int64_t *p_end, int64_t *n_params_global) {
+    if (!c || !p_begin || !p_end || !n_params_global) return fail(GASLOC_EINVAL, "NULL argument");
+    *p_begin = c->p_begin;
+    *p_end = c->p_end;
+    *n_params_global = c->P_global;
     return GASLOC_OK;
 }
 
@@ -549,6 +577,21 @@ int gasloc_start(gasloc_ctx *c) {
 
     const int32_t n = c->n;
     const int32_t nh = c->hp.per_worker_h ? n : 1;
+    // the context's pieces of the problem's tensors: each tensor cut to
+    // [p_begin, p_end), with the global index of its first element
+    std::vector<int64_t> piece_goff;
+    c->numels.clear();
+    {
+        int64_t off = 0;
+        for (int64_t ne : c->layout) {
+            const int64_t lo = std::max(off, c->p_begin), hi = std::min(off + ne, c->p_end);
+            if (hi > lo) {
+                c->numels.push_back(hi - lo);
+                piece_goff.push_back(lo);
+            }
+            off += ne;
+        }
+    }
     // size check before any allocation
     int64_t need = 0;
     for (int64_t ne : c->numels) {
@@ -579,14 +622,13 @@ int gasloc_start(gasloc_ctx *c) {
     // replica store
     c->tens_h.clear();
     c->goff.clear();
-    int64_t g = 0;
     for (size_t t = 0; t < c->numels.size(); ++t) {
         TensorDesc d{};
         d.numel = c->numels[t];
         d.wstride = round_up(d.numel, kPadFloats);
         d.hstride = c->hp.per_worker_h ? d.wstride : 0;
-        d.goff = g;
-        g += d.numel;
+        d.goff = piece_goff[t];
+        d.loff = piece_goff[t] - c->p_begin;
         void **arrs[6] = {&d.x, &d.y, &d.m, &d.v, &d.b, &d.c};
         for (void **a : arrs) {
             *a = c->dalloc(static_cast<size_t>(n) * d.wstride * esize_of(c));
@@ -971,7 +1013,7 @@ int gasloc_consensus_error_async(gasloc_ctx *c, double *host_dst) {
     NvtxRange r("gasloc_consensus_error_async");
     int rc = check_started(c);
     if (rc) return rc;
-    if (!host_dst) return fail(GASLOC_EINVAL, "host_dst is NULL");
+    if (!host_dst) return fail(GASLOC_EINVAL, "dst is NULL");
     const double *src = c->ce_d;
     if (!c->ce_valid || c->round == 0) {
         CeArgs a{c->tens_d, c->tiles_a, c->ntiles_a, c->n, c->hp.storage, c->partials, c->ticket, c->ce_d, c->err_d};
@@ -980,7 +1022,8 @@ int gasloc_consensus_error_async(gasloc_ctx *c, double *host_dst) {
     } else {
         src = c->ce_ring + (c->round - 1) % kCeRing;
     }
-    cudaError_t e = cudaMemcpyAsync(host_dst, src, sizeof(double), cudaMemcpyDeviceToHost, c->stream);
+    // host or device memory: the copy's direction follows from the address
+    cudaError_t e = cudaMemcpyAsync(host_dst, src, sizeof(double), cudaMemcpyDefault, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "copying the consensus error");
     return GASLOC_OK;
 }
@@ -1068,7 +1111,7 @@ int gasloc_read(gasloc_ctx *c, int32_t which, int32_t worker, float *host) {
         for (const TensorDesc &d : c->tens_h) {
             int64_t stride = 0;
             const char *p = buffer_base(d, which, &stride) + static_cast<size_t>(worker * stride) * es;
-            cudaError_t e = cudaMemcpyAsync(host + d.goff, p, static_cast<size_t>(d.numel) * 4,
+            cudaError_t e = cudaMemcpyAsync(host + d.loff, p, static_cast<size_t>(d.numel) * 4,
                                             cudaMemcpyDeviceToHost, c->stream);
             if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
         }
@@ -1085,7 +1128,7 @@ int gasloc_read(gasloc_ctx *c, int32_t which, int32_t worker, float *host) {
             rc = launch_checked(c, launch_convert(p + static_cast<size_t>(k0) * es, st.p, len, false, c->stream),
                                 "widen kernel");
             if (rc) return rc;
-            cudaError_t e = cudaMemcpyAsync(host + d.goff + k0, st.p, static_cast<size_t>(len) * 4,
+            cudaError_t e = cudaMemcpyAsync(host + d.loff + k0, st.p, static_cast<size_t>(len) * 4,
                                             cudaMemcpyDeviceToHost, c->stream);
             if (e != cudaSuccess) return cuda_fail(e, "device-to-host copy");
         }
@@ -1112,12 +1155,12 @@ int gasloc_write(gasloc_ctx *c, int32_t which, int32_t worker, const float *host
         char *row0 = p + static_cast<size_t>(w0 * stride) * es;
         cudaError_t e = cudaSuccess;
         if (es == 4) {
-            e = cudaMemcpyAsync(row0, host + d.goff, bytes, cudaMemcpyHostToDevice, c->stream);
+            e = cudaMemcpyAsync(row0, host + d.loff, bytes, cudaMemcpyHostToDevice, c->stream);
             if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
         } else {
             for (int64_t k0 = 0; k0 < d.numel; k0 += st.elems) {
                 const int64_t len = d.numel - k0 < st.elems ? d.numel - k0 : st.elems;
-                e = cudaMemcpyAsync(st.p, host + d.goff + k0, static_cast<size_t>(len) * 4, cudaMemcpyHostToDevice,
+                e = cudaMemcpyAsync(st.p, host + d.loff + k0, static_cast<size_t>(len) * 4, cudaMemcpyHostToDevice,
                                     c->stream);
                 if (e != cudaSuccess) return cuda_fail(e, "host-to-device copy");
                 rc = launch_checked(c, launch_convert(st.p, row0 + static_cast<size_t>(k0) * es, len, true, c->stream),
@@ -1223,6 +1266,7 @@ struct CkptHeader {
     int32_t has_Hi;
     int32_t storage;
     int32_t pad;
+    int64_t p_begin, p_end;   // the range of the problem's parameters the checkpoint holds
 };
 }  // namespace
 
@@ -1235,10 +1279,12 @@ int gasloc_save(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "wb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s' for writing", path);
     CkptHeader h{};
-    std::memcpy(h.magic, "GASLOCK3", 8);
-    h.version = 3;
+    std::memcpy(h.magic, "GASLOCK4", 8);
+    h.version = 4;
     h.n = c->n;
-    h.P = c->P;
+    h.P = c->P_global;
+    h.p_begin = c->p_begin;
+    h.p_end = c->p_end;
     h.n_tensors = static_cast<int64_t>(c->numels.size());
     h.seed = c->seed;
     h.kind = c->spec.kind;
@@ -1284,9 +1330,10 @@ int gasloc_load(gasloc_ctx *c, const char *path) {
     FILE *f = std::fopen(path, "rb");
     if (!f) return fail(GASLOC_EIO, "cannot open '%s'", path);
     CkptHeader h{};
-    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK3", 8) == 0 && h.version == 3;
+    bool ok = std::fread(&h, sizeof h, 1, f) == 1 && std::memcmp(h.magic, "GASLOCK4", 8) == 0 && h.version == 4;
     if (!ok) { std::fclose(f); return fail(GASLOC_EIO, "'%s' is not a checkpoint", path); }
-    if (h.n != c->n || h.P != c->P || h.n_tensors != static_cast<int64_t>(c->numels.size()) || h.seed != c->seed ||
+    if (h.n != c->n || h.P != c->P_global || h.p_begin != c->p_begin || h.p_end != c->p_end ||
+        h.n_tensors != static_cast<int64_t>(c->numels.size()) || h.seed != c->seed ||
         h.kind != c->spec.kind || h.rows != c->spec.rows || h.cols != c->spec.cols ||
         h.per_worker_h != c->hp.per_worker_h || h.storage != c->hp.storage) {
         std::fclose(f);

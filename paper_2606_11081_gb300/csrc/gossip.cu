@@ -32,7 +32,7 @@
 // Consensus error: per element e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
 // S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x; fp32 per
 // element (the thread owning the column, or for G > 1 one thread per column
-// after the tile's barrier), fp64 across elements,
+// after the tile's barrier), each element's term widened to fp64 on its own,
 // one partial per CTA, the last CTA (atomic ticket, nothing waits) adds the
 // partials in CTA order.
 //
@@ -570,11 +570,9 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
             if (active && (G == 1 || g == 0)) {
                 const float s1[4] = {s1a.x, s1a.y, s1b.x, s1b.y}, s2[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
-                float e = 0.f;
 #pragma unroll
-                for (int l = 0; l < 4; ++l)
-                    if (l < nvalid) e = __fadd_rn(e, __fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
-                ce_acc += static_cast<double>(e);
+                for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
+                    if (l < nvalid) ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
             }
             ptx::fence_proxy_async_smem();   // outputs visible to the bulk stores
             __syncwarp();

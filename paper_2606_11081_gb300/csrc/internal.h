@@ -22,7 +22,9 @@ struct TensorDesc {
     int64_t numel;     // valid elements per worker
     int64_t wstride;   // floats between consecutive workers
     int64_t hstride;   // floats between workers in h (0 when shared)
-    int64_t goff;      // global index of element 0 (concatenation order)
+    int64_t goff;      // global index of element 0 (concatenation order): keys the generators
+    int64_t loff;      // index of element 0 in the context's own elements (goff minus the
+                       // first global index the context holds): places host and output arrays
 };
 
 // A contiguous run of at most `tile` elements of one tensor.  start is a

@@ -240,8 +240,8 @@ __global__ void __launch_bounds__(256) average_kernel(const TensorDesc *tens, co
                 s[3] = __fadd_rn(s[3], v.w);
             }
         }
-        if (!span_ok(d.goff + off, d.goff + off + nvalid, n_params, err)) continue;
-        float *o = dst + d.goff + off;
+        if (!span_ok(d.loff + off, d.loff + off + nvalid, n_params, err)) continue;
+        float *o = dst + d.loff + off;
         const float4 r = make_float4(__fmul_rn(s[0], inv_n), __fmul_rn(s[1], inv_n), __fmul_rn(s[2], inv_n),
                                      __fmul_rn(s[3], inv_n));
         if (nvalid == 4 && (reinterpret_cast<uintptr_t>(o) & 15u) == 0) {
@@ -259,14 +259,14 @@ __global__ void gather_kernel(const TensorDesc *tens, int32_t ntens, int32_t whi
     const int64_t q = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
     if (q >= n) return;
     const int64_t k = idx[q];
-    // binary search for the tensor holding global index k
+    // binary search for the tensor holding the context's element k
     int lo = 0, hi = ntens - 1;
     while (lo < hi) {
         const int mid = (lo + hi + 1) / 2;
-        if (tens[mid].goff <= k) lo = mid; else hi = mid - 1;
+        if (tens[mid].loff <= k) lo = mid; else hi = mid - 1;
     }
     const TensorDesc d = tens[lo];
-    const int64_t off = k - d.goff;
+    const int64_t off = k - d.loff;
     if (k < 0 || off < 0 || off >= d.numel) {
         atomicCAS(err, kDevOk, kDevBadIndex);
         out[q] = 0.0f;

@@ -41,3 +41,38 @@ def workload_pair(name, kidx=None):
     w = wl.WORKLOADS[name]
     return w, make_pair(w.n_workers, w.n_params, w.topology, w.seed, wl.hparams_of(w), w.numels,
                         draw_hmax=w.draw_hmax, kidx=kidx)
+
+
+U32 = 2.0 ** -24
+
+
+def ce_bound(x):
+    """Relative error bound of the library's consensus error of the replicas x
+    ([n, P] stored values) against the exact value (the oracle's fp64 one).
+
+    Per element the library forms dv_i = x_i - x_0 (x_0: worker 0's value),
+    S1 = sum dv_i and S2 = sum dv_i^2 over ascending i and e = S2 - (S1/n) S1,
+    in fp32 with one rounding per operation (u = 2^-24).  With a_i = x_i - x_0
+    and D = sum a_i^2: S2 is within gamma_{n+1} D of D, S1 within gamma_n
+    sum|a_i| <= gamma_n sqrt(n D) of sum a_i, so (S1/n) S1 (with the roundings
+    of 1/n and of the product) is within about (2n + 2) u D of its exact value
+    (S1^2 / n <= D), and the final rounding adds u e: the element's error is at
+    most about (3n + 3) u D + u e; (3n + 4) u D + 2 u e is taken to cover the
+    higher-order terms.  Over the elements, in fp64, the total's relative
+    error is at most (3n + 4) u kappa + 2 u with kappa = sum D / sum e >= 1,
+    plus the fp64 sums of both sides over P elements (2 P 2^-53)."""
+    x = np.asarray(x, np.float64)
+    n, P = x.shape
+    e = ((x - x.mean(0)) ** 2).sum()
+    if e == 0.0:
+        return 0.0
+    kappa = ((x - x[0]) ** 2).sum() / e
+    return (3 * n + 4) * U32 * kappa + 2 * U32 + 2 * P * 2.0 ** -53
+
+
+def assert_ce(got, st, x=None):
+    """The library's consensus error `got` against the oracle state's, within
+    ce_bound of the oracle's replicas."""
+    ref = st.consensus_error()
+    tol = ce_bound(st.get_all("x") if x is None else x)
+    assert abs(got - ref) <= tol * abs(ref) + 1e-30, (got, ref, tol)

@@ -132,3 +132,22 @@ def test_start_without_gpu_fails_cleanly(lib):
         assert e.value.code in (g.ECUDA, g.ENOMEM)
     finally:
         g.gasloc_destroy(c)
+
+
+def test_range_validation(lib):
+    ctx = g.gasloc_init(4, 1000, "ring", 1)
+    try:
+        assert g.gasloc_get_range(ctx) == (0, 1000, 1000)
+        for a, b in [(-1, 10), (5, 5), (10, 5), (0, 1001), (1000, 1001)]:
+            with pytest.raises(g.GaslocError) as e:
+                g.gasloc_set_range(ctx, a, b)
+            assert e.value.code == g.EINVAL, (a, b)
+        g.gasloc_set_range(ctx, 250, 999)
+        assert g.gasloc_get_range(ctx) == (250, 999, 1000)
+        # the layout still describes the whole problem
+        with pytest.raises(g.GaslocError) as e:
+            g.gasloc_set_layout(ctx, [500, 249])
+        assert e.value.code == g.EINVAL
+        g.gasloc_set_layout(ctx, [500, 500])
+    finally:
+        g.gasloc_destroy(ctx)

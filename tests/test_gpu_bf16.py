@@ -9,7 +9,7 @@ import paper_2606_11081_gb300 as g
 from paper_2606_11081_gb300 import build as gbuild
 from paper_2606_11081_gb300 import workloads as wl
 
-from _pairs import make_pair, workload_pair
+from _pairs import make_pair, workload_pair, assert_ce
 
 pytestmark = pytest.mark.gpu
 BF = dict(storage="bf16")
@@ -56,7 +56,7 @@ def test_bf16_trajectory(mode, N, topo, kw):
             st.local_steps(H)
             ctx.gossip_round()
             st.gossip_round()
-            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+            assert_ce(ctx.consensus_error(), st)
         same(ctx, st, ("x", "b", "m", "v"))
 
 
@@ -77,7 +77,7 @@ def test_bf16_dense_mixing(mode, N, topo, kw):
             st.local_steps(H)
             ctx.gossip_round()
             st.gossip_round()
-            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+            assert_ce(ctx.consensus_error(), st)
         same(ctx, st, ("x", "b", "m", "v", "y"))
 
 
@@ -128,7 +128,7 @@ def test_bf16_bench_workload_full_size_sampled():
         for which in ("x", "b", "m", "v"):
             for i in range(w.n_workers):
                 np.testing.assert_array_equal(ctx.gather(which, i, kidx), st.get(which, i).astype(np.float32))
-        assert ctx.consensus_error() == pytest.approx(ctx.consensus_error_now(), rel=1e-6)
+        assert ctx.consensus_error() == pytest.approx(ctx.consensus_error_now(), rel=1e-12)
     finally:
         ctx.close()
         torch.cuda.synchronize()

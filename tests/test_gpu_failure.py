@@ -11,7 +11,7 @@ import oracle
 import paper_2606_11081_gb300 as g
 from paper_2606_11081_gb300 import build as gbuild
 
-from _pairs import make_pair
+from _pairs import make_pair, assert_ce
 
 pytestmark = pytest.mark.gpu
 
@@ -40,7 +40,7 @@ def test_bounded_wait_expires_and_context_survives():
             ctx.gossip_round()
             st.local_steps(1)
             st.gossip_round()
-        assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)
+        assert_ce(ctx.consensus_error(), st)
         np.testing.assert_array_equal(ctx.read_all("x"), st.get_all("x").astype(np.float32))
         with pytest.raises(g.GaslocError):
             g._check(g.gasloc_selftest_bounded_wait(ctx.h, 0))      # limit out of range

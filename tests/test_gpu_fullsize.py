@@ -68,7 +68,7 @@ def test_workload_full_size_sampled(name):
             st.gossip_round()
         ce_fused = ctx.consensus_error()
         ce_now = ctx.consensus_error_now()
-        assert ce_fused == pytest.approx(ce_now, rel=1e-6) and ce_fused > 0
+        assert ce_fused == pytest.approx(ce_now, rel=1e-12) and ce_fused > 0
         for which in ("x", "b", "m", "v"):
             for i in range(w.n_workers):
                 a = ctx.gather(which, i, kidx)

@@ -18,7 +18,7 @@ import paper_2606_11081_gb300 as g
 from paper_2606_11081_gb300 import build as gbuild
 from paper_2606_11081_gb300 import workloads as wl
 
-from _pairs import TOL, make_pair, oracle_problem, within_tol
+from _pairs import TOL, assert_ce, ce_bound, make_pair, oracle_problem, within_tol
 
 pytestmark = pytest.mark.gpu
 
@@ -137,7 +137,7 @@ def test_trajectory_parity(mode, N, topo, kw):
             st.local_steps(H)
             ctx.gossip_round()
             st.gossip_round()
-            assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+            assert_ce(ctx.consensus_error(), st)
         assert_state_equal(ctx, st, ("x", "b", "m", "v"))
 
 
@@ -153,7 +153,7 @@ def test_edge_case_shapes(N, P, topo):
             ctx.gossip_round()
             st.gossip_round()
         assert_state_equal(ctx, st, ("x", "b"))
-        assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5, abs=1e-30)
+        assert_ce(ctx.consensus_error(), st)
 
 
 def test_ring_n4_p1m_full_size():
@@ -167,7 +167,7 @@ def test_ring_n4_p1m_full_size():
             ctx.gossip_round()
             st.gossip_round()
             if r % 10 == 9:
-                assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)
+                assert_ce(ctx.consensus_error(), st)
         assert_state_equal(ctx, st, ("x", "b", "m", "v"))
         np.testing.assert_allclose(ctx.average_host(), st.average(), rtol=2e-6, atol=1e-7)
 
@@ -180,14 +180,15 @@ def test_consensus_error_closed_form_and_paths():
     with ctx:
         for i in range(N):
             ctx.write("x", i, np.full(P, float(i), np.float32))
-        # per-element fp32 shifted sums: relative error below ~N * 2^-22
-        assert ctx.consensus_error() == pytest.approx(P * (N * N - 1) / 12, rel=5e-6)
+        # per-element fp32 shifted sums, within the bound of the shifted form
+        xs = np.repeat(np.arange(N, dtype=np.float64)[:, None], P, axis=1)
+        assert ctx.consensus_error() == pytest.approx(P * (N * N - 1) / 12, rel=ce_bound(xs))
         ctx.local_steps(1)
         ctx.gossip_round()
         fused = ctx.consensus_error()
-        # the fused and the standalone reductions shift each column by different
-        # replicas (sent value vs new x of worker 0): equal to fp32 rounding
-        assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-6)
+        # the fused and the standalone reductions take the same per-element
+        # terms (both shift by worker 0's new x); only the fp64 order differs
+        assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-12)
 
 
 @pytest.mark.parametrize("N", [8, 32])
@@ -208,11 +209,9 @@ def test_consensus_error_near_consensus_far_from_zero(N):
     x = np.stack([(a + 1e-3 * (i - (N - 1) / 2)).astype(np.float32) for i in range(N)])
     xd = x.astype(np.float64)
     exact = ((xd - xd.mean(0)) ** 2).sum() / N
-    # the shifted form's bound for these values: relative (3N + 2) u kappa + u,
-    # kappa = sum_i (x_i - x_0)^2 / sum_i (x_i - xbar)^2 (worker 0's shift)
-    kappa = ((xd - xd[0]) ** 2).sum() / (((xd - xd.mean(0)) ** 2).sum())
-    u = 2.0 ** -24
-    tol = (3 * N + 2) * u * kappa + u
+    # the shifted form's bound for these values (ce_bound: worker 0's shift
+    # makes kappa = sum (x_i - x_0)^2 / sum (x_i - xbar)^2 about 4 here)
+    tol = ce_bound(xd)
     with ctx:
         for i in range(N):
             ctx.write("x", i, x[i])
@@ -261,9 +260,9 @@ def test_tensor_list_equals_flat():
             for c in (a, b):
                 c.local_steps(3)
                 c.gossip_round()
-        # per-element terms are identical; the fp32 sums of a 16-byte column
-        # group different elements where a tensor boundary is not 4-aligned
-        assert a.consensus_error() == pytest.approx(b.consensus_error(), rel=1e-6)
+        # per-element terms are identical and each enters the fp64 sum on its
+        # own: only the order of the fp64 sums differs
+        assert a.consensus_error() == pytest.approx(b.consensus_error(), rel=1e-12)
         for w in ("x", "y", "m", "v", "b", "c", "h"):
             np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
         # the per-tensor buffers are separate allocations with the real sizes

@@ -10,7 +10,7 @@ import paper_2606_11081_gb300 as g
 from paper_2606_11081_gb300 import build as gbuild
 from paper_2606_11081_gb300 import workloads as wl
 
-from _pairs import make_pair
+from _pairs import make_pair, assert_ce
 
 pytestmark = pytest.mark.gpu
 
@@ -119,7 +119,7 @@ def test_async_consensus_error_reads():
         a.synchronize()
         got = host.numpy().tolist()
     assert got == want
-    assert want[R] == pytest.approx(st.consensus_error(), rel=1e-5)
+    assert_ce(want[R], st)
 
 
 def test_hparam_change_matches_oracle():
@@ -145,7 +145,7 @@ def test_hparam_change_matches_oracle():
             st.gossip_round()
         for w in ("x", "y", "m", "v", "b"):
             np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)
-        assert ctx.consensus_error() == pytest.approx(st.consensus_error(), rel=1e-5)
+        assert_ce(ctx.consensus_error(), st)
 
 
 def test_run_with_lr_schedule_matches_stepwise():
