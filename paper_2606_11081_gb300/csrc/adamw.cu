@@ -13,9 +13,9 @@
 // the step counters and writes the next step's scalars.
 //
 // fp32 storage (adamw_kernel): one thread owns a column of 4 consecutive
-// elements of a tile and walks the active workers U at a time (U = 4, or 3
-// with per-worker h), issuing all of their loads before any arithmetic so
-// that about 256 bytes of requests per thread stay in flight.
+// elements of a tile and walks the active workers U at a time (U from 2 to 4,
+// chosen per launch from the number of workers stepped and whether each has
+// its own h: see Batch), issuing all of their loads before any arithmetic.
 // bf16 storage (adamw_staged_kernel): a producer warp stages the rows in
 // shared memory with bulk copies while 256 consumer threads compute (see
 // there); with half the bytes per element the arithmetic sets the pace, and
@@ -476,21 +476,38 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
     }
 }
 
-// Workers per load batch of adamw_kernel: 16-byte loads, so that a thread
-// keeps about 256 bytes of loads in flight.
-template <typename T> struct Batch { static constexpr int kShared = 4, kPerWorkerH = 3; };
+// Workers per load batch of adamw_kernel (16-byte loads of 4 or 5 rows per
+// worker, all issued before the batch's arithmetic), chosen per launch from
+// the number of workers it steps.  Measured on GB300 (fraction of the copy
+// peak, whole launches at full size; every variant runs 2 CTAs of 256 threads
+// per SM):
+//   shared curvature:  8 workers  U = 4: 1.002, U = 3: 0.987, U = 2: 0.937
+//                      16 workers U = 4: 0.957, U = 3: 0.987, U = 2: 0.937
+//   own curvature:     32 / 26 / 22 / 17 / 16 / 11 workers U = 2: 1.001-1.007
+//                      against U = 3: 0.964-0.980, U = 4: 0.84 (spills);
+//                      7 / 3 workers U = 3: 1.02 / 1.03 against U = 2: 0.99 / 0.95.
+template <typename T> struct Batch {
+    static constexpr int kSharedFew = 4, kSharedMany = 3;       // shared h: <= 8 workers, more
+    static constexpr int kOwnFew = 3, kOwnMany = 2;             // own h: <= 7 workers, more
+    static constexpr int kSharedFewMax = 8, kOwnFewMax = 7;
+};
 
+template <int U, bool P, typename T>
+int occupancy(int block) {
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<U, P, false, T>, block, 0) != cudaSuccess)
+        return 1;
+    return nb > 0 ? nb : 1;
+}
+
+// CTAs per SM that every batch variant of the storage reaches (the grid is
+// sized once per context)
 template <typename T>
 int blocks_per_sm(int block, bool per_worker_h) {
-    int nb = 0;
-    const cudaError_t e =
-        per_worker_h
-            ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kPerWorkerH, true, false, T>,
-                                                            block, 0)
-            : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, adamw_kernel<Batch<T>::kShared, false, false, T>,
-                                                            block, 0);
-    if (e != cudaSuccess) return 1;
-    return nb > 0 ? nb : 1;
+    using B = Batch<T>;
+    const int a = per_worker_h ? occupancy<B::kOwnFew, true, T>(block) : occupancy<B::kSharedFew, false, T>(block);
+    const int b = per_worker_h ? occupancy<B::kOwnMany, true, T>(block) : occupancy<B::kSharedMany, false, T>(block);
+    return a < b ? a : b;
 }
 
 template <bool P, bool S>
@@ -532,16 +549,21 @@ void launch_staged(const AdamwArgs &a, int grid, cudaStream_t s) {
 
 template <typename T>
 void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
-    constexpr int UP = Batch<T>::kPerWorkerH, US = Batch<T>::kShared;   // per-worker h: 5 loads per worker
+    using B = Batch<T>;
     const bool sched = a.lr_steps > 0;
-    if (a.per_worker_h && sched)
-        adamw_kernel<UP, true, true, T><<<grid, kBlock, 0, s>>>(a);
-    else if (a.per_worker_h)
-        adamw_kernel<UP, true, false, T><<<grid, kBlock, 0, s>>>(a);
-    else if (sched)
-        adamw_kernel<US, false, true, T><<<grid, kBlock, 0, s>>>(a);
-    else
-        adamw_kernel<US, false, false, T><<<grid, kBlock, 0, s>>>(a);
+    if (a.per_worker_h) {   // 5 loads per worker
+        const bool few = a.n_active <= B::kOwnFewMax;
+        if (few && sched) adamw_kernel<B::kOwnFew, true, true, T><<<grid, kBlock, 0, s>>>(a);
+        else if (few) adamw_kernel<B::kOwnFew, true, false, T><<<grid, kBlock, 0, s>>>(a);
+        else if (sched) adamw_kernel<B::kOwnMany, true, true, T><<<grid, kBlock, 0, s>>>(a);
+        else adamw_kernel<B::kOwnMany, true, false, T><<<grid, kBlock, 0, s>>>(a);
+    } else {                // 4 loads per worker and the tile's shared h
+        const bool few = a.n_active <= B::kSharedFewMax;
+        if (few && sched) adamw_kernel<B::kSharedFew, false, true, T><<<grid, kBlock, 0, s>>>(a);
+        else if (few) adamw_kernel<B::kSharedFew, false, false, T><<<grid, kBlock, 0, s>>>(a);
+        else if (sched) adamw_kernel<B::kSharedMany, false, true, T><<<grid, kBlock, 0, s>>>(a);
+        else adamw_kernel<B::kSharedMany, false, false, T><<<grid, kBlock, 0, s>>>(a);
+    }
 }
 
 }  // namespace

@@ -121,7 +121,8 @@ def test_heterogeneous_steps_per_worker_h():
 
 MODES = ["nesterov", "sgdm", "sgd", "eq2", "dadam", "local_dadam"]
 GRAPHS = [(8, "exp", {}), (16, "matching", {}), (8, "torus:2x4", {"weights": "metropolis"}),
-          (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}), (6, "2peer", {"weights": "lazy"})]
+          (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}), (6, "2peer", {"weights": "lazy"}),
+          (11, "ring", {"per_worker_h": True})]   # own curvature, more than 7 workers: batches of 2 and a tail
 
 
 @pytest.mark.parametrize("mode", MODES)
