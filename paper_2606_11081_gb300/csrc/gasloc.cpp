@@ -76,16 +76,16 @@ EncodeTiledFn encode_tiled() {
     return fn;
 }
 
-// 2-D map over one array of one tensor: [n workers][numel] fp32 with a row
-// pitch of wstride floats, boxes of [n x 256]; out-of-range elements read as
-// zero and are not written.
-bool make_map(CUtensorMap *m, void *base, int64_t numel, int64_t wstride, int32_t n, int storage) {
+// 2-D map over one array of one tensor: [n workers][numel] elements with a
+// row pitch of wstride elements, boxes of [n x box]; out-of-range elements
+// read as zero and are not written.
+bool make_map(CUtensorMap *m, void *base, int64_t numel, int64_t wstride, int32_t n, int storage, int box_elems) {
     EncodeTiledFn enc = encode_tiled();
     if (!enc) return false;
     const bool bf = storage == kStoreBF16;
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(numel), static_cast<cuuint64_t>(n)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(wstride) * (bf ? 2 : 4)};
-    const cuuint32_t box[2] = {256, static_cast<cuuint32_t>(n)};
+    const cuuint32_t box[2] = {static_cast<cuuint32_t>(box_elems), static_cast<cuuint32_t>(n)};
     const cuuint32_t estr[2] = {1, 1};
     return enc(m, bf ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, dims, strides, box,
                estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -665,7 +665,8 @@ int gasloc_start(gasloc_ctx *c) {
         const TensorDesc &d = c->tens_h[t];
         void *arrs[3] = {d.x, d.y, d.b};
         for (int k = 0; k < 3; ++k)
-            if (!make_map(&maps[t * 3 + k], arrs[k], d.numel, d.wstride, n, c->hp.storage)) {
+            if (!make_map(&maps[t * 3 + k], arrs[k], d.numel, d.wstride, n, c->hp.storage,
+                          c->tile_g < 256 ? c->tile_g : 256)) {
                 c->release_all();
                 return fail(GASLOC_ECUDA, "cuTensorMapEncodeTiled failed for tensor %zu", t);
             }
@@ -713,7 +714,7 @@ int gasloc_start(gasloc_ctx *c) {
     c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0, c->hp.storage);
     for (int m = 0; m < 6; ++m) {
         const GossipShape sm = gossip_shape(n, m, c->hp.storage);
-        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm.smem, sm.dense != 0));
+        c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm));
     }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
 

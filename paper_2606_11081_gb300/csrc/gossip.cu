@@ -70,7 +70,11 @@ static_assert(kOffFlags + 16 <= kOffStages, "smem layout");
 static_assert(kOffStages % 128 == 0, "stage alignment");
 __host__ __device__ constexpr size_t stage_offset(int) { return kOffStages; }
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
-constexpr int kBox = 256;                            // elements per TMA box row
+constexpr int kBox = 256;                            // elements per TMA box row (at most)
+// Threads per column above 16 workers: 8, so that a tile is 128 elements
+// (box rows of 128) and a stage of 32 workers' 3 rows is 48 KB, which leaves
+// room for more stages per SM than 96 KB stages would.
+constexpr int kGroupsMany = 8;
 
 // Rows staged per worker: kind 0 = the mixed quantity, kind 1 = own x (own y
 // for the DAdam modes), kind 2 = own b.
@@ -126,6 +130,13 @@ __device__ __forceinline__ float4 keep_tail(float4 v, float4 keep, int nvalid) {
     if (nvalid < 3) v.z = keep.z;
     if (nvalid < 4) v.w = keep.w;
     return v;
+}
+
+// Two consecutive elements from shared memory (8-byte aligned for fp32).
+__device__ __forceinline__ float2 load2_smem(const float *p) { return *reinterpret_cast<const float2 *>(p); }
+__device__ __forceinline__ float2 load2_smem(const bf16 *p) {
+    const uint32_t u = *reinterpret_cast<const uint32_t *>(p);
+    return make_float2(bf_lo(u), bf_hi(u));
 }
 
 // Consensus-error sums of two lanes: dv = x - shift, s1 += dv, s2 += dv dv.
@@ -221,7 +232,9 @@ constexpr int kDenseMax = 8;
 constexpr int kDenseRow = 8;   // dense row i lives in tp->w[kDenseRow + i] and its neighbour mask in
                                // tp->nbr[kDenseRow + i][0] (rows >= n are free)
 
-template <int MODE, typename T, bool DENSE>
+// NARROW: 128-element tiles and box rows (kGroupsMany threads per column,
+// more than 16 workers); otherwise box rows of 256 elements.
+template <int MODE, typename T, bool DENSE, bool NARROW>
 __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kernel(const GossipArgs a) {
     using R = ModeRows<MODE>;
     using E = Elem<T>;
@@ -240,7 +253,9 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
     const int S = a.stages;
     const size_t stage_elems = static_cast<size_t>(R::kRows) * n * TILE;
     constexpr int kVec = 16 / static_cast<int>(sizeof(T));   // elements per 16 bytes
-    const int NQ = TILE / kBox;   // sub-boxes per tile: kind k, sub-box q, worker j at ((k NQ + q) n + j) kBox
+    constexpr int bsh = NARROW ? 7 : 8;   // elements per box row (the tensor maps' box): 1 << bsh
+    constexpr int BOX = 1 << bsh;
+    const int NQ = TILE / BOX;   // sub-boxes per tile: kind k, sub-box q, worker j at ((k NQ + q) n + j) BOX
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     {   // neighbour table -> shared memory: rows 0..n-1 of nbr and w, and deg,
@@ -316,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         const bool none_fresh = (a.fresh_mask & all_mask) == 0u;
         const bool uniform = all_fresh || none_fresh;
         const int kvar = R::kMixX ? 1 : 0;   // the kind whose source depends on freshness
-        auto blk = [&](T *st, int k, int q) { return st + static_cast<size_t>(k * NQ + q) * n * kBox; };
+        auto blk = [&](T *st, int k, int q) { return st + static_cast<size_t>(k * NQ + q) * n * BOX; };
         auto tmap = [&](int tensor, int arr) {   // arr: 0 x, 1 y, 2 b
             return static_cast<const unsigned char *>(a.maps) + (static_cast<size_t>(tensor) * 3 + arr) * 128;
         };
@@ -333,15 +348,15 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         };
         auto store_tile = [&](int64_t j) {   // box stores of tile j, spread over lanes
             const Tile tl = a.tiles[first + j * gstride];
-            const int nq = (tl.len + kBox - 1) / kBox;
+            const int nq = (tl.len + BOX - 1) / BOX;
             T *st = stages + (j % S) * stage_elems;
             const int nops = (R::kHasB ? 2 : 1) * nq;
             fence_maps(tl.tensor);
             for (int o = lane; o < nops; o += 32) {
                 const int k = 1 + o / nq, q = o % nq;
                 const int arr = k == 1 ? 0 : 2;
-                if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
-                tma_store_2d_p<kStorePolicy>(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * kBox), 0,
+                if (!aligned16_ok((tl.start + q * BOX) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
+                tma_store_2d_p<kStorePolicy>(tmap(tl.tensor, arr), static_cast<int32_t>(tl.start + q * BOX), 0,
                                              blk(st, k, q), st_pol);
             }
             bulk_commit();
@@ -370,7 +385,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             }
             const Tile tl = a.tiles[first + it * gstride];
             const TensorDesc &d = a.tens[tl.tensor];
-            const int nq = (tl.len + kBox - 1) / kBox;
+            const int nq = (tl.len + BOX - 1) / BOX;
             const int lenr = (tl.len + kVec - 1) / kVec * kVec;   // whole 16-byte chunks
             T *st = stages + s * stage_elems;
             fence_maps(tl.tensor);
@@ -378,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             uint32_t tx = 0;
             for (int k = 0; k < R::kRows; ++k) {
                 if (k == kvar && !uniform) tx += static_cast<uint32_t>(n) * static_cast<uint32_t>(lenr) * sizeof(T);
-                else tx += static_cast<uint32_t>(nq) * static_cast<uint32_t>(n * kBox * sizeof(T));
+                else tx += static_cast<uint32_t>(nq) * static_cast<uint32_t>(n * BOX * sizeof(T));
             }
             if (lane == 0) ptx::mbar_arrive_expect_tx(&full[s], tx);
             __syncwarp();
@@ -386,20 +401,20 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             for (int o = lane; o < nbox; o += 32) {
                 const int k = o / nq, q = o % nq;
                 if (k == kvar && !uniform) continue;
-                if (!aligned16_ok((tl.start + q * kBox) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
+                if (!aligned16_ok((tl.start + q * BOX) * static_cast<int64_t>(sizeof(T)), a.err)) continue;
                 tma_load_2d_p<kLoadPolicy>(blk(st, k, q), tmap(tl.tensor, arr_of(k)),
-                                           static_cast<int32_t>(tl.start + q * kBox), 0, &full[s], ld_pol);
+                                           static_cast<int32_t>(tl.start + q * BOX), 0, &full[s], ld_pol);
             }
             if (!uniform) {   // per-worker source: y if the worker is fresh, else x
                 for (int j = lane; j < n; j += 32) {
                     const bool fresh = (a.fresh_mask >> j) & 1u;
                     const T *src = static_cast<const T *>(fresh ? d.y : d.x) + j * d.wstride + tl.start;
                     for (int q = 0; q < nq; ++q) {
-                        const int w = lenr - q * kBox < kBox ? lenr - q * kBox : kBox;
-                        if (!row_ok(j, n, tl.start + q * kBox, w, d.wstride, a.err) ||
+                        const int w = lenr - q * BOX < BOX ? lenr - q * BOX : BOX;
+                        if (!row_ok(j, n, tl.start + q * BOX, w, d.wstride, a.err) ||
                             !aligned16_ok(static_cast<int64_t>(w) * sizeof(T), a.err))
                             continue;
-                        ptx::bulk_g2s(blk(st, kvar, q) + static_cast<size_t>(j) * kBox, src + q * kBox,
+                        ptx::bulk_g2s(blk(st, kvar, q) + static_cast<size_t>(j) * BOX, src + q * BOX,
                                       static_cast<uint32_t>(w * sizeof(T)), &full[s]);
                     }
                 }
@@ -431,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
         const int g = threadIdx.x / cols;
         const int col = threadIdx.x % cols;
         const int e0 = 4 * col;
-        const int qb = e0 / kBox, rb = e0 % kBox;   // sub-box of the column, offset in it
+        const int qb = e0 >> bsh, rb = e0 & (BOX - 1);   // sub-box of the column, offset in it
         const float inv_n = static_cast<float>(1.0 / n);
         const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
                          x2::splat(a.gamma), x2::splat(a.eta)};
@@ -447,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             T *st = stages + s * stage_elems;
             // row of worker j, kind k, at this thread's column
             auto cp = [&](int k, int j) {
-                return st + (static_cast<size_t>(k) * NQ + qb) * n * kBox + static_cast<size_t>(j) * kBox + rb;
+                return st + (static_cast<size_t>(k) * NQ + qb) * n * BOX + static_cast<size_t>(j) * BOX + rb;
             };
             float2 s1a = x2::splat(0.f), s1b = s1a, s2a = s1a, s2b = s1a;   // lanes 0-1, 2-3
             const bool active = ok && e0 < tlen;
@@ -555,20 +570,33 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
             }
             if (G > 1) {
                 // Every group's new rows are in shared memory after this
-                // barrier; one thread per column reduces them exactly as the
-                // G = 1 path does (shift by worker 0's new x, ascending i).
+                // barrier.  The column's G threads share its 4 elements
+                // (4 / G each, or one each for the first 4 of G >= 4), and
+                // each reduces its elements exactly as the G = 1 path does:
+                // shift by worker 0's new x, ascending i.
                 consumer_barrier();
-                if (g == 0 && active) {
-                    const float4 x0 = E::load4_smem(cp(1, 0));
-                    for (int i = 0; i < n; ++i) {
-                        const float4 xv = E::load4_smem(cp(1, i));
-                        ce_terms(x2::lo(xv), x2::lo(x0), s1a, s2a);
-                        ce_terms(x2::hi(xv), x2::hi(x0), s1b, s2b);
+                if (active && G == 2) {   // elements 2g, 2g + 1 as a pair
+                    const int l0 = 2 * g;
+                    if (l0 < nvalid) {
+                        const float2 x0 = load2_smem(cp(1, 0) + l0);
+                        float2 s1 = x2::splat(0.f), s2 = s1;
+                        for (int i = 0; i < n; ++i) ce_terms(load2_smem(cp(1, i) + l0), x0, s1, s2);
+                        ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1.x, inv_n), s1.x, s2.x));
+                        if (l0 + 1 < nvalid)
+                            ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1.y, inv_n), s1.y, s2.y));
                     }
+                } else if (active && g < 4 && g < nvalid) {   // G >= 4: element g
+                    const float x0 = E::load1(cp(1, 0) + g);
+                    float s1 = 0.f, s2 = 0.f;
+                    for (int i = 0; i < n; ++i) {
+                        const float dv = __fsub_rn(E::load1(cp(1, i) + g), x0);
+                        s1 = __fadd_rn(s1, dv);
+                        s2 = __fmaf_rn(dv, dv, s2);
+                    }
+                    ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1, inv_n), s1, s2));
                 }
-            }
-            // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
-            if (active && (G == 1 || g == 0)) {
+            } else if (active) {
+                // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
                 const float s1[4] = {s1a.x, s1a.y, s1b.x, s1b.y}, s2[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
 #pragma unroll
                 for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
@@ -608,48 +636,30 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
 }
 
 template <int MODE>
-void *kernel_ptr(int storage, bool dense) {
-    // dense mixing exists for bf16 only, and not for Eq. 2
+void *kernel_ptr(int storage, bool dense, bool narrow) {
+    // dense mixing exists for bf16 only, and not for Eq. 2; narrow tiles only
+    // without it (more than 16 workers)
     constexpr bool kCanDense = MODE != kOutEq2;
-    if (storage != kStoreBF16) return reinterpret_cast<void *>(gossip_kernel<MODE, float, false>);
-    if (dense && kCanDense) return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, kCanDense>);
-    return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, false>);
+    if (narrow)
+        return storage == kStoreBF16 ? reinterpret_cast<void *>(gossip_kernel<MODE, bf16, false, true>)
+                                     : reinterpret_cast<void *>(gossip_kernel<MODE, float, false, true>);
+    if (storage != kStoreBF16) return reinterpret_cast<void *>(gossip_kernel<MODE, float, false, false>);
+    if (dense && kCanDense) return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, kCanDense, false>);
+    return reinterpret_cast<void *>(gossip_kernel<MODE, bf16, false, false>);
 }
 
-void *mode_kernel(int mode, int storage, bool dense) {
+void *mode_kernel(int mode, int storage, bool dense, bool narrow) {
     switch (mode) {
-    case kOutSgd: return kernel_ptr<kOutSgd>(storage, dense);
-    case kOutSgdm: return kernel_ptr<kOutSgdm>(storage, dense);
-    case kOutNesterov: return kernel_ptr<kOutNesterov>(storage, dense);
-    case kOutEq2: return kernel_ptr<kOutEq2>(storage, false);
-    case kOutDadam: return kernel_ptr<kOutDadam>(storage, dense);
-    default: return kernel_ptr<kOutLocalDadam>(storage, dense);
+    case kOutSgd: return kernel_ptr<kOutSgd>(storage, dense, narrow);
+    case kOutSgdm: return kernel_ptr<kOutSgdm>(storage, dense, narrow);
+    case kOutNesterov: return kernel_ptr<kOutNesterov>(storage, dense, narrow);
+    case kOutEq2: return kernel_ptr<kOutEq2>(storage, false, narrow);
+    case kOutDadam: return kernel_ptr<kOutDadam>(storage, dense, narrow);
+    default: return kernel_ptr<kOutLocalDadam>(storage, dense, narrow);
     }
 }
 
 int mode_rows(int mode) { return (mode == kOutSgd || mode == kOutDadam) ? 2 : 3; }
-
-template <typename T, bool D>
-void launch_td(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
-    switch (a.mode) {
-    case kOutSgd: gossip_kernel<kOutSgd, T, D><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutSgdm: gossip_kernel<kOutSgdm, T, D><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutNesterov: gossip_kernel<kOutNesterov, T, D><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutEq2: gossip_kernel<kOutEq2, T, false><<<grid, kThreads, smem, s>>>(a); break;
-    case kOutDadam: gossip_kernel<kOutDadam, T, D><<<grid, kThreads, smem, s>>>(a); break;
-    default: gossip_kernel<kOutLocalDadam, T, D><<<grid, kThreads, smem, s>>>(a); break;
-    }
-}
-template <typename T>
-void launch_t(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
-    if constexpr (std::is_same<T, bf16>::value) {
-        if (a.dense) {
-            launch_td<T, true>(a, grid, smem, s);
-            return;
-        }
-    }
-    launch_td<T, false>(a, grid, smem, s);
-}
 
 }  // namespace
 
@@ -661,8 +671,8 @@ GossipShape gossip_shape(int n, int mode, int storage) {
     // bytes, is issue-bound and loses the extra consensus-error pass (65%
     // against 70%).  Up to 4 workers one thread per column (the 4-worker
     // ring: 0.51 of the copy peak against 0.48 with two, 0.36 with four).
-    // From 9 to 16 workers two threads per column, above four.
-    sh.groups = n <= 4 ? 1 : (n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : 4));
+    // From 9 to 16 workers two threads per column, above eight (kGroupsMany: 128-element tiles).
+    sh.groups = n <= 4 ? 1 : (n <= 8 ? (storage == kStoreBF16 ? 1 : 2) : (n <= 16 ? 2 : kGroupsMany));
     // Dense mixing (every row of the column widened once, then w_ij * s_j
     // over all j with w_ij = 0 off the graph) for bf16 with one thread per
     // column: the 8-worker exponential graph's gossip went from 0.885 to 1.006
@@ -692,8 +702,8 @@ GossipShape gossip_shape(int n, int mode, int storage) {
 cudaError_t gossip_set_smem(size_t smem) {
     for (int st = 0; st <= kStoreBF16; ++st)
         for (int m = 0; m <= kOutLocalDadam; ++m)
-            for (int d = 0; d < 2; ++d) {
-                const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m, st, d != 0),
+            for (int v = 0; v < 3; ++v) {   // neighbour lists, dense, narrow
+                const cudaError_t e = cudaFuncSetAttribute(mode_kernel(m, st, v == 1, v == 2),
                                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                            static_cast<int>(smem));
                 if (e != cudaSuccess) return e;
@@ -701,23 +711,23 @@ cudaError_t gossip_set_smem(size_t smem) {
     return cudaSuccess;
 }
 
-int gossip_blocks_per_sm(int mode, int storage, size_t smem, bool dense) {
+int gossip_blocks_per_sm(int mode, int storage, const GossipShape &sh) {
     int nb = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-            &nb, reinterpret_cast<const void *>(mode_kernel(mode, storage, dense)), kThreads, smem) != cudaSuccess)
+            &nb, reinterpret_cast<const void *>(mode_kernel(mode, storage, sh.dense != 0, sh.tile == 128)), kThreads,
+            sh.smem) != cudaSuccess)
         return 1;
     return nb > 0 ? nb : 1;
 }
 
 cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream_t s) {
     if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups) ||
-        a.tile % kBox != 0 || a.maps == nullptr)
+        (a.tile != 128 && a.tile % kBox != 0) || (a.tile == 128 && a.dense) || a.maps == nullptr)
         return cudaErrorInvalidValue;
-    if (a.storage == kStoreBF16)
-        launch_t<bf16>(a, grid, smem, s);
-    else
-        launch_t<float>(a, grid, smem, s);
-    return cudaGetLastError();
+    void *kernel = mode_kernel(a.mode, a.storage, a.dense != 0, a.tile == 128);
+    void *args[] = {const_cast<GossipArgs *>(&a)};
+    const cudaError_t e = cudaLaunchKernel(kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), args, smem, s);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace gasloc

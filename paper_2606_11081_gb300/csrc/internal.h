@@ -192,7 +192,7 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s
 
 // Occupancy-derived persistent grid sizes.
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage);
-int gossip_blocks_per_sm(int mode, int storage, size_t smem, bool dense);
+int gossip_blocks_per_sm(int mode, int storage, const GossipShape &shape);
 int ce_blocks_per_sm(int block, int storage);
 cudaError_t gossip_set_smem(size_t smem);
 
