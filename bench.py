@@ -255,7 +255,7 @@ def run_reference(args, w):
               "workers (fp32 oracle, OpenMP over elements)" % (slice_p, w.n_workers))
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * el / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic", "config": workload_config(w, args),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": orc.lib.oc_num_threads(),
                              "kind": "oracle", "sample": sample},
@@ -576,7 +576,8 @@ def main():
                                       (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / NOMINAL_HBM_GBS}},
             "graph": {"ms_per_step": graph_ms, "value": units / (graph_ms * K / 1e3),
                       "note": "the same rounds through gasloc_run (one captured round replayed), "
-                              "timed after the main measurement; this GPU's replica set"},
+                              "timed after the main measurement; this GPU's parameters (its range when "
+                              "the replicas are split over GPUs)"},
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clk,
             "consensus_error": ce,
         }
