@@ -286,15 +286,17 @@ def workload_config(w, args, world=1):
             "l2": "inputs larger than L2 (%.1f GB replica state per GPU, no flush)" % state_gb}
 
 
-def adamw_bytes_of(w, steps, es):
+def adamw_bytes_of(w, steps, es, P=None):
     """Algorithmic bytes of every AdamW launch of one round (a launch per
-    sub-step; sub-step s steps the workers with H_i > s)."""
+    sub-step; sub-step s steps the workers with H_i > s) over P parameters
+    per replica (default: all of them)."""
+    P = w.n_params if P is None else P
     per_h = bool(w.hp.get("per_worker_h"))
     out = []
     for s in range(max(steps)):
         act = sum(1 for h in steps if h > s)
         if act:
-            out.append(((8 * es * act) if per_h else (7 * es * act + es)) * w.n_params)
+            out.append(((8 * es * act) if per_h else (7 * es * act + es)) * P)
     return out
 
 
@@ -358,7 +360,7 @@ def substep_profile(g, ctx, torch, stream, w, Hi, es, peak, reps=3):
         e1.record(stream)
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / reps
-        b = adamw_bytes_of(w, mask, es)[0]
+        b = adamw_bytes_of(w, mask, es, ctx.P)[0]
         out.append(kernel_entry(b, ms, peak, substep=s + 1, active_workers=act, ms=ms, bytes=b))
     g.gasloc_set_local_steps(ctx.h, Hi)
     ctx.gossip_round()   # back to a round boundary
@@ -485,7 +487,7 @@ def main():
     # algorithmic bytes (of this GPU's range)
     es = 2 if w.hp.get("storage") == "bf16" else 4      # bytes per stored element
     steps = [H] * N if H > 0 else Hi
-    adamw_per_launch = adamw_bytes_of(w, steps, es)
+    adamw_per_launch = adamw_bytes_of(w, steps, es, P)
     adamw_launches = len(adamw_per_launch)
     adamw_bytes = sum(adamw_per_launch)
     gossip_bytes = 5 * es * N * P
@@ -496,7 +498,11 @@ def main():
     dom_gbs = adamw_gbs if dom == "adamw" else gossip_gbs
     dom_bytes_launch = adamw_bytes / adamw_launches if dom == "adamw" else gossip_bytes
     dom_ms_launch = local_ms / K / adamw_launches if dom == "adamw" else gossip_ms / K
-    traffic = kernel_traffic(dom, w.name)
+    def traffic_of(kernel):
+        # a profile is of a launch over all the parameters: this GPU's share
+        t = kernel_traffic(kernel, w.name)
+        return None if t is None else t * P / w.n_params
+    traffic = traffic_of(dom)
 
     # the same rounds replayed from a CUDA graph (gasloc_run)
     graph_ms = measure_graph(ctx, torch, stream, K, H)
@@ -561,13 +567,13 @@ def main():
                                    "ms_per_round": gossip_ms / K, "bytes_per_round": gossip_bytes},
                         "ce": {"gbs": ce_gbs, "frac": ce_gbs / peak, "frac_of_nominal_8tbs": ce_gbs / NOMINAL_HBM_GBS,
                                "ms_per_launch": ce_ms, "bytes_per_launch": ce_bytes,
-                               "traffic": kernel_traffic("ce", w.name),
+                               "traffic": traffic_of("ce"),
                                "note": "standalone reduction (after a direct write of x); each round's "
                                        "value comes fused from the gossip kernel"},
                         "average": {"gbs": avg_gbs, "frac": avg_gbs / peak,
                                     "frac_of_nominal_8tbs": avg_gbs / NOMINAL_HBM_GBS,
                                     "ms_per_launch": avg_ms, "bytes_per_launch": avg_bytes,
-                                    "traffic": kernel_traffic("average", w.name),
+                                    "traffic": traffic_of("average"),
                                     "note": "network average x-bar (end of a run)"},
                         "round": {"bytes": adamw_bytes + gossip_bytes,
                                   "gbs": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9,
