@@ -130,3 +130,62 @@ def test_range_checkpoint_keeps_its_range(tmp_path):
                     c.local_steps(1)
                     c.gossip_round()
             np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
+
+
+def _rank_main(rank, world, port, out, N, P, topo, seed, rounds):
+    import os
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    sys.path.insert(0, root)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    import torch
+    import torch.distributed as dist
+    import bench
+    import paper_2606_11081_gb300 as g
+    from paper_2606_11081_gb300 import workloads as wl
+    torch.cuda.set_device(0)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        hp = dict(wl.COMMON_HP, weights="metropolis", edge_prob=0.5, per_worker_h=True)
+        ctx = g.Context(N, P, topo, seed, hparams=g.make_hparams(**hp), draw_hmax=4,
+                        p_range=bench.shard_range(P, world, rank))
+        ce = torch.zeros(rounds, dtype=torch.float64, device="cuda")
+        for k in range(rounds):
+            ctx.local_steps(g.PER_WORKER_STEPS)
+            ctx.gossip_round()
+            bench.ce_exchange(dist, ctx, ce, k)     # the one exchange of a round
+        torch.cuda.synchronize()
+        out[rank] = (ctx.read_all("x"), ce.cpu().numpy())
+        ctx.close()
+    finally:
+        dist.destroy_process_group()
+
+
+def test_ranks_on_parameter_ranges_with_host_collectives():
+    # Two ranks, each holding one range of the parameters, exchange their
+    # consensus-error shares through bench.ce_exchange (the all-reduce of the
+    # multi-GPU bench).  Run here as two processes on this one GPU with a
+    # host (gloo) all-reduce: no kernel waits on another process.  Together
+    # they must reproduce one context holding everything.
+    import socket
+    import torch.multiprocessing as mp
+    N, P, topo, seed, rounds = 8, 3 * 4096 + 901, "exp", 61, 3
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    mgr = mp.get_context("spawn").Manager()
+    out = mgr.dict()
+    mp.start_processes(_rank_main, args=(2, port, out, N, P, topo, seed, rounds), nprocs=2, join=True,
+                       start_method="spawn")
+    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True)
+    with _ctx(N, P, topo, seed, hp, draw_hmax=4) as whole:
+        ces = []
+        for _ in range(rounds):
+            whole.local_steps(g.PER_WORKER_STEPS)
+            whole.gossip_round()
+            ces.append(whole.consensus_error())
+        x = whole.read_all("x")
+    np.testing.assert_array_equal(np.concatenate([out[0][0], out[1][0]], axis=1), x)
+    for r in range(2):
+        np.testing.assert_allclose(out[r][1], ces, rtol=1e-12)
