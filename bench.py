@@ -674,9 +674,14 @@ def measure_e2e(g, torch, w, hp, H, K, p_range=None, dist_mod=None):
     out = torch.empty(P, dtype=torch.float32, pin_memory=True)
     ces = torch.zeros(K, dtype=torch.float64, pin_memory=True)
     ce_dev = torch.zeros(K, dtype=torch.float64, device="cuda") if dist_mod else None
-    # untimed warm-up of the host-to-device path (one worker's centre row);
-    # the timed region below uploads everything again
-    g.gasloc_write_ptr(ctx.h, "c", 0, cs[0].data_ptr())
+    # untimed warm-up of the host-to-device path: one upload of every input
+    # (the first transfer from freshly written pinned pages runs slower); the
+    # timed region below uploads everything again
+    g.gasloc_write_ptr(ctx.h, "x", -1, x0.data_ptr())
+    for i in range(N):
+        g.gasloc_write_ptr(ctx.h, "c", i, cs[i].data_ptr())
+    for i in range(nh):
+        g.gasloc_write_ptr(ctx.h, "h", i, hs[i].data_ptr())
     torch.cuda.synchronize()
     if dist_mod:
         dist_mod.barrier()
@@ -724,7 +729,8 @@ def measure_e2e(g, torch, w, hp, H, K, p_range=None, dist_mod=None):
             "d2h_bytes_per_step": d2h / K, "seconds": el,
             "upload_s": t1 - t0, "rounds_s": t2 - t1, "download_s": t3,
             "value_blocking_read": N * P * K / tb,
-            "note": "initial replicas, centres and curvature uploaded once per run (amortised); "
+            "note": "initial replicas, centres and curvature uploaded once per run (amortised, after "
+                    "one untimed upload of the same buffers); "
                     "every round's consensus error copied to pinned host memory without "
                     "blocking, one wait after the last round; average read at the end; "
                     "value_blocking_read: rounds only, waiting for each round's value"}
