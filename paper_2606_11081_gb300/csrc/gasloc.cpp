@@ -48,6 +48,7 @@ constexpr int kTileA = 1024;          // init / adamw / ce / average tiles (4 x 
 constexpr int kMaxLocalSteps = 1024;
 constexpr int kCeRing = 4096;
 constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
+constexpr int kDirectTilesPerCta = 8;   // the direct gossip variant up to this many 1024-element tiles per CTA
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -125,6 +126,7 @@ struct gasloc_ctx {
     int tile_g = 0;
     int grid_a = 0, grid_ce = 0;
     int grid_gm[6] = {0, 0, 0, 0, 0, 0};   // gossip grid per outer mode
+    int grid_gd[6] = {0, 0, 0, 0, 0, 0};   // direct gossip grid per outer mode (0: not used)
     Topo *topo_d = nullptr, *topo_scratch = nullptr;
     void *maps_d = nullptr;   // [tensor][x, y, b] CUtensorMap
     double *partials = nullptr;
@@ -717,6 +719,16 @@ int gasloc_start(gasloc_ctx *c) {
         c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm));
     }
     c->grid_ce = std::min(max_grid, c->sms * ce_blocks_per_sm(256, c->hp.storage));
+    // the direct gossip variant pays where each CTA of the pipelined one
+    // would walk only a few tiles (few workers, a replica store of up to a few
+    // hundred MB): one memory round trip per tile instead of a pipeline that
+    // never fills
+    for (int m = 0; m < 6; ++m) {
+        c->grid_gd[m] = 0;
+        if (!gossip_direct_fits(n, c->hp.storage)) continue;
+        const int gd = std::min(max_grid, c->sms * gossip_direct_blocks_per_sm(m));
+        if (c->ntiles_a <= static_cast<int64_t>(kDirectTilesPerCta) * gd) c->grid_gd[m] = gd;
+    }
 
     int rc = upload_schedule(c);
     if (rc) { c->release_all(); return rc; }
@@ -859,6 +871,12 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     a.fresh_mask = c->fresh_mask;
     a.state = c->state_d;
     const GossipShape gs = gossip_shape(c->n, hp.outer_mode, hp.storage);
+    const int grid_direct = c->grid_gd[hp.outer_mode];
+    a.direct = grid_direct > 0 ? 1 : 0;
+    if (a.direct) {
+        a.tiles = c->tiles_a;
+        a.ntiles = c->ntiles_a;
+    }
     a.tile = gs.tile;
     a.groups = gs.groups;
     a.stages = gs.stages;
@@ -874,7 +892,8 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     a.ce_ring = c->ce_ring;
     a.ce_ring_len = kCeRing;
     a.err = c->err_d;
-    const int rc = launch_checked(c, launch_gossip(a, c->grid_gm[hp.outer_mode], gs.smem, s), "gossip kernel");
+    const int rc = launch_checked(c, launch_gossip(a, a.direct ? grid_direct : c->grid_gm[hp.outer_mode], gs.smem, s),
+                                  "gossip kernel");
     if (rc) return rc;
     c->round += 1;
     c->fresh_mask = 0;

@@ -635,6 +635,183 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
     }
 }
 
+// ---------------------------------------------------------------------------
+// Direct variant for few workers and small replicas (n <= kDirectMaxWorkers,
+// fp32, a few 1024-element tiles per CTA).  With a replica store of about a
+// hundred MB each CTA of the pipelined kernel above walks only 3-4 tiles, and
+// every tile pays the whole chain of a stage: TMA load, consumers, release,
+// box stores reading the stage, reload.  Here each thread loads its column of
+// 4 elements for every worker and every row the update needs straight into
+// registers (all loads of the tile issued before any arithmetic), forms every
+// worker's update and stores x and b back: one memory round trip per tile.
+// The arithmetic, its order and the consensus-error terms are those of the
+// kernel above with one thread per column, so the results are bit-identical.
+constexpr int kDirectMaxWorkers = 4;
+constexpr int kDirectThreads = 256;   // a column of 4 elements each: 1024-element tiles
+
+template <int MODE>
+__global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const GossipArgs a) {
+    using R = ModeRows<MODE>;
+    using E = Elem<float>;
+    __shared__ Topo tp;
+    __shared__ double red[kDirectThreads / 32];
+    __shared__ int last;
+    const int n = a.n_workers;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int q = threadIdx.x; q < n * kMaxWorkers; q += blockDim.x) {   // the rows of the table in use
+        const int i = q / kMaxWorkers, c = q % kMaxWorkers;
+        tp.nbr[i][c] = a.topo->nbr[i][c];
+        tp.w[i][c] = a.topo->w[i][c];
+    }
+    if (threadIdx.x < n) tp.deg[threadIdx.x] = a.topo->deg[threadIdx.x];
+    __syncthreads();
+    const int64_t round = __ldcg(&a.state->round);
+    const bool first_round = round == 0;
+    const float inv_n = static_cast<float>(1.0 / n);
+    const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
+                     x2::splat(a.gamma), x2::splat(a.eta)};
+    const uint32_t fresh = a.fresh_mask;
+    double ce_acc = 0.0;
+    const int e0 = 4 * threadIdx.x;
+    int32_t cur = -1;
+    TensorDesc d{};
+    for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
+        const Tile tl = a.tiles[ti];
+        if (e0 >= tl.len) continue;
+        if (tl.tensor != cur) {
+            d = a.tens[tl.tensor];
+            cur = tl.tensor;
+        }
+        const float *X = static_cast<const float *>(d.x), *Y = static_cast<const float *>(d.y);
+        const float *B = static_cast<const float *>(d.b);
+        const int64_t off = tl.start + e0;
+        const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
+        // rows of every worker: kind 0 the mixed quantity, kind 1 own x (own
+        // y in the DAdam modes), kind 2 own b -- as the pipelined kernel stages them
+        float4 rows[R::kRows][kDirectMaxWorkers];
+#pragma unroll
+        for (int j = 0; j < kDirectMaxWorkers; ++j) {
+            if (j >= n || !row_ok(j, n, off, 4, d.wstride, a.err)) {
+#pragma unroll
+                for (int k = 0; k < R::kRows; ++k) rows[k][j] = make_float4(0.f, 0.f, 0.f, 0.f);
+                continue;
+            }
+            const int64_t o = j * d.wstride + off;
+            const bool fr = (fresh >> j) & 1u;
+            const float *k0 = R::kMixX ? X : (fr ? Y : X);
+            const float *k1 = R::kMixX ? (fr ? Y : X) : X;
+            rows[0][j] = E::load4<Cache::kL2>(k0 + o);
+            rows[1][j] = E::load4<Cache::kL2>(k1 + o);
+            if (R::kHasB) rows[R::kRows - 1][j] = E::load4<Cache::kL2>(B + o);
+        }
+        float2 s1a = x2::splat(0.f), s1b = s1a, s2a = s1a, s2b = s1a;
+        float4 sh = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < kDirectMaxWorkers; ++i) {
+            if (i >= n) continue;
+            float2 acc01 = x2::splat(0.f), acc23 = acc01;
+            int dg = tp.deg[i];
+            if (!span_ok(dg, dg + 1, kMaxWorkers, a.err)) dg = -1;
+            for (int q = 0; q <= dg; ++q) {
+                const int j = tp.nbr[i][q];
+                if (!span_ok(j, j + 1, n, a.err)) continue;
+                const float2 w = x2::splat(tp.w[i][q]);
+                float4 sj = rows[0][0];
+#pragma unroll
+                for (int jj = 1; jj < kDirectMaxWorkers; ++jj)   // register select, no dynamic index
+                    if (jj == j) sj = rows[0][jj];
+                float2 s01 = x2::lo(sj), s23 = x2::hi(sj);
+                if (MODE == kOutEq2) {   // z_j = x_j + eta (y_j - x_j)
+                    float4 xj = rows[1][0];
+#pragma unroll
+                    for (int jj = 1; jj < kDirectMaxWorkers; ++jj)
+                        if (jj == j) xj = rows[1][jj];
+                    s01 = x2::fma(ok2.eta, x2::sub(s01, x2::lo(xj)), x2::lo(xj));
+                    s23 = x2::fma(ok2.eta, x2::sub(s23, x2::hi(xj)), x2::hi(xj));
+                }
+                acc01 = x2::fma(w, s01, acc01);
+                acc23 = x2::fma(w, s23, acc23);
+            }
+            float4 xo, yo, zo = make_float4(0.f, 0.f, 0.f, 0.f), bo = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (R::kMixX) {
+                xo = rows[0][i];
+                yo = rows[1][i];
+            } else {
+                xo = rows[1][i];
+                yo = xo;
+            }
+            if (R::kHasB) bo = rows[R::kRows - 1][i];
+            if (MODE == kOutEq2) {
+                const float4 y0 = rows[0][i];
+                zo = x2::join(x2::fma(ok2.eta, x2::sub(x2::lo(y0), x2::lo(xo)), x2::lo(xo)),
+                              x2::fma(ok2.eta, x2::sub(x2::hi(y0), x2::hi(xo)), x2::hi(xo)));
+            }
+            const float4 zp = (MODE == kOutEq2 && first_round) ? zo : bo;
+            float2 b01 = x2::lo(bo), b23 = x2::hi(bo);
+            const float2 n01 = outer_pair<MODE>(acc01, x2::lo(xo), x2::lo(yo), b01, x2::lo(zo), x2::lo(zp), ok2);
+            const float2 n23 = outer_pair<MODE>(acc23, x2::hi(xo), x2::hi(yo), b23, x2::hi(zo), x2::hi(zp), ok2);
+            const float4 xn4 = x2::join(n01, n23), bn4 = x2::join(b01, b23);
+            if (i == 0) sh = xn4;
+            ce_terms(x2::lo(xn4), x2::lo(sh), s1a, s2a);
+            ce_terms(x2::hi(xn4), x2::hi(sh), s1b, s2b);
+            const int64_t o = i * d.wstride + off;
+            if (!row_ok(i, n, off, 4, d.wstride, a.err)) continue;
+            float *Xw = static_cast<float *>(d.x) + o;
+            float *Bw = static_cast<float *>(d.b) + o;
+            if (nvalid == 4) {
+                E::store4<Cache::kL2>(Xw, xn4);
+                if (R::kHasB) E::store4<Cache::kL2>(Bw, bn4);
+            } else {
+                const float xa[4] = {xn4.x, xn4.y, xn4.z, xn4.w}, ba[4] = {bn4.x, bn4.y, bn4.z, bn4.w};
+                for (int l = 0; l < nvalid; ++l) {
+                    Xw[l] = xa[l];
+                    if (R::kHasB) Bw[l] = ba[l];
+                }
+            }
+        }
+        // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
+        const float s1[4] = {s1a.x, s1a.y, s1b.x, s1b.y}, s2[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
+#pragma unroll
+        for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
+            if (l < nvalid) ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
+    }
+    // block reduction, one partial per CTA, the last CTA adds them in CTA order
+    for (int o = 16; o > 0; o >>= 1) ce_acc += __shfl_down_sync(0xffffffffu, ce_acc, o);
+    if (lane == 0) red[warp] = ce_acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double sum = 0.0;
+        for (int w = 0; w < kDirectThreads / 32; ++w) sum += red[w];
+        a.partials[blockIdx.x] = sum;
+        __threadfence();
+        const unsigned t = atomicAdd(a.ticket, 1u);
+        last = (t == gridDim.x - 1) ? 1 : 0;
+    }
+    __syncthreads();
+    if (last && warp == 0) {
+        __threadfence();
+        double sum = 0.0;
+        for (unsigned b = lane; b < gridDim.x; b += 32) sum += __ldcg(a.partials + b);
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_down_sync(0xffffffffu, sum, o);
+        if (lane == 0) {
+            a.ce_ring[round % a.ce_ring_len] = sum / static_cast<double>(n);
+            *a.ticket = 0u;
+            a.state->round = round + 1;
+        }
+    }
+}
+
+void *direct_kernel(int mode) {
+    switch (mode) {
+    case kOutSgd: return reinterpret_cast<void *>(gossip_direct_kernel<kOutSgd>);
+    case kOutSgdm: return reinterpret_cast<void *>(gossip_direct_kernel<kOutSgdm>);
+    case kOutNesterov: return reinterpret_cast<void *>(gossip_direct_kernel<kOutNesterov>);
+    case kOutEq2: return reinterpret_cast<void *>(gossip_direct_kernel<kOutEq2>);
+    case kOutDadam: return reinterpret_cast<void *>(gossip_direct_kernel<kOutDadam>);
+    default: return reinterpret_cast<void *>(gossip_direct_kernel<kOutLocalDadam>);
+    }
+}
+
 template <int MODE>
 void *kernel_ptr(int storage, bool dense, bool narrow) {
     // dense mixing exists for bf16 only, and not for Eq. 2; narrow tiles only
@@ -711,6 +888,16 @@ cudaError_t gossip_set_smem(size_t smem) {
     return cudaSuccess;
 }
 
+int gossip_direct_blocks_per_sm(int mode) {
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, reinterpret_cast<const void *>(direct_kernel(mode)),
+                                                      kDirectThreads, 0) != cudaSuccess)
+        return 1;
+    return nb > 0 ? nb : 1;
+}
+
+bool gossip_direct_fits(int n, int storage) { return storage == kStoreF32 && n <= kDirectMaxWorkers; }
+
 int gossip_blocks_per_sm(int mode, int storage, const GossipShape &sh) {
     int nb = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(
@@ -724,8 +911,14 @@ cudaError_t launch_gossip(const GossipArgs &a, int grid, size_t smem, cudaStream
     if (a.stages < 2 || a.stages > kMaxStages || a.groups < 1 || a.tile != 4 * (kConsumers / a.groups) ||
         (a.tile != 128 && a.tile % kBox != 0) || (a.tile == 128 && a.dense) || a.maps == nullptr)
         return cudaErrorInvalidValue;
-    void *kernel = mode_kernel(a.mode, a.storage, a.dense != 0, a.tile == 128);
     void *args[] = {const_cast<GossipArgs *>(&a)};
+    if (a.direct) {   // a.tiles is then the 1024-element tile table
+        if (a.storage != kStoreF32 || a.n_workers > kDirectMaxWorkers) return cudaErrorInvalidValue;
+        const cudaError_t e = cudaLaunchKernel(direct_kernel(a.mode), dim3(static_cast<unsigned>(grid)),
+                                               dim3(kDirectThreads), args, 0, s);
+        return e != cudaSuccess ? e : cudaGetLastError();
+    }
+    void *kernel = mode_kernel(a.mode, a.storage, a.dense != 0, a.tile == 128);
     const cudaError_t e = cudaLaunchKernel(kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), args, smem, s);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

@@ -138,6 +138,8 @@ struct GossipArgs {
     int32_t groups;        // consumer threads per 16-byte column
     int32_t stages;
     int32_t dense;         // dense mixing variant (GossipShape::dense)
+    int32_t direct;        // the direct variant (few workers, small replicas): tiles is the
+                           // 1024-element tile table
     float eta_out, mu, eta, alpha, oma, gamma;
     double *partials;      // [gridDim] per-CTA consensus-error partials
     unsigned int *ticket;  // last-CTA-done counter (returns to 0)
@@ -193,6 +195,10 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s
 // Occupancy-derived persistent grid sizes.
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage);
 int gossip_blocks_per_sm(int mode, int storage, const GossipShape &shape);
+// The direct gossip variant: whether it serves n workers with this storage,
+// and its CTAs per SM.
+bool gossip_direct_fits(int n, int storage);
+int gossip_direct_blocks_per_sm(int mode);
 int ce_blocks_per_sm(int block, int storage);
 cudaError_t gossip_set_smem(size_t smem);
 

@@ -122,7 +122,8 @@ def test_heterogeneous_steps_per_worker_h():
 MODES = ["nesterov", "sgdm", "sgd", "eq2", "dadam", "local_dadam"]
 GRAPHS = [(8, "exp", {}), (16, "matching", {}), (8, "torus:2x4", {"weights": "metropolis"}),
           (32, "exp", {"weights": "metropolis", "edge_prob": 0.5}), (6, "2peer", {"weights": "lazy"}),
-          (11, "ring", {"per_worker_h": True})]   # own curvature, more than 7 workers: batches of 2 and a tail
+          (11, "ring", {"per_worker_h": True}),   # own curvature, more than 7 workers: batches of 2 and a tail
+          (4, "ring", {}), (3, "matching", {})]   # few workers, small replicas: the direct gossip variant
 
 
 @pytest.mark.parametrize("mode", MODES)
@@ -136,6 +137,23 @@ def test_trajectory_parity(mode, N, topo, kw):
         for r in range(R):
             ctx.local_steps(H)
             st.local_steps(H)
+            ctx.gossip_round()
+            st.gossip_round()
+            assert_ce(ctx.consensus_error(), st)
+        assert_state_equal(ctx, st, ("x", "b", "m", "v"))
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_direct_gossip_with_workers_that_took_no_step(mode):
+    # Few workers and a small replica store take the direct gossip variant;
+    # workers without a local step this round send x, the others y.
+    Hi = np.array([0, 2, 1, 0], np.int32)
+    hp = dict(per_worker_h=True, lr=2e-3, outer=mode, eta=0.9, alpha=0.8, gamma=0.3, noise_sigma=0.02)
+    ctx, st = make_pair(4, 3 * 1024 + 7, "ring", seed=17, hp=hp, Hi=Hi)
+    with ctx:
+        for _ in range(3):
+            ctx.local_steps(g.PER_WORKER_STEPS)
+            st.local_steps(0, Hi)
             ctx.gossip_round()
             st.gossip_round()
             assert_ce(ctx.consensus_error(), st)
