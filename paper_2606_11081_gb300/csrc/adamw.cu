@@ -252,18 +252,23 @@ constexpr int kStagedThreads = kStagedConsumers + 32;
 constexpr int kStagedTile = 4 * kStagedConsumers;   // elements per tile (the host's tile size)
 constexpr uint64_t kStagedWaitNs = 2000000000ull;
 
-template <bool PER_WORKER_H>
+template <typename T, bool PER_WORKER_H>
 struct StagedShape {
-    // Measured on the 8-worker GPT-2-small bf16 workload (fraction of the copy
-    // peak): groups of 4 workers, 2 stages, 3 CTAs per SM 0.931; 3 stages and
-    // 2 CTAs 0.842; groups of 2 with 3 or 4 stages and 3 CTAs 0.853 / 0.856;
-    // single workers, 4 stages, 4 CTAs 0.725.
-    static constexpr int kGroup = PER_WORKER_H ? 3 : 4;           // workers per unit
-    static constexpr int kStages = 2;                             // ring depth
-    static constexpr int kMinBlocks = 3;                          // CTAs per SM
+    // bf16, measured on the 8-worker GPT-2-small bf16 workload (fraction of
+    // the copy peak): groups of 4 workers, 2 stages, 3 CTAs per SM 0.931; 3
+    // stages and 2 CTAs 0.842; groups of 2 with 3 or 4 stages and 3 CTAs
+    // 0.853 / 0.856; single workers, 4 stages, 4 CTAs 0.725.  fp32 (small
+    // replica stores only), measured on the 4-worker 1 Mi ring: groups of 2
+    // workers with 3 stages of 4 KB rows and 2 CTAs per SM 0.781; 2 stages
+    // and 3 CTAs 0.769; single workers, 4 stages 0.727; groups of 4 with 2
+    // stages (one CTA) 0.669; against 0.707 for the register-batched kernel.
+    static constexpr bool kBf = std::is_same<T, bf16>::value;
+    static constexpr int kGroup = kBf ? (PER_WORKER_H ? 3 : 4) : 2;   // workers per unit
+    static constexpr int kStages = kBf ? 2 : 3;                   // ring depth
+    static constexpr int kMinBlocks = kBf ? 3 : 2;                // CTAs per SM
     static constexpr int kArrs = PER_WORKER_H ? 5 : 4;            // rows per worker
     static constexpr int kSegs = kArrs * kGroup + (PER_WORKER_H ? 0 : 1);
-    static constexpr size_t kStageBytes = static_cast<size_t>(kSegs) * kStagedTile * sizeof(bf16);
+    static constexpr size_t kStageBytes = static_cast<size_t>(kSegs) * kStagedTile * sizeof(T);
     static constexpr size_t kBarOffset = kStages * kStageBytes;
     static constexpr size_t kDescOffset = kBarOffset + 2 * kStages * sizeof(uint64_t);
     static constexpr size_t kSmem = kDescOffset + kStages * 64;
@@ -282,12 +287,12 @@ __device__ __forceinline__ void mbar_release(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
 }
 
-template <bool PER_WORKER_H, bool SCHED>
-__global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMinBlocks)
+template <bool PER_WORKER_H, bool SCHED, typename T = bf16>
+__global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::kMinBlocks)
     adamw_staged_kernel(const AdamwArgs a) {
-    using T = bf16;
     using E = Elem<T>;
-    using SS = StagedShape<PER_WORKER_H>;
+    using SS = StagedShape<T, PER_WORKER_H>;
+    constexpr int kVec = 16 / static_cast<int>(sizeof(T));   // elements per 16-byte piece
     constexpr int G = SS::kGroup;
     constexpr int kStages = SS::kStages;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -361,7 +366,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
             const Tile tl = a.tiles[ti];
             const TensorDesc &d = a.tens[tl.tensor];
             const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
-            const int lenr = (tl.len + 7) & ~7;   // whole 16-byte pieces (the row padding is allocated)
+            const int lenr = (tl.len + kVec - 1) / kVec * kVec;   // whole 16-byte pieces (the row padding is allocated)
             const uint32_t bytes = static_cast<uint32_t>(lenr) * sizeof(T);
             const int nsegs = SS::kArrs * nw + (PER_WORKER_H ? 0 : 1);
             if (lane == 0) {
@@ -432,15 +437,16 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
             const int nvalid = u.len - e0 < 4 ? u.len - e0 : 4;
             const uint32_t k0 = static_cast<uint32_t>(u.goff + off);   // global index of the column's first element
             const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
+            using Raw = typename E::Raw;   // 4 elements
             float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (!PER_WORKER_H) hs = E::unpack(*reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * G) + e0));
+            if (!PER_WORKER_H) hs = E::unpack(*reinterpret_cast<const Raw *>(seg(s, SS::kArrs * G) + e0));
 #pragma unroll
             for (int w = 0; w < G; ++w) {
                 if (w >= nw) break;
                 const int i = a.worker[a0 + w];
                 if (!row_ok(i, a.n_workers, off, 4, wstride, a.err)) continue;
-                const uint2 *rw = reinterpret_cast<const uint2 *>(seg(s, SS::kArrs * w) + e0);
-                constexpr int kSegStep = kStagedTile / 4;   // uint2 words per row
+                const Raw *rw = reinterpret_cast<const Raw *>(seg(s, SS::kArrs * w) + e0);
+                constexpr int kSegStep = kStagedTile / 4;   // Raw words per row
                 const float4 Yu = E::unpack(rw[0]), Mu = E::unpack(rw[kSegStep]), Vu = E::unpack(rw[2 * kSegStep]),
                              Cu = E::unpack(rw[3 * kSegStep]);
                 const float4 h4 = PER_WORKER_H ? E::unpack(rw[4 * kSegStep]) : hs;
@@ -448,7 +454,12 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<PER_WORKER_H>::kMi
                 const float2 isb = x2::splat(tab.isb[i]);
                 const float2 dec = SCHED ? x2::splat(tab.decay[i]) : x2::splat(a.decay);
                 float2 m01, v01, m23, v23, xi01, xi23;
-                noise4_pairs(k0, tab.key_lo[i], tab.key_hi[i], xi01, xi23);
+                if constexpr (SS::kBf) {   // 16-bit grid, one hash per element pair
+                    noise4_pairs(k0, tab.key_lo[i], tab.key_hi[i], xi01, xi23);
+                } else {                   // 24-bit grid, one hash per element
+                    xi01 = noise_pair(k0, tab.key_lo[i], tab.key_hi[i]);
+                    xi23 = noise_pair(k0 + 2, tab.key_lo[i], tab.key_hi[i]);
+                }
                 const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4), xi01, nstep,
                                               isb, dec, kc, m01, v01);
                 const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4), xi23, nstep,
@@ -510,17 +521,18 @@ int blocks_per_sm(int block, bool per_worker_h) {
     return a < b ? a : b;
 }
 
-template <bool P, bool S>
+template <bool P, bool S, typename T>
 const void *staged_ptr() {
-    return reinterpret_cast<const void *>(adamw_staged_kernel<P, S>);
+    return reinterpret_cast<const void *>(adamw_staged_kernel<P, S, T>);
 }
 
 // Occupancy of the staged kernel with its shared memory (the attribute is set
 // here, before the first launch).
+template <typename T>
 int staged_blocks_per_sm(bool per_worker_h) {
-    const size_t smem = per_worker_h ? StagedShape<true>::kSmem : StagedShape<false>::kSmem;
-    const void *k[2] = {per_worker_h ? staged_ptr<true, false>() : staged_ptr<false, false>(),
-                        per_worker_h ? staged_ptr<true, true>() : staged_ptr<false, true>()};
+    const size_t smem = per_worker_h ? StagedShape<T, true>::kSmem : StagedShape<T, false>::kSmem;
+    const void *k[2] = {per_worker_h ? staged_ptr<true, false, T>() : staged_ptr<false, false, T>(),
+                        per_worker_h ? staged_ptr<true, true, T>() : staged_ptr<false, true, T>()};
     for (const void *f : k)
         if (cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
             cudaSuccess)
@@ -530,20 +542,21 @@ int staged_blocks_per_sm(bool per_worker_h) {
     return nb > 0 ? nb : 1;
 }
 
+template <typename T>
 void launch_staged(const AdamwArgs &a, int grid, cudaStream_t s) {
     const bool sched = a.lr_steps > 0;
     if (a.per_worker_h) {
-        constexpr size_t m = StagedShape<true>::kSmem;
+        constexpr size_t m = StagedShape<T, true>::kSmem;
         if (sched)
-            adamw_staged_kernel<true, true><<<grid, kStagedThreads, m, s>>>(a);
+            adamw_staged_kernel<true, true, T><<<grid, kStagedThreads, m, s>>>(a);
         else
-            adamw_staged_kernel<true, false><<<grid, kStagedThreads, m, s>>>(a);
+            adamw_staged_kernel<true, false, T><<<grid, kStagedThreads, m, s>>>(a);
     } else {
-        constexpr size_t m = StagedShape<false>::kSmem;
+        constexpr size_t m = StagedShape<T, false>::kSmem;
         if (sched)
-            adamw_staged_kernel<false, true><<<grid, kStagedThreads, m, s>>>(a);
+            adamw_staged_kernel<false, true, T><<<grid, kStagedThreads, m, s>>>(a);
         else
-            adamw_staged_kernel<false, false><<<grid, kStagedThreads, m, s>>>(a);
+            adamw_staged_kernel<false, false, T><<<grid, kStagedThreads, m, s>>>(a);
     }
 }
 
@@ -569,13 +582,17 @@ void launch(const AdamwArgs &a, int grid, cudaStream_t s) {
 }  // namespace
 
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage) {
-    return storage == kStoreBF16 ? staged_blocks_per_sm(per_worker_h) : blocks_per_sm<float>(block, per_worker_h);
+    return storage == kStoreBF16 ? staged_blocks_per_sm<bf16>(per_worker_h) : blocks_per_sm<float>(block, per_worker_h);
 }
+
+int adamw_staged_fp32_blocks_per_sm(bool per_worker_h) { return staged_blocks_per_sm<float>(per_worker_h); }
 
 cudaError_t launch_adamw(const AdamwArgs &a, int grid, int block, cudaStream_t s) {
     (void)block;
     if (a.storage == kStoreBF16)
-        launch_staged(a, grid, s);
+        launch_staged<bf16>(a, grid, s);
+    else if (a.staged)
+        launch_staged<float>(a, grid, s);
     else
         launch<float>(a, grid, s);
     return cudaGetLastError();

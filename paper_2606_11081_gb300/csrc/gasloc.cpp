@@ -49,6 +49,7 @@ constexpr int kMaxLocalSteps = 1024;
 constexpr int kCeRing = 4096;
 constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
 constexpr int kDirectTilesPerCta = 8;   // the direct gossip variant up to this many 1024-element tiles per CTA
+constexpr int kStagedTilesPerCta = 8;   // fp32 stores take the staged AdamW up to this many tiles per CTA
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -125,6 +126,7 @@ struct gasloc_ctx {
     int64_t ntiles_g = 0;
     int tile_g = 0;
     int grid_a = 0, grid_ce = 0;
+    int grid_as = 0;                       // staged fp32 AdamW grid where it is used (0: not)
     int grid_gm[6] = {0, 0, 0, 0, 0, 0};   // gossip grid per outer mode
     int grid_gd[6] = {0, 0, 0, 0, 0, 0};   // direct gossip grid per outer mode (0: not used)
     Topo *topo_d = nullptr, *topo_scratch = nullptr;
@@ -714,6 +716,14 @@ int gasloc_start(gasloc_ctx *c) {
     if (e != cudaSuccess) { c->release_all(); return cuda_fail(e, "table upload"); }
 
     c->grid_a = c->sms * adamw_blocks_per_sm(256, c->hp.per_worker_h != 0, c->hp.storage);
+    // with fp32 storage and a small store (a few tiles per CTA) the staged
+    // AdamW, whose producer warp loads the next unit while the consumers
+    // compute, hides the load latency that is otherwise on every tile's path
+    c->grid_as = 0;
+    if (c->hp.storage == GASLOC_STORAGE_F32) {
+        const int gs = c->sms * adamw_staged_fp32_blocks_per_sm(c->hp.per_worker_h != 0);
+        if (c->ntiles_a <= static_cast<int64_t>(kStagedTilesPerCta) * gs) c->grid_as = gs;
+    }
     for (int m = 0; m < 6; ++m) {
         const GossipShape sm = gossip_shape(n, m, c->hp.storage);
         c->grid_gm[m] = std::min(max_grid, c->sms * gossip_blocks_per_sm(m, c->hp.storage, sm));
@@ -809,6 +819,7 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.tiles = c->tiles_a;
     a.ntiles = c->ntiles_a;
     a.n_workers = c->n;
+    a.staged = c->grid_as > 0 ? 1 : 0;
     a.err = c->err_d;
     a.table = c->table_d;
     a.state = c->state_d;
@@ -841,7 +852,7 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
         a.active_mask = mask;
         a.n_active = na;
         a.from_x_mask = ~c->fresh_mask;
-        const int rc = launch_checked(c, launch_adamw(a, c->grid_a, 256, s), "adamw kernel");
+        const int rc = launch_checked(c, launch_adamw(a, a.staged ? c->grid_as : c->grid_a, 256, s), "adamw kernel");
         if (rc) return rc;
         for (int q = 0; q < na; ++q) c->nsteps[a.worker[q]] += 1;
         c->fresh_mask |= mask;

@@ -120,6 +120,7 @@ struct AdamwArgs {
     float decay;                          // fl32(1 - lr * weight_decay) without a schedule
     float beta1, beta2, omb1, omb2, eps, sigma;
     int32_t n_workers;                    // rows of every per-worker array
+    int32_t staged;                       // fp32: the staged kernel (small replica stores)
     int32_t *err;                         // device error word (checked build)
 };
 
@@ -194,6 +195,8 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, int32_t *err, cudaStream_t s
 
 // Occupancy-derived persistent grid sizes.
 int adamw_blocks_per_sm(int block, bool per_worker_h, int storage);
+// CTAs per SM of the staged AdamW with fp32 storage (used for small stores).
+int adamw_staged_fp32_blocks_per_sm(bool per_worker_h);
 int gossip_blocks_per_sm(int mode, int storage, const GossipShape &shape);
 // The direct gossip variant: whether it serves n workers with this storage,
 // and its CTAs per SM.

@@ -143,6 +143,30 @@ def test_trajectory_parity(mode, N, topo, kw):
         assert_state_equal(ctx, st, ("x", "b", "m", "v"))
 
 
+@pytest.mark.parametrize("N,kw,Hi", [
+    (8, {}, None),                                           # shared h, batches of 4
+    (16, {"lr_total_steps": 6}, None),                       # shared h, batches of 3, lr schedule
+    (5, {"per_worker_h": True}, [2, 0, 1, 2, 1]),            # own h, batches of 3, some workers idle
+    (12, {"per_worker_h": True, "lr_total_steps": 6}, None),  # own h, batches of 2, lr schedule
+])
+def test_register_batched_adamw_on_large_stores(N, kw, Hi):
+    # fp32 stores of a few MB per replica and more take the register-batched
+    # AdamW (small ones the staged kernel, which the other tests here use):
+    # 4 Mi + 333 parameters, every element against the oracle
+    P, R = (1 << 22) + 333, 2
+    hp = dict(kw, lr=2e-3, noise_sigma=0.02)
+    Hi_a = None if Hi is None else np.array(Hi, np.int32)
+    ctx, st = make_pair(N, P, "exp", seed=29, hp=hp, Hi=Hi_a)
+    H = 2 if Hi is None else g.PER_WORKER_STEPS
+    with ctx:
+        for _ in range(R):
+            ctx.local_steps(H)
+            st.local_steps(2 if Hi is None else 0, Hi_a)
+            ctx.gossip_round()
+            st.gossip_round()
+        assert_state_equal(ctx, st, ("x", "y", "m", "v", "b"))
+
+
 @pytest.mark.parametrize("mode", MODES)
 def test_direct_gossip_with_workers_that_took_no_step(mode):
     # Few workers and a small replica store take the direct gossip variant;
