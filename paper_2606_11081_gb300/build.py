@@ -21,7 +21,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 # the same sources with every kernel's index checks compiled in (-DGASLOC_CHECKED)
 LIB_CHECKED = os.path.join(HERE, "libgasloc_checked.so")
 BUILD_DIR_CHECKED = os.path.join(HERE, "_build_checked")
-SOURCES = ["gasloc.cpp", "setup.cu", "adamw.cu", "gossip.cu", "ce.cu", "ce_noalloc.cu"]
+SOURCES = ["gasloc.cpp", "setup.cu", "adamw.cu", "gossip.cu", "round.cu", "ce.cu", "ce_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

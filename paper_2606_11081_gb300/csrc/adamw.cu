@@ -21,20 +21,14 @@
 // there); with half the bytes per element the arithmetic sets the pace, and
 // the consumers must not wait on their own loads.
 //
-// Per element, in fp32 with one IEEE rounding per operation (the oracle's
-// order; pairs of lanes share f32x2 instructions, which round each lane as
-// the scalar operation does); with bf16 storage the loads widen exactly and
-// each stored value is rounded to bf16 (nearest, ties to even):
-//   d = y - c;  t = h d;  g = fma(sigma, xi, t)
-//   y = y * decay
-//   m = fma(beta1, m, (1 - beta1) g)
-//   v = fma(beta2, v, (1 - beta2) (g g))
-//   den = fma(sqrt(v), isb, eps)
-//   y = fma(-step, m / den, y)
+// Per element: the arithmetic of adamw_math.cuh (in fp32, one IEEE rounding
+// per operation); with bf16 storage the loads widen exactly and each stored
+// value is rounded to bf16 (nearest, ties to even).
 #include <cuda_runtime.h>
 
 #include <type_traits>
 
+#include "adamw_math.cuh"
 #include "check.cuh"
 #include "elem.cuh"
 #include "f32x2.cuh"
@@ -54,44 +48,6 @@ constexpr int kBlock = 256;   // threads; a tile is 4 * kBlock elements
 // workload (1.008 against 0.966 of the copy peak) and 2% on the 16-worker one.
 constexpr Cache kLdIterate = Cache::kL2, kLdMoments = Cache::kL2, kLdCentre = Cache::kL2, kLdCurv = Cache::kL2;
 constexpr Cache kSt = Cache::kL2;
-
-// Per-step constants, each in both halves of a register pair.
-struct Consts {
-    float2 b1, b2, omb1, omb2, eps, sigma;
-};
-
-// Two lanes of the step; each paired operation rounds each lane exactly as
-// the scalar operation does (f32x2.cuh), so the sequence is the one above.
-__device__ __forceinline__ float2 adamw_pair(float2 y, float2 m_in, float2 v_in, float2 c, float2 h, float2 xi,
-                                             float2 nstep, float2 isb, float2 decay, const Consts &k,
-                                             float2 &m_out, float2 &v_out) {
-    const float2 d = x2::sub(y, c);
-    const float2 t = x2::mul(h, d);
-    const float2 g = x2::fma(k.sigma, xi, t);
-    y = x2::mul(y, decay);
-    const float2 m = x2::fma(k.b1, m_in, x2::mul(k.omb1, g));
-    const float2 v = x2::fma(k.b2, v_in, x2::mul(k.omb2, x2::mul(g, g)));
-    const float2 den = x2::fma(make_float2(__fsqrt_rn(v.x), __fsqrt_rn(v.y)), isb, k.eps);
-    y = x2::fma(nstep, make_float2(__fdiv_rn(m.x, den.x), __fdiv_rn(m.y, den.y)), y);
-    m_out = m;
-    v_out = v;
-    return y;
-}
-
-// Gradient noise, uniform on [-sqrt3, sqrt3) with unit variance.
-// fp32 storage, 24 bits per element: u = word(k) and
-// xi = ((u >> 8) * 2^-23 - 1) * sqrt3.  (u >> 8) * 2^-23 - 1 equals
-// ((u >> 8) - 2^23) * 2^-23 exactly and sqrt3 * 2^-23 is exact, so
-// xi = fl(((u >> 8) - 2^23) * (sqrt3 * 2^-23)): the same real product rounded
-// once, from one integer conversion.
-__device__ __forceinline__ float noise_int(uint32_t k, uint32_t klo, uint32_t khi) {
-    const uint32_t u = noise_word(k, klo, khi);
-    return __int2float_rn(static_cast<int32_t>(u >> 8) - (1 << 23));
-}
-__device__ __forceinline__ float2 noise_pair(uint32_t k, uint32_t klo, uint32_t khi) {
-    const float scale = static_cast<float>(1.7320508075688772) * 0x1p-23f;
-    return x2::mul(make_float2(noise_int(k, klo, khi), noise_int(k + 1, klo, khi)), x2::splat(scale));
-}
 
 // bf16 storage, 16 bits per element: element 2j takes the low half of
 // word(j), element 2j + 1 the high half, and xi = q * (sqrt3 * 2^-15) with
@@ -144,15 +100,8 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     __syncthreads();
     if (last_copy && threadIdx.x < 32) {
         const int i = threadIdx.x;
-        if (i < a.n_workers && ((a.active_mask >> i) & 1u)) {
-            const int64_t n = a.state->nsteps[i] + 1;
-            const double p1 = __dmul_rn(a.state->p1[i], a.beta1d), p2 = __dmul_rn(a.state->p2[i], a.beta2d);
-            a.state->nsteps[i] = n;
-            a.state->p1[i] = p1;
-            a.state->p2[i] = p2;
-            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d),
-                               lr_of_step(n + 1, a.lr_sched, a.lr_steps, a.lr_after), a.wd, a.seed);
-        }
+        if (i < a.n_workers && ((a.active_mask >> i) & 1u))
+            advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd, a.seed);
         if (i == 0) *a.ticket = 0u;
     }
     int32_t cur = -1;
@@ -321,15 +270,8 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
     __syncthreads();
     if (last_copy && threadIdx.x < 32) {
         const int i = threadIdx.x;
-        if (i < a.n_workers && ((a.active_mask >> i) & 1u)) {
-            const int64_t n = a.state->nsteps[i] + 1;
-            const double p1 = __dmul_rn(a.state->p1[i], a.beta1d), p2 = __dmul_rn(a.state->p2[i], a.beta2d);
-            a.state->nsteps[i] = n;
-            a.state->p1[i] = p1;
-            a.state->p2[i] = p2;
-            write_step_scalars(a.table, i, n + 1, __dmul_rn(p1, a.beta1d), __dmul_rn(p2, a.beta2d),
-                               lr_of_step(n + 1, a.lr_sched, a.lr_steps, a.lr_after), a.wd, a.seed);
-        }
+        if (i < a.n_workers && ((a.active_mask >> i) & 1u))
+            advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd, a.seed);
         if (i == 0) *a.ticket = 0u;
     }
 

@@ -50,6 +50,8 @@ constexpr int kCeRing = 4096;
 constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
 constexpr int kDirectTilesPerCta = 8;   // the direct gossip variant up to this many 1024-element tiles per CTA
 constexpr int kStagedTilesPerCta = 8;   // fp32 stores take the staged AdamW up to this many tiles per CTA
+constexpr int kRoundTile = 256 * kRoundColumn;   // tiles of the fused round kernel
+constexpr int64_t kRoundMaxElems = 8LL * kTileA;  // the fused round up to this many elements per CTA
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
 
@@ -129,6 +131,9 @@ struct gasloc_ctx {
     int grid_as = 0;                       // staged fp32 AdamW grid where it is used (0: not)
     int grid_gm[6] = {0, 0, 0, 0, 0, 0};   // gossip grid per outer mode
     int grid_gd[6] = {0, 0, 0, 0, 0, 0};   // direct gossip grid per outer mode (0: not used)
+    Tile *tiles_r = nullptr;               // tiles of the fused round kernel (where it is used)
+    int64_t ntiles_r = 0;
+    int grid_r[6] = {0, 0, 0, 0, 0, 0};    // fused round grid per outer mode (0: not used)
     Topo *topo_d = nullptr, *topo_scratch = nullptr;
     void *maps_d = nullptr;   // [tensor][x, y, b] CUtensorMap
     double *partials = nullptr;
@@ -655,15 +660,23 @@ int gasloc_start(gasloc_ctx *c) {
             for (int64_t s = 0; s < c->numels[t]; s += tile)
                 v.push_back(Tile{static_cast<int32_t>(t), static_cast<int32_t>(std::min<int64_t>(tile, c->numels[t] - s)), s});
     };
-    std::vector<Tile> ta, tg;
+    std::vector<Tile> ta, tg, tr;
     make_tiles(kTileA, ta);
     make_tiles(c->tile_g, tg);
+    const bool fusable = round_fits(n, c->hp.storage);
+    if (fusable) make_tiles(kRoundTile, tr);
     c->ntiles_a = static_cast<int64_t>(ta.size());
     c->ntiles_g = static_cast<int64_t>(tg.size());
+    c->ntiles_r = static_cast<int64_t>(tr.size());
 
     c->tens_d = static_cast<TensorDesc *>(c->dalloc(sizeof(TensorDesc) * c->tens_h.size()));
     c->tiles_a = static_cast<Tile *>(c->dalloc(sizeof(Tile) * ta.size()));
     c->tiles_g = static_cast<Tile *>(c->dalloc(sizeof(Tile) * tg.size()));
+    c->tiles_r = nullptr;
+    if (fusable) {
+        c->tiles_r = static_cast<Tile *>(c->dalloc(sizeof(Tile) * tr.size()));
+        if (!c->tiles_r) return oom("tables");
+    }
     std::vector<CUtensorMap> maps(c->tens_h.size() * 3);
     for (size_t t = 0; t < c->tens_h.size(); ++t) {
         const TensorDesc &d = c->tens_h[t];
@@ -699,7 +712,9 @@ int gasloc_start(gasloc_ctx *c) {
     }
     DevState st0{};
     for (int i = 0; i < kMaxWorkers; ++i) st0.p1[i] = st0.p2[i] = 1.0;
-    cudaError_t es[8];
+    cudaError_t es[9];
+    es[8] = fusable ? cudaMemcpyAsync(c->tiles_r, tr.data(), sizeof(Tile) * tr.size(), cudaMemcpyHostToDevice, c->stream)
+                    : cudaSuccess;
     es[7] = cudaMemcpyAsync(c->state_d, &st0, sizeof st0, cudaMemcpyHostToDevice, c->stream);
     es[6] = cudaMemcpyAsync(c->maps_d, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice,
                             c->stream);
@@ -738,6 +753,14 @@ int gasloc_start(gasloc_ctx *c) {
         if (!gossip_direct_fits(n, c->hp.storage)) continue;
         const int gd = std::min(max_grid, c->sms * gossip_direct_blocks_per_sm(m));
         if (c->ntiles_a <= static_cast<int64_t>(kDirectTilesPerCta) * gd) c->grid_gd[m] = gd;
+    }
+    // the fused round (gasloc_outer_round, gasloc_run) for the same small stores:
+    // both separate kernels are bound by their ramp and tail there
+    for (int m = 0; m < 6; ++m) {
+        c->grid_r[m] = 0;
+        if (!fusable) continue;
+        const int gr = std::min(max_grid, c->sms * round_blocks_per_sm(m, c->hp.per_worker_h != 0));
+        if (c->P <= kRoundMaxElems * gr) c->grid_r[m] = gr;
     }
 
     int rc = upload_schedule(c);
@@ -912,6 +935,85 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     return GASLOC_OK;
 }
 
+// Enqueues one whole round: H local steps, then the gossip round.  Where the
+// fused round kernel serves the store and every worker takes the round's last
+// step from the same iterate (all from x, or all from y), the first H - 1
+// steps are AdamW launches and the last step runs fused with the gossip
+// round; otherwise the round is enqueued as the two calls would enqueue it.
+// The results are the same either way, bit for bit.
+int enqueue_round(gasloc_ctx *c, int32_t H, cudaStream_t s) {
+    const gasloc_hparams &hp = c->hp;
+    int32_t Hu = H;   // the workers' common step count (-1: they differ)
+    if (H == GASLOC_PER_WORKER_STEPS) {
+        Hu = c->Hi[0];
+        for (int32_t i = 1; i < c->n; ++i)
+            if (c->Hi[i] != Hu) Hu = -1;
+    }
+    const uint32_t all = c->n == 32 ? 0xffffffffu : (1u << c->n) - 1u;
+    const int grid = c->grid_r[hp.outer_mode];
+    const bool fuse = grid > 0 && Hu >= 1 && (Hu >= 2 || c->fresh_mask == 0 || c->fresh_mask == all);
+    int rc;
+    if (!fuse) {
+        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, s);
+        return rc ? rc : enqueue_gossip(c, s);
+    }
+    if (Hu > 1) {
+        rc = enqueue_local_steps(c, Hu - 1, s);
+        if (rc) return rc;
+    }
+    rc = refresh_step_table(c, s);
+    if (rc) return rc;
+    if (!c->topo_static || !c->topo_ready) {
+        rc = build_topology(c, c->round, &c->state_d->round, c->topo_d, s);
+        if (rc) return rc;
+        c->topo_ready = c->topo_static;
+    }
+    RoundArgs a{};
+    a.tens = c->tens_d;
+    a.tiles = c->tiles_r;
+    a.ntiles = c->ntiles_r;
+    a.table = c->table_d;
+    a.state = c->state_d;
+    a.topo = c->topo_d;
+    a.beta1d = hp.beta1;
+    a.beta2d = hp.beta2;
+    a.wd = hp.weight_decay;
+    a.lr_sched = c->lr_sched_d;
+    a.lr_steps = c->lr_steps;
+    a.lr_after = c->lr_after;
+    a.seed = c->seed;
+    a.n_workers = c->n;
+    a.mode = hp.outer_mode;
+    a.per_worker_h = hp.per_worker_h;
+    a.from_x = c->fresh_mask == 0 ? 1 : 0;
+    a.sched = c->lr_steps > 0 ? 1 : 0;
+    a.decay = static_cast<float>(1.0 - hp.lr * hp.weight_decay);
+    a.beta1 = static_cast<float>(hp.beta1);
+    a.beta2 = static_cast<float>(hp.beta2);
+    a.omb1 = static_cast<float>(1.0 - hp.beta1);
+    a.omb2 = static_cast<float>(1.0 - hp.beta2);
+    a.eps = static_cast<float>(hp.eps);
+    a.sigma = static_cast<float>(hp.noise_sigma);
+    a.eta_out = static_cast<float>(hp.outer_lr);
+    a.mu = static_cast<float>(hp.outer_momentum);
+    a.eta = static_cast<float>(hp.eta);
+    a.alpha = static_cast<float>(hp.alpha);
+    a.oma = static_cast<float>(1.0 - hp.alpha);
+    a.gamma = static_cast<float>(hp.gamma);
+    a.partials = c->partials;
+    a.ticket = c->ticket;
+    a.ce_ring = c->ce_ring;
+    a.ce_ring_len = kCeRing;
+    a.err = c->err_d;
+    rc = launch_checked(c, launch_round(a, grid, s), "round kernel");
+    if (rc) return rc;
+    for (int32_t i = 0; i < c->n; ++i) c->nsteps[i] += 1;
+    c->round += 1;
+    c->fresh_mask = 0;
+    c->ce_valid = true;
+    return GASLOC_OK;
+}
+
 int check_H(const gasloc_ctx *c, int32_t H) {
     if (H != GASLOC_PER_WORKER_STEPS && (H < 0 || H > kMaxLocalSteps))
         return fail(GASLOC_EINVAL, "H must be in [0, %d] or GASLOC_PER_WORKER_STEPS", kMaxLocalSteps);
@@ -938,6 +1040,15 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     const int rc = check_started(c);
     if (rc) return rc;
     return enqueue_gossip(c, c->stream);
+}
+
+int gasloc_outer_round(gasloc_ctx *c, int32_t H) {
+    NvtxRange r("gasloc_outer_round");
+    int rc = check_started(c);
+    if (rc) return rc;
+    rc = check_H(c, H);
+    if (rc) return rc;
+    return enqueue_round(c, H, c->stream);
 }
 
 int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) {
@@ -976,8 +1087,7 @@ int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) 
         const bool ce0 = c->ce_valid;
         e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
         if (e != cudaSuccess) return cuda_fail(e, "begin capture");
-        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, c->cap_stream);
-        if (!rc) rc = enqueue_gossip(c, c->cap_stream);
+        rc = enqueue_round(c, H, c->cap_stream);
         cudaGraph_t g = nullptr;
         const cudaError_t e2 = cudaStreamEndCapture(c->cap_stream, &g);
         c->graph_launches = c->launches - launches0;

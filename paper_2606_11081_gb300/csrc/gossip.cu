@@ -50,14 +50,13 @@
 #include "elem.cuh"
 #include "f32x2.cuh"
 #include "internal.h"
+#include "mix.cuh"
 #include "ptx.cuh"
 
 namespace gasloc {
 
 namespace {
 
-constexpr int kOutSgd = 0, kOutSgdm = 1, kOutNesterov = 2, kOutEq2 = 3, kOutDadam = 4,
-              kOutLocalDadam = 5;
 constexpr int kConsumers = 256;                      // 8 warps
 constexpr int kThreads = kConsumers + 32;            // + producer warp
 constexpr int kMaxStages = 4;
@@ -76,54 +75,6 @@ constexpr int kBox = 256;                            // elements per TMA box row
 // room for more stages per SM than 96 KB stages would.
 constexpr int kGroupsMany = 8;
 
-// Rows staged per worker: kind 0 = the mixed quantity, kind 1 = own x (own y
-// for the DAdam modes), kind 2 = own b.
-template <int MODE>
-struct ModeRows {
-    static constexpr int kRows = (MODE == kOutSgd || MODE == kOutDadam) ? 2 : 3;
-    static constexpr bool kMixX = MODE == kOutDadam || MODE == kOutLocalDadam;
-    static constexpr bool kHasB = kRows == 3;
-};
-
-// Outer-step constants, each in both halves of a register pair.
-struct OuterK {
-    float2 neta_out, mu, alpha, oma, gamma, eta;
-};
-
-// Two lanes of the outer update (f32x2.cuh: each lane rounds as the scalar
-// operation would).  acc = mixed value, x = own x, y = own y (DAdam modes),
-// b = own b (updated), z / zprev = Eq. 2's z_t and z_{t-1}.
-template <int MODE>
-__device__ __forceinline__ float2 outer_pair(float2 acc, float2 x, float2 y, float2 &b, float2 z, float2 zprev,
-                                             const OuterK &k) {
-    switch (MODE) {
-    case kOutSgd:
-        return x2::fma(k.neta_out, x2::sub(x, acc), x);
-    case kOutSgdm: {
-        const float2 D = x2::sub(x, acc);
-        b = x2::fma(k.mu, b, D);
-        return x2::fma(k.neta_out, b, x);
-    }
-    case kOutNesterov: {
-        const float2 D = x2::sub(x, acc);
-        b = x2::fma(k.mu, b, D);
-        return x2::fma(k.neta_out, x2::fma(k.mu, b, D), x);
-    }
-    case kOutEq2: {
-        const float2 xn = x2::fma(k.alpha, acc, x2::mul(k.oma, z));
-        b = z;
-        return x2::fma(k.gamma, x2::sub(z, zprev), xn);
-    }
-    case kOutDadam:
-        return x2::add(acc, x2::sub(y, x));
-    default: {  // Local-DAdam
-        const float2 D = x2::sub(x, acc);
-        b = x2::fma(k.mu, b, D);
-        return x2::fma(k.neta_out, x2::fma(k.mu, b, D), y);
-    }
-    }
-}
-
 // Lanes at or past nvalid (>= 1) take keep's value.
 __device__ __forceinline__ float4 keep_tail(float4 v, float4 keep, int nvalid) {
     if (nvalid < 2) v.y = keep.y;
@@ -137,13 +88,6 @@ __device__ __forceinline__ float2 load2_smem(const float *p) { return *reinterpr
 __device__ __forceinline__ float2 load2_smem(const bf16 *p) {
     const uint32_t u = *reinterpret_cast<const uint32_t *>(p);
     return make_float2(bf_lo(u), bf_hi(u));
-}
-
-// Consensus-error sums of two lanes: dv = x - shift, s1 += dv, s2 += dv dv.
-__device__ __forceinline__ void ce_terms(float2 x, float2 shift, float2 &s1, float2 &s2) {
-    const float2 dv = x2::sub(x, shift);
-    s1 = x2::add(s1, dv);
-    s2 = x2::fma(dv, dv, s2);
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
@@ -646,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, MODE == kOutEq2 ? 1 : 2) gossip_kern
 // worker's update and stores x and b back: one memory round trip per tile.
 // The arithmetic, its order and the consensus-error terms are those of the
 // kernel above with one thread per column, so the results are bit-identical.
-constexpr int kDirectMaxWorkers = 4;
+constexpr int kDirectMaxWorkers = kColumnWorkers;
 constexpr int kDirectThreads = 256;   // a column of 4 elements each: 1024-element tiles
 
 template <int MODE>
@@ -657,19 +601,12 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
     __shared__ double red[kDirectThreads / 32];
     __shared__ int last;
     const int n = a.n_workers;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int q = threadIdx.x; q < n * kMaxWorkers; q += blockDim.x) {   // the rows of the table in use
-        const int i = q / kMaxWorkers, c = q % kMaxWorkers;
-        tp.nbr[i][c] = a.topo->nbr[i][c];
-        tp.w[i][c] = a.topo->w[i][c];
-    }
-    if (threadIdx.x < n) tp.deg[threadIdx.x] = a.topo->deg[threadIdx.x];
+    copy_topo_rows(a.topo, tp, n);
     __syncthreads();
     const int64_t round = __ldcg(&a.state->round);
-    const bool first_round = round == 0;
-    const float inv_n = static_cast<float>(1.0 / n);
     const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
                      x2::splat(a.gamma), x2::splat(a.eta)};
+    const float inv_n = static_cast<float>(1.0 / n);
     const uint32_t fresh = a.fresh_mask;
     double ce_acc = 0.0;
     const int e0 = 4 * threadIdx.x;
@@ -685,9 +622,7 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
         const float *X = static_cast<const float *>(d.x), *Y = static_cast<const float *>(d.y);
         const float *B = static_cast<const float *>(d.b);
         const int64_t off = tl.start + e0;
-        const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-        // rows of every worker: kind 0 the mixed quantity, kind 1 own x (own
-        // y in the DAdam modes), kind 2 own b -- as the pipelined kernel stages them
+        // all loads of the tile issued before any arithmetic
         float4 rows[R::kRows][kDirectMaxWorkers];
 #pragma unroll
         for (int j = 0; j < kDirectMaxWorkers; ++j) {
@@ -704,96 +639,14 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
             rows[1][j] = E::load4<Cache::kL2>(k1 + o);
             if (R::kHasB) rows[R::kRows - 1][j] = E::load4<Cache::kL2>(B + o);
         }
-        float2 s1a = x2::splat(0.f), s1b = s1a, s2a = s1a, s2b = s1a;
-        float4 sh = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int i = 0; i < kDirectMaxWorkers; ++i) {
-            if (i >= n) continue;
-            float2 acc01 = x2::splat(0.f), acc23 = acc01;
-            int dg = tp.deg[i];
-            if (!span_ok(dg, dg + 1, kMaxWorkers, a.err)) dg = -1;
-            for (int q = 0; q <= dg; ++q) {
-                const int j = tp.nbr[i][q];
-                if (!span_ok(j, j + 1, n, a.err)) continue;
-                const float2 w = x2::splat(tp.w[i][q]);
-                float4 sj = rows[0][0];
-#pragma unroll
-                for (int jj = 1; jj < kDirectMaxWorkers; ++jj)   // register select, no dynamic index
-                    if (jj == j) sj = rows[0][jj];
-                float2 s01 = x2::lo(sj), s23 = x2::hi(sj);
-                if (MODE == kOutEq2) {   // z_j = x_j + eta (y_j - x_j)
-                    float4 xj = rows[1][0];
-#pragma unroll
-                    for (int jj = 1; jj < kDirectMaxWorkers; ++jj)
-                        if (jj == j) xj = rows[1][jj];
-                    s01 = x2::fma(ok2.eta, x2::sub(s01, x2::lo(xj)), x2::lo(xj));
-                    s23 = x2::fma(ok2.eta, x2::sub(s23, x2::hi(xj)), x2::hi(xj));
-                }
-                acc01 = x2::fma(w, s01, acc01);
-                acc23 = x2::fma(w, s23, acc23);
-            }
-            float4 xo, yo, zo = make_float4(0.f, 0.f, 0.f, 0.f), bo = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (R::kMixX) {
-                xo = rows[0][i];
-                yo = rows[1][i];
-            } else {
-                xo = rows[1][i];
-                yo = xo;
-            }
-            if (R::kHasB) bo = rows[R::kRows - 1][i];
-            if (MODE == kOutEq2) {
-                const float4 y0 = rows[0][i];
-                zo = x2::join(x2::fma(ok2.eta, x2::sub(x2::lo(y0), x2::lo(xo)), x2::lo(xo)),
-                              x2::fma(ok2.eta, x2::sub(x2::hi(y0), x2::hi(xo)), x2::hi(xo)));
-            }
-            const float4 zp = (MODE == kOutEq2 && first_round) ? zo : bo;
-            float2 b01 = x2::lo(bo), b23 = x2::hi(bo);
-            const float2 n01 = outer_pair<MODE>(acc01, x2::lo(xo), x2::lo(yo), b01, x2::lo(zo), x2::lo(zp), ok2);
-            const float2 n23 = outer_pair<MODE>(acc23, x2::hi(xo), x2::hi(yo), b23, x2::hi(zo), x2::hi(zp), ok2);
-            const float4 xn4 = x2::join(n01, n23), bn4 = x2::join(b01, b23);
-            if (i == 0) sh = xn4;
-            ce_terms(x2::lo(xn4), x2::lo(sh), s1a, s2a);
-            ce_terms(x2::hi(xn4), x2::hi(sh), s1b, s2b);
-            const int64_t o = i * d.wstride + off;
-            if (!row_ok(i, n, off, 4, d.wstride, a.err)) continue;
-            float *Xw = static_cast<float *>(d.x) + o;
-            float *Bw = static_cast<float *>(d.b) + o;
-            if (nvalid == 4) {
-                E::store4<Cache::kL2>(Xw, xn4);
-                if (R::kHasB) E::store4<Cache::kL2>(Bw, bn4);
-            } else {
-                const float xa[4] = {xn4.x, xn4.y, xn4.z, xn4.w}, ba[4] = {bn4.x, bn4.y, bn4.z, bn4.w};
-                for (int l = 0; l < nvalid; ++l) {
-                    Xw[l] = xa[l];
-                    if (R::kHasB) Bw[l] = ba[l];
-                }
-            }
-        }
-        // consensus-error terms of the column: e = S2 - (S1 / n) S1 per element
-        const float s1[4] = {s1a.x, s1a.y, s1b.x, s1b.y}, s2[4] = {s2a.x, s2a.y, s2b.x, s2b.y};
-#pragma unroll
-        for (int l = 0; l < 4; ++l)   // each element's term enters the fp64 sum on its own
-            if (l < nvalid) ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(s1[l], inv_n), s1[l], s2[l]));
+        column_update<MODE, 4>(rows, tp, n, ok2, round == 0, static_cast<float *>(d.x), static_cast<float *>(d.b),
+                               d.wstride, off, tl.len - e0 < 4 ? tl.len - e0 : 4, inv_n, ce_acc, a.err);
     }
-    // block reduction, one partial per CTA, the last CTA adds them in CTA order
-    for (int o = 16; o > 0; o >>= 1) ce_acc += __shfl_down_sync(0xffffffffu, ce_acc, o);
-    if (lane == 0) red[warp] = ce_acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double sum = 0.0;
-        for (int w = 0; w < kDirectThreads / 32; ++w) sum += red[w];
-        a.partials[blockIdx.x] = sum;
-        __threadfence();
-        const unsigned t = atomicAdd(a.ticket, 1u);
-        last = (t == gridDim.x - 1) ? 1 : 0;
-    }
-    __syncthreads();
-    if (last && warp == 0) {
-        __threadfence();
-        double sum = 0.0;
-        for (unsigned b = lane; b < gridDim.x; b += 32) sum += __ldcg(a.partials + b);
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_down_sync(0xffffffffu, sum, o);
-        if (lane == 0) {
+    // one partial per CTA; the last CTA adds them in CTA order, stores the
+    // round's value and advances the round counter
+    if (ce_partial_and_ticket(ce_acc, red, &last, a.partials, a.ticket) && threadIdx.x < 32) {
+        const double sum = ce_sum_partials(a.partials);
+        if (threadIdx.x == 0) {
             a.ce_ring[round % a.ce_ring_len] = sum / static_cast<double>(n);
             *a.ticket = 0u;
             a.state->round = round + 1;

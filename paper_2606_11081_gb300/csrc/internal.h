@@ -149,6 +149,36 @@ struct GossipArgs {
     int32_t *err;
 };
 
+// A round's last local step fused with its gossip round (round.cu): every
+// worker takes the step; few workers, fp32 storage.
+constexpr int kRoundColumn = 2;                  // elements per thread of the fused round kernel
+struct RoundArgs {
+    const TensorDesc *tens;
+    const Tile *tiles;                    // tiles of 256 * kRoundColumn elements
+    int64_t ntiles;
+    StepTable *table;                     // this step's scalars; the next step's on return
+    DevState *state;                      // step counters and round, advanced by the last CTA
+    const Topo *topo;
+    double beta1d, beta2d, wd;            // for the next step's scalars
+    const double *lr_sched;               // lr of local steps 1..lr_steps
+    int64_t lr_steps;
+    double lr_after;                      // lr of later steps
+    uint64_t seed;
+    int32_t n_workers;
+    int32_t mode;                         // GASLOC_OUTER_*
+    int32_t per_worker_h;
+    int32_t from_x;                       // every worker's step starts from x (its first of the round)
+    int32_t sched;                        // the weight-decay factor comes from the step table
+    float decay;                          // fl32(1 - lr * weight_decay) without a schedule
+    float beta1, beta2, omb1, omb2, eps, sigma;
+    float eta_out, mu, eta, alpha, oma, gamma;
+    double *partials;                     // [gridDim] per-CTA consensus-error partials
+    unsigned int *ticket;                 // last-CTA-done counter (returns to 0)
+    double *ce_ring;                      // consensus error of round t goes to ce_ring[t % ring]
+    int32_t ce_ring_len;
+    int32_t *err;                         // device error word (checked build)
+};
+
 struct CeArgs {
     const TensorDesc *tens;
     const Tile *tiles;
@@ -178,6 +208,11 @@ struct GossipShape {
 };
 GossipShape gossip_shape(int n, int mode, int storage);
 cudaError_t launch_ce(const CeArgs &a, int grid, int block, cudaStream_t s);
+// The fused round kernel: whether it serves n workers with this storage, its
+// CTAs per SM, and its launch.
+bool round_fits(int n, int storage);
+int round_blocks_per_sm(int mode, bool per_worker_h);
+cudaError_t launch_round(const RoundArgs &a, int grid, cudaStream_t s);
 cudaError_t launch_average(const TensorDesc *tens, const Tile *tiles, int64_t ntiles,
                            int32_t n_workers, int32_t storage, float *dst, int64_t n_params, int32_t *err,
                            int grid, cudaStream_t s);

@@ -31,4 +31,18 @@ __device__ __forceinline__ void write_step_scalars(StepTable *t, int i, int64_t 
     t->key_hi[i] = static_cast<uint32_t>(key >> 32);
 }
 
+// Worker i has taken a local step: its counters advance (n, beta1^n,
+// beta2^n) and its next step's scalars are written to the table.
+__device__ __forceinline__ void advance_step(DevState *st, StepTable *t, int i, double beta1, double beta2,
+                                             const double *lr_sched, int64_t lr_steps, double lr_after, double wd,
+                                             uint64_t seed) {
+    const int64_t n = st->nsteps[i] + 1;
+    const double p1 = __dmul_rn(st->p1[i], beta1), p2 = __dmul_rn(st->p2[i], beta2);
+    st->nsteps[i] = n;
+    st->p1[i] = p1;
+    st->p2[i] = p2;
+    write_step_scalars(t, i, n + 1, __dmul_rn(p1, beta1), __dmul_rn(p2, beta2),
+                       lr_of_step(n + 1, lr_sched, lr_steps, lr_after), wd, seed);
+}
+
 }  // namespace gasloc

@@ -62,7 +62,7 @@ def test_checked_build_reports_a_failing_check(checked_lib):
 def test_parity_suites_under_index_checks(checked_lib):
     suites = ["tests/test_gpu_parity.py", "tests/test_gpu_bf16.py", "tests/test_gpu_run.py",
               "tests/test_gpu_failure.py", "tests/test_gpu_properties.py", "tests/test_gpu_fullsize.py",
-              "tests/test_zz_no_alloc.py"]
+              "tests/test_gpu_round.py", "tests/test_zz_no_alloc.py"]
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-m", "gpu", "-p", "no:cacheprovider"] + suites,
                        env=_env(checked_lib), cwd=ROOT, capture_output=True, text=True, timeout=1200)
     assert r.returncode == 0, r.stdout[-4000:] + r.stderr[-2000:]
