@@ -50,7 +50,6 @@ constexpr int kCeRing = 4096;
 constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
 constexpr int kDirectTilesPerCta = 8;   // the direct gossip variant up to this many 1024-element tiles per CTA
 constexpr int kStagedTilesPerCta = 8;   // fp32 stores take the staged AdamW up to this many tiles per CTA
-constexpr int kRoundTile = 256 * kRoundColumn;   // tiles of the fused round kernel
 constexpr int64_t kRoundMaxElems = 8LL * kTileA;  // the fused round up to this many elements per CTA
 
 int64_t round_up(int64_t v, int64_t m) { return (v + m - 1) / m * m; }
@@ -1002,6 +1001,7 @@ int enqueue_round(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.gamma = static_cast<float>(hp.gamma);
     a.partials = c->partials;
     a.ticket = c->ticket;
+    a.step_ticket = c->ticket + 1;   // the AdamW launches' slot
     a.ce_ring = c->ce_ring;
     a.ce_ring_len = kCeRing;
     a.err = c->err_d;

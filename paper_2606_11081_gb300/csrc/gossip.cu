@@ -601,7 +601,7 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
     __shared__ double red[kDirectThreads / 32];
     __shared__ int last;
     const int n = a.n_workers;
-    copy_topo_rows(a.topo, tp, n);
+    copy_topo_rows(a.topo, tp, n, blockDim.x);
     __syncthreads();
     const int64_t round = __ldcg(&a.state->round);
     const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),

@@ -151,10 +151,11 @@ struct GossipArgs {
 
 // A round's last local step fused with its gossip round (round.cu): every
 // worker takes the step; few workers, fp32 storage.
-constexpr int kRoundColumn = 2;                  // elements per thread of the fused round kernel
+constexpr int kRoundColumn = 2;                  // elements per consumer thread of the fused round kernel
+constexpr int kRoundTile = 512;                  // elements per tile of the fused round kernel
 struct RoundArgs {
     const TensorDesc *tens;
-    const Tile *tiles;                    // tiles of 256 * kRoundColumn elements
+    const Tile *tiles;                    // tiles of kRoundTile elements
     int64_t ntiles;
     StepTable *table;                     // this step's scalars; the next step's on return
     DevState *state;                      // step counters and round, advanced by the last CTA
@@ -174,6 +175,7 @@ struct RoundArgs {
     float eta_out, mu, eta, alpha, oma, gamma;
     double *partials;                     // [gridDim] per-CTA consensus-error partials
     unsigned int *ticket;                 // last-CTA-done counter (returns to 0)
+    unsigned int *step_ticket;            // CTAs that read the step's scalars (returns to 0)
     double *ce_ring;                      // consensus error of round t goes to ce_ring[t % ring]
     int32_t ce_ring_len;
     int32_t *err;                         // device error word (checked build)

@@ -106,10 +106,10 @@ struct Col<4> {
     static __device__ __forceinline__ void store(float *p, float4 v) { __stcg(reinterpret_cast<float4 *>(p), v); }
 };
 
-// The first n rows of the round's neighbour table into shared memory (all
-// threads of the block take part; the caller synchronises).
-__device__ __forceinline__ void copy_topo_rows(const Topo *src, Topo &tp, int n) {
-    for (int q = threadIdx.x; q < n * kMaxWorkers; q += blockDim.x) {
+// The first n rows of the round's neighbour table into shared memory, by
+// threads 0..nthreads-1 (the caller synchronises them).
+__device__ __forceinline__ void copy_topo_rows(const Topo *src, Topo &tp, int n, int nthreads) {
+    for (int q = threadIdx.x; q < n * kMaxWorkers; q += nthreads) {
         const int i = q / kMaxWorkers, c = q % kMaxWorkers;
         tp.nbr[i][c] = src->nbr[i][c];
         tp.w[i][c] = src->w[i][c];

@@ -20,9 +20,10 @@
 // their ramp and tail rather than by HBM, and one kernel pays those once.
 //
 // The step's per-worker scalars come from the step table; the last CTA to
-// finish (atomic ticket, nothing waits) advances every worker's step counters,
-// writes their next step's scalars, adds the CTAs' consensus-error partials in
-// CTA order, stores the round's value and advances the round counter.
+// have read them (atomic ticket, nothing waits) advances every worker's step
+// counters and writes their next step's scalars while the others work.  The
+// last CTA to finish adds the CTAs' consensus-error partials in CTA order,
+// stores the round's value and advances the round counter.
 #include <cuda_runtime.h>
 
 #include "adamw_math.cuh"
@@ -37,11 +38,13 @@ namespace gasloc {
 
 namespace {
 
-constexpr int kConsumers = 256;                    // 8 warps, a column of kV elements each
-constexpr int kThreads = kConsumers + 32;          // + the producer warp
 constexpr int kV = kRoundColumn;                   // elements per consumer thread
-constexpr int kTile = kConsumers * kV;             // elements per tile
+constexpr int kTile = kRoundTile;                  // elements per tile
+constexpr int kConsumers = kTile / kV;             // a column of kV elements each
+constexpr int kThreads = kConsumers + 32;          // + the producer warp
 constexpr int kStages = 2;
+constexpr int kMinBlocks = 2;                      // CTAs per SM
+static_assert(kConsumers % 32 == 0 && kConsumers * kV == kTile, "whole warps of consumers");
 constexpr uint64_t kWaitNs = 2000000000ull;
 
 // Rows of a tile in a stage: per worker (slot j * kPer + kind) the iterate
@@ -72,12 +75,17 @@ struct TileDesc {
 };
 static_assert(sizeof(TileDesc) <= 128, "one 128-byte slot per stage");
 
+// Barrier of the consumer warps only (the producer does not take part).
+__device__ __forceinline__ void consumer_sync() {
+    asm volatile("barrier.sync 1, %0;" ::"r"(kConsumers) : "memory");
+}
+
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
 }
 
 template <int MODE, bool PER_WORKER_H, bool FROM_X>
-__global__ void __launch_bounds__(kThreads, 2) round_kernel(const RoundArgs a) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const RoundArgs a) {
     using R = ModeRows<MODE>;
     using RR = Rows<MODE, PER_WORKER_H, FROM_X>;
     using C = Col<kV>;
@@ -92,18 +100,9 @@ __global__ void __launch_bounds__(kThreads, 2) round_kernel(const RoundArgs a) {
     __shared__ float s_nstep[kColumnWorkers], s_isb[kColumnWorkers], s_dec[kColumnWorkers];
     __shared__ uint32_t s_klo[kColumnWorkers], s_khi[kColumnWorkers];
     __shared__ double red[kThreads / 32];
-    __shared__ int last;
+    __shared__ int last, last_copy;
     __shared__ int abort_flag;
     const int n = a.n_workers;
-    copy_topo_rows(a.topo, tp, n);
-    if (threadIdx.x < n) {   // this step's scalars of worker i
-        const int i = threadIdx.x;
-        s_nstep[i] = -a.table->step[i];
-        s_isb[i] = a.table->isb[i];
-        s_dec[i] = a.sched ? a.table->decay[i] : a.decay;
-        s_klo[i] = a.table->key_lo[i];
-        s_khi[i] = a.table->key_hi[i];
-    }
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&full[s], 1);
@@ -112,8 +111,8 @@ __global__ void __launch_bounds__(kThreads, 2) round_kernel(const RoundArgs a) {
         ptx::fence_mbar_init();
         abort_flag = 0;
     }
-    __syncthreads();
-    const int64_t round = __ldcg(&a.state->round);
+    __syncthreads();   // the producer starts its copies at once; the consumers first read the round's tables
+    const int64_t round = __ldcg(&a.state->round);   // advanced by the last CTA to finish, after every CTA read it
     const int64_t my_n = a.ntiles > blockIdx.x ? (a.ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
     const int lane = threadIdx.x & 31;
     auto slot = [&](int s, int k) { return stages + (static_cast<size_t>(s) * RR::kSlots + k) * kTile; };
@@ -196,6 +195,28 @@ __global__ void __launch_bounds__(kThreads, 2) round_kernel(const RoundArgs a) {
         }
     } else {
         // ------------------------------------------------------------ consumers ---
+        copy_topo_rows(a.topo, tp, n, kConsumers);
+        if (threadIdx.x < n) {   // this step's scalars of worker i
+            const int i = threadIdx.x;
+            s_nstep[i] = -a.table->step[i];
+            s_isb[i] = a.table->isb[i];
+            s_dec[i] = a.sched ? a.table->decay[i] : a.decay;
+            s_klo[i] = a.table->key_lo[i];
+            s_khi[i] = a.table->key_hi[i];
+        }
+        consumer_sync();
+        // The last CTA to have read the step's scalars (atomic ticket; nothing
+        // waits) advances every worker's counters and writes the next step's
+        // scalars, while the other CTAs already work on their tiles.
+        if (threadIdx.x == 0) last_copy = atomicAdd(a.step_ticket, 1u) == gridDim.x - 1u;
+        consumer_sync();
+        if (last_copy && threadIdx.x < 32) {
+            const int i = threadIdx.x;
+            if (i < n)
+                advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd,
+                             a.seed);
+            if (i == 0) *a.step_ticket = 0u;
+        }
         const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
                         x2::splat(a.eps), x2::splat(a.sigma)};
         const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
@@ -267,11 +288,8 @@ __global__ void __launch_bounds__(kThreads, 2) round_kernel(const RoundArgs a) {
     }
 
     if (ce_partial_and_ticket(ce_acc, red, &last, a.partials, a.ticket) && threadIdx.x < 32) {
-        const int i = threadIdx.x;
-        if (i < n)
-            advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd, a.seed);
         const double sum = ce_sum_partials(a.partials);
-        if (i == 0) {
+        if (threadIdx.x == 0) {
             a.ce_ring[round % a.ce_ring_len] = sum / static_cast<double>(n);
             *a.ticket = 0u;
             a.state->round = round + 1;
