@@ -300,26 +300,12 @@ def adamw_bytes_of(w, steps, es, P=None):
     return out
 
 
-def round_bytes_of(w, steps, es, adamw_bytes, gossip_bytes, fused, P=None):
-    """Algorithmic bytes of one round: its AdamW launches and its gossip
-    round, less, where the round's last local step runs fused with the gossip
-    round (gasloc_outer_round), the rows the gossip no longer reads: the new
-    y, and x too when that step started from x (one step per round)."""
-    P = w.n_params if P is None else P
-    if not fused:
-        return adamw_bytes + gossip_bytes
-    saved = (2 if max(steps) == 1 else 1) * es * w.n_workers * P
-    return adamw_bytes + gossip_bytes - saved
-
-
 def time_rounds(ctx, torch, stream, K, H, after_round=None, split=False):
     """K rounds timed with CUDA events on the launch stream; returns (total ms,
     local-step ms, gossip ms), the last two summed over the rounds when
-    `split`.  A round is one gasloc_outer_round call (the round's last local
-    step fused with the gossip round where the store allows); with `split`
-    the local steps and the gossip round are the two calls, with events
-    around each (an event between two kernels keeps the second from starting
-    before the first ends, so the rounds' total is taken without them).
+    `split` (events around the local steps and the gossip round of each
+    round; an event between two kernels keeps the second from starting before
+    the first ends, so the rounds' total is taken without them).
     after_round(k) runs after round k's gossip (the ranks' exchange)."""
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)] if split else None
     t_start = torch.cuda.Event(enable_timing=True)
@@ -328,12 +314,12 @@ def time_rounds(ctx, torch, stream, K, H, after_round=None, split=False):
     for k in range(K):
         if split:
             ev[k][0].record(stream)
-            ctx.local_steps(H)
+        ctx.local_steps(H)
+        if split:
             ev[k][1].record(stream)
-            ctx.gossip_round()
+        ctx.gossip_round()
+        if split:
             ev[k][2].record(stream)
-        else:
-            ctx.outer_round(H)
         if after_round is not None:
             after_round(k)
     t_end.record(stream)
@@ -344,6 +330,41 @@ def time_rounds(ctx, torch, stream, K, H, after_round=None, split=False):
     local_ms = sum(ev[k][0].elapsed_time(ev[k][1]) for k in range(K))
     gossip_ms = sum(ev[k][1].elapsed_time(ev[k][2]) for k in range(K))
     return ms, local_ms, gossip_ms
+
+
+def measure_fused(ctx, torch, stream, K, H, w, steps, es, round_bytes, peak):
+    """The same rounds through gasloc_fused_round, where its fused kernel
+    serves the store (None elsewhere): the round's last local step runs in
+    the gossip kernel, which reads that step's iterate once instead of the
+    local-step kernel writing it and the gossip kernel reading it back.  A
+    labelled variant outside the one-pass-per-step byte model the targets use;
+    its rate is over its own algorithmic bytes (the round's, less the rows the
+    gossip no longer reads: the new y, and x too when the step started from
+    x)."""
+    l0 = ctx.launches
+    ctx.local_steps(H)
+    ctx.gossip_round()
+    l1 = ctx.launches
+    ctx.fused_round(H)
+    if ctx.launches - l1 != (l1 - l0) - 1:   # fused: one launch fewer per round
+        torch.cuda.synchronize()
+        return None
+    for _ in range(2):
+        ctx.fused_round(H)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        ctx.fused_round(H)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / K
+    saved = (2 if max(steps) == 1 else 1) * es * w.n_workers * w.n_params
+    fb = round_bytes - saved
+    return dict(kernel_entry(fb, ms, peak), ms_per_round=ms, bytes=fb,
+                value=float(w.n_workers) * w.n_params / (ms / 1e3),
+                note="gasloc_fused_round: the last local step fused into the gossip kernel; a variant outside "
+                     "the byte model of the targets (one HBM pass per local step), not the measured path")
 
 
 def kernel_entry(bytes_, time_ms, peak, **extra):
@@ -396,19 +417,17 @@ def measure_workload(g, torch, wl, name, K, warmup, peak):
         Hi = g.gasloc_get_local_steps(ctx.h, w.n_workers).tolist() if w.H < 0 else None
         stream = torch.cuda.current_stream()
         for _ in range(warmup):
-            ctx.outer_round(H)
+            ctx.local_steps(H)
+            ctx.gossip_round()
         torch.cuda.synchronize()
-        l0 = ctx.launches
         ms, _, _ = time_rounds(ctx, torch, stream, K, H)
-        l1 = ctx.launches
         ms_split, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H, split=True)
-        fused = (ctx.launches - l1) - (l1 - l0) == K   # one launch fewer per round
         steps = [H] * w.n_workers if H > 0 else Hi
         ab = adamw_bytes_of(w, steps, es)
         gb = 5 * es * w.n_workers * w.n_params
-        rb = round_bytes_of(w, steps, es, sum(ab), gb, fused)
         graph_ms = measure_graph(ctx, torch, stream, K, H)
         units = float(w.n_workers) * w.n_params
+        fused = measure_fused(ctx, torch, stream, K, H, w, steps, es, sum(ab) + gb, peak)
         return {
             "rounds": K, "ms_per_round": ms / K, "value": units * K / (ms / 1e3),
             "ms_per_round_split": ms_split / K,
@@ -416,8 +435,9 @@ def measure_workload(g, torch, wl, name, K, warmup, peak):
             "adamw": kernel_entry(sum(ab), local_ms / K, peak, ms_per_round=local_ms / K,
                                   bytes_per_round=sum(ab), launches_per_round=len(ab)),
             "gossip": kernel_entry(gb, gossip_ms / K, peak, ms_per_round=gossip_ms / K, bytes_per_round=gb),
-            "round": kernel_entry(rb, ms / K, peak, bytes=rb, fused=fused),
+            "round": kernel_entry(sum(ab) + gb, ms / K, peak, bytes=sum(ab) + gb),
             "storage": "bf16" if es == 2 else "f32",
+            "fused_round": fused,
         }
     finally:
         ctx.close()
@@ -473,7 +493,8 @@ def main():
     exchange = (lambda k: ce_exchange(pg, ctx, ce_dev, k)) if pg else None
 
     for k in range(args.warmup):
-        ctx.outer_round(H)
+        ctx.local_steps(H)
+        ctx.gossip_round()
         if exchange:
             exchange(k)
     torch.cuda.synchronize()
@@ -489,9 +510,7 @@ def main():
     launches = ctx.launches - l0
     # the same number of rounds again with events around each kernel, for the
     # kernels' own rates
-    l1 = ctx.launches
     ms_split, local_ms, gossip_ms = time_rounds(ctx, torch, stream, K, H, exchange, split=True)
-    fused = (ctx.launches - l1) - launches == K   # the round's last step ran fused with its gossip
     clk = clocks.stop()
     N, P = w.n_workers, ctx.P        # P: the parameters this GPU holds
     units = float(N) * P * K
@@ -509,7 +528,6 @@ def main():
     adamw_launches = len(adamw_per_launch)
     adamw_bytes = sum(adamw_per_launch)
     gossip_bytes = 5 * es * N * P
-    round_bytes = round_bytes_of(w, steps, es, adamw_bytes, gossip_bytes, fused, P)
     peak, peak_kind = peak_hbm()
     adamw_gbs = adamw_bytes / (local_ms / K / 1e3) / 1e9
     gossip_gbs = gossip_bytes / (gossip_ms / K / 1e3) / 1e9
@@ -594,10 +612,11 @@ def main():
                                     "ms_per_launch": avg_ms, "bytes_per_launch": avg_bytes,
                                     "traffic": traffic_of("average"),
                                     "note": "network average x-bar (end of a run)"},
-                        "round": {"bytes": round_bytes, "fused": fused,
-                                  "gbs": round_bytes / (ms / K / 1e3) / 1e9,
-                                  "frac": round_bytes / (ms / K / 1e3) / 1e9 / peak,
-                                  "frac_of_nominal_8tbs": round_bytes / (ms / K / 1e3) / 1e9 / NOMINAL_HBM_GBS}},
+                        "round": {"bytes": adamw_bytes + gossip_bytes,
+                                  "gbs": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9,
+                                  "frac": (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / peak,
+                                  "frac_of_nominal_8tbs":
+                                      (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / NOMINAL_HBM_GBS}},
             "graph": {"ms_per_step": graph_ms, "value": units / (graph_ms * K / 1e3),
                       "note": "the same rounds through gasloc_run (one captured round replayed), "
                               "timed after the main measurement; this GPU's parameters (its range when "
@@ -714,7 +733,8 @@ def measure_e2e(g, torch, w, hp, H, K, p_range=None, dist_mod=None):
     # round completes; the host waits once, after the last round
     base = ces.data_ptr()
     for k in range(K):
-        ctx.outer_round(H)
+        ctx.local_steps(H)
+        ctx.gossip_round()
         if dist_mod:
             ce_exchange(dist_mod, ctx, ce_dev, k)
             ces[k:k + 1].copy_(ce_dev[k:k + 1], non_blocking=True)
@@ -731,7 +751,8 @@ def measure_e2e(g, torch, w, hp, H, K, p_range=None, dist_mod=None):
     # the same rounds with a blocking read after each one, for comparison
     tb = time.perf_counter()
     for k in range(K):
-        ctx.outer_round(H)
+        ctx.local_steps(H)
+        ctx.gossip_round()
         if dist_mod:
             ce_exchange(dist_mod, ctx, ce_dev, k)
             float(ce_dev[k].item())

@@ -217,23 +217,26 @@ int gasloc_local_steps(gasloc_ctx *ctx, int32_t H);
  * A worker that took no local step this round sends x_i.  Asynchronous. */
 int gasloc_gossip_round(gasloc_ctx *ctx);
 
-/* One complete outer round of Algorithm 1: H local steps (as
+/* One complete outer round of Algorithm 1 -- H local steps (as
  * gasloc_local_steps: H > 0, GASLOC_PER_WORKER_STEPS or 0) followed by a
- * gossip round.  The results are those of gasloc_local_steps(ctx, H) followed
- * by gasloc_gossip_round(ctx), bit for bit.  For a store of at most 4 workers
- * with fp32 storage and up to 8192 parameters per CTA of the GPU's grid
- * (about 2.5 M on a 152-SM GPU), where every worker takes the round's last
- * step from the same iterate (all from x or all from y), that last step runs
- * in one kernel with the gossip round: one pass over the store instead of
- * two.  Asynchronous; EINVAL for H outside [0, 1024] and not
+ * gossip round -- with the round's last local step fused into the gossip
+ * kernel where the store allows: at most 4 workers with fp32 storage, up to
+ * 8192 parameters per CTA of the GPU's grid (about 2.5 M on a 152-SM GPU),
+ * every worker taking that step from the same iterate (all from x or all
+ * from y).  The results are those of gasloc_local_steps(ctx, H) followed by
+ * gasloc_gossip_round(ctx), bit for bit (the consensus error to the rounding
+ * of its fp64 sum order); elsewhere the call enqueues exactly those two.  The
+ * fused kernel reads the round's last iterate once instead of writing it for
+ * the gossip kernel to read back: a variant outside the one-pass-per-step
+ * byte model of the separate kernels, which gasloc_run and the benchmark's
+ * rounds use.  Asynchronous; EINVAL for H outside [0, 1024] and not
  * GASLOC_PER_WORKER_STEPS, ESTATE for GASLOC_PER_WORKER_STEPS without H_i. */
-int gasloc_outer_round(gasloc_ctx *ctx, int32_t H);
+int gasloc_fused_round(gasloc_ctx *ctx, int32_t H);
 
 /* Runs `rounds` complete outer rounds -- H local steps (H > 0, or
  * GASLOC_PER_WORKER_STEPS for each worker's H_i, or 0) followed by a gossip
- * round -- exactly as that many gasloc_outer_round calls (or gasloc_local_steps +
- * gasloc_gossip_round pairs) would, but replayed from a CUDA graph of one
- * round (the launches of gasloc_outer_round) that is captured
+ * round -- exactly as that many gasloc_local_steps + gasloc_gossip_round
+ * calls would, but replayed from a CUDA graph of one round that is captured
  * on the first call and reused until the hyperparameters, H or the H_i
  * change.  Every per-step scalar is derived on the device from device-resident
  * step counters, so the replayed rounds need no host work.  Must start at a

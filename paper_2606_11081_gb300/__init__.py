@@ -74,7 +74,7 @@ SIGNATURES = {
     "gasloc_get_local_steps": (ctypes.c_int, [_P, _I32P]),
     "gasloc_local_steps": (ctypes.c_int, [_P, _I32]),
     "gasloc_gossip_round": (ctypes.c_int, [_P]),
-    "gasloc_outer_round": (ctypes.c_int, [_P, _I32]),
+    "gasloc_fused_round": (ctypes.c_int, [_P, _I32]),
     "gasloc_run": (ctypes.c_int, [_P, _I32, _I32, _DP]),
     "gasloc_consensus_error": (ctypes.c_int, [_P, _DP]),
     "gasloc_consensus_error_now": (ctypes.c_int, [_P, _DP]),
@@ -212,10 +212,11 @@ def gasloc_gossip_round(ctx) -> None:
     _check(_lib.gasloc_gossip_round(ctx))
 
 
-def gasloc_outer_round(ctx, H: int) -> None:
-    """H local steps then a gossip round (the last step fused with the gossip
-    round where the store is small enough)."""
-    _check(_lib.gasloc_outer_round(ctx, H))
+def gasloc_fused_round(ctx, H: int) -> None:
+    """H local steps then a gossip round, the last step fused with the gossip
+    round where the store allows (a variant outside the separate kernels'
+    byte model; gasloc_run and the benchmark use the separate kernels)."""
+    _check(_lib.gasloc_fused_round(ctx, H))
 
 
 def gasloc_run(ctx, rounds: int, H: int, trace: bool = False):
@@ -447,8 +448,8 @@ class Context:
     def gossip_round(self) -> None:
         gasloc_gossip_round(self.h)
 
-    def outer_round(self, H: int) -> None:
-        gasloc_outer_round(self.h, H)
+    def fused_round(self, H: int) -> None:
+        gasloc_fused_round(self.h, H)
 
     def run(self, rounds: int, H: int, trace: bool = False):
         return gasloc_run(self.h, rounds, H, trace)

@@ -215,6 +215,12 @@ struct StagedShape {
     static constexpr int kGroup = kBf ? (PER_WORKER_H ? 3 : 4) : 2;   // workers per unit
     static constexpr int kStages = kBf ? 2 : 3;                   // ring depth
     static constexpr int kMinBlocks = kBf ? 3 : 2;                // CTAs per SM
+    // Units claimed from a global counter (bf16: 0.962 -> 1.025 of the copy
+    // peak on the 8-worker GPT-2-small bf16 workload, whose ~2,000 units per
+    // CTA let slower CTAs fall behind a static split), or a static grid stride
+    // (fp32 small stores: at a few units per CTA the claim's latency cost more,
+    // 0.78 -> 0.72 on the 4-worker 1 Mi ring).
+    static constexpr bool kDynamic = kBf;
     static constexpr int kArrs = PER_WORKER_H ? 5 : 4;            // rows per worker
     static constexpr int kSegs = kArrs * kGroup + (PER_WORKER_H ? 0 : 1);
     static constexpr size_t kStageBytes = static_cast<size_t>(kSegs) * kStagedTile * sizeof(T);
@@ -228,7 +234,8 @@ struct StagedShape {
 struct UnitDesc {
     int64_t start, wstride, goff;   // tile start in the tensor, row stride, global index of element 0
     void *y, *m, *v;
-    int32_t len, pad;
+    int32_t len;                    // elements of the tile; -1: no unit is left (the stage carries no rows)
+    int32_t a0;                     // the unit's first worker slot (index into a.worker)
 };
 static_assert(sizeof(UnitDesc) <= 64, "one 64-byte slot per stage");
 
@@ -276,9 +283,13 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
     }
 
     // units of this CTA: its tiles (grid stride) x the groups of G active workers
+    // units: the tiles x the groups of G active workers (unit u: tile
+    // u / ngroups, group u % ngroups), claimed one at a time from a global
+    // counter by the CTAs' producers where SS::kDynamic (a CTA that drew slower
+    // memory simply claims fewer), else every group of tiles blockIdx.x,
+    // blockIdx.x + gridDim.x, ... in turn
     const int ngroups = (a.n_active + G - 1) / G;
-    const int64_t my_tiles = a.ntiles > blockIdx.x ? (a.ntiles - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
-    const int64_t my_n = my_tiles * ngroups;
+    const int64_t nunits = a.ntiles * ngroups;
     const int lane = threadIdx.x & 31;
     auto seg = [&](int s, int k) {   // row k of stage s
         return stages + (static_cast<size_t>(s) * SS::kSegs + k) * kStagedTile;
@@ -288,7 +299,12 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
         // ---------------------------------------------------------- producer ---
         int64_t issued = 0;
         bool aborted = false;
-        for (int64_t it = 0; it < my_n; ++it) {
+        unsigned long long next = 0;   // the unit claimed for the next stage (lane 0's claim, broadcast)
+        if (SS::kDynamic) {
+            if (lane == 0) next = atomicAdd(a.work, 1ull);
+            next = __shfl_sync(0xffffffffu, next, 0);
+        }
+        for (int64_t it = 0;; ++it) {
             const int s = static_cast<int>(it % kStages);
             if (it >= kStages) {
                 const int64_t j = it - kStages;
@@ -303,8 +319,24 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
                 aborted = true;
                 break;
             }
-            const int64_t ti = blockIdx.x + (it / ngroups) * gridDim.x;
-            const int a0 = static_cast<int>(it % ngroups) * G;
+            const unsigned long long unit =
+                SS::kDynamic ? next
+                             : static_cast<unsigned long long>(blockIdx.x + (it / ngroups) * gridDim.x) * ngroups +
+                                   static_cast<unsigned long long>(it % ngroups);
+            if (unit >= static_cast<unsigned long long>(nunits)) {   // none left: tell the consumers
+                if (lane == 0) {
+                    descs[s].len = -1;
+                    mbar_release(&full[s]);
+                }
+                issued = it + 1;
+                break;
+            }
+            if (SS::kDynamic) {
+                if (lane == 0) next = atomicAdd(a.work, 1ull);   // the next claim, in flight during this unit's copies
+                next = __shfl_sync(0xffffffffu, next, 0);
+            }
+            const int64_t ti = static_cast<int64_t>(unit / ngroups);
+            const int a0 = static_cast<int>(unit % ngroups) * G;
             const Tile tl = a.tiles[ti];
             const TensorDesc &d = a.tens[tl.tensor];
             const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
@@ -322,6 +354,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
                 u.m = d.m;
                 u.v = d.v;
                 u.len = tl.len;
+                u.a0 = a0;
                 ptx::mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsegs) * bytes);
             }
             __syncwarp();
@@ -355,6 +388,15 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
             for (int64_t j = issued - kStages > 0 ? issued - kStages : 0; j < issued; ++j)
                 ptx::mbar_wait_bounded(&full[j % kStages], static_cast<uint32_t>((j / kStages) & 1), kStagedWaitNs);
         }
+        // every producer has made its last claim before it counts itself out;
+        // the last one returns the counter to 0 for the next launch
+        if (SS::kDynamic && lane == 0) {
+            __threadfence();
+            if (atomicAdd(a.work + 1, 1ull) == gridDim.x - 1ull) {
+                atomicExch(a.work, 0ull);
+                atomicExch(a.work + 1, 0ull);
+            }
+        }
         return;
     }
 
@@ -362,17 +404,19 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
     const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
                     x2::splat(a.eps), x2::splat(a.sigma)};
     const int e0 = 4 * threadIdx.x;
-    for (int64_t it = 0; it < my_n; ++it) {
+    for (int64_t it = 0;; ++it) {
         const int s = static_cast<int>(it % kStages);
-        bool ok = abort_flag == 0;
-        if (ok && !ptx::mbar_wait_bounded(&full[s], static_cast<uint32_t>((it / kStages) & 1), kStagedWaitNs)) {
-            ok = false;
+        if (abort_flag != 0 ||
+            !ptx::mbar_wait_bounded(&full[s], static_cast<uint32_t>((it / kStages) & 1), kStagedWaitNs)) {
+            // a failed wait: stop here (the producer's waits are bounded too)
             abort_flag = 1;
             atomicCAS(a.err, static_cast<int32_t>(kDevOk), static_cast<int32_t>(kDevWaitTimeout));
+            break;
         }
-        const int a0 = static_cast<int>(it % ngroups) * G;
         const UnitDesc &u = descs[s];
-        if (ok && e0 < u.len) {
+        if (u.len < 0) break;   // no unit is left
+        const int a0 = u.a0;
+        if (e0 < u.len) {
             T *Yw = as<T>(u.y), *Mw = as<T>(u.m), *Vw = as<T>(u.v);
             const int64_t wstride = u.wstride;
             const int64_t off = u.start + e0;

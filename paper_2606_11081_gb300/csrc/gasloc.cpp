@@ -137,6 +137,7 @@ struct gasloc_ctx {
     void *maps_d = nullptr;   // [tensor][x, y, b] CUtensorMap
     double *partials = nullptr;
     unsigned int *ticket = nullptr;
+    unsigned long long *work = nullptr;   // unit counter of the staged AdamW: [0] claimed, [1] producers done
     double *ce_d = nullptr;          // [0] standalone reduction result
     double *ce_ring = nullptr;       // consensus error of round t at [t % kCeRing]
     DevState *state_d = nullptr;     // device-resident step counters
@@ -693,6 +694,7 @@ int gasloc_start(gasloc_ctx *c) {
     const int max_grid = c->sms * 32;
     c->partials = static_cast<double *>(c->dalloc(sizeof(double) * max_grid));
     c->ticket = static_cast<unsigned int *>(c->dalloc(sizeof(unsigned int) * 4));
+    c->work = static_cast<unsigned long long *>(c->dalloc(sizeof(unsigned long long) * 4));
     c->ce_d = static_cast<double *>(c->dalloc(sizeof(double) * 2));
     c->ce_ring = static_cast<double *>(c->dalloc(sizeof(double) * kCeRing));
     c->state_d = static_cast<DevState *>(c->dalloc(sizeof(DevState)));
@@ -702,6 +704,7 @@ int gasloc_start(gasloc_ctx *c) {
     // a run costs the kernel and the copy only
     c->avg_d = static_cast<float *>(c->dalloc(static_cast<size_t>(c->P) * 4));
     if (!c->tens_d || !c->tiles_a || !c->tiles_g || !c->maps_d || !c->topo_d || !c->topo_scratch || !c->partials || !c->ticket ||
+        !c->work ||
         !c->ce_d || !c->err_d || !c->ce_ring || !c->state_d || !c->table_d || !c->avg_d)
         return oom("tables");
     if (cudaMallocHost(&c->pinned, 64 + sizeof(Topo)) != cudaSuccess) {
@@ -721,6 +724,7 @@ int gasloc_start(gasloc_ctx *c) {
     es[1] = cudaMemcpyAsync(c->tiles_a, ta.data(), sizeof(Tile) * ta.size(), cudaMemcpyHostToDevice, c->stream);
     es[2] = cudaMemcpyAsync(c->tiles_g, tg.data(), sizeof(Tile) * tg.size(), cudaMemcpyHostToDevice, c->stream);
     es[3] = cudaMemsetAsync(c->ticket, 0, sizeof(unsigned int) * 4, c->stream);
+    if (es[3] == cudaSuccess) es[3] = cudaMemsetAsync(c->work, 0, sizeof(unsigned long long) * 4, c->stream);
     es[4] = cudaMemsetAsync(c->err_d, 0, sizeof(int32_t) * 4, c->stream);
     es[5] = cudaMemsetAsync(c->ce_d, 0, sizeof(double) * 2, c->stream);
     for (cudaError_t x : es)
@@ -753,8 +757,7 @@ int gasloc_start(gasloc_ctx *c) {
         const int gd = std::min(max_grid, c->sms * gossip_direct_blocks_per_sm(m));
         if (c->ntiles_a <= static_cast<int64_t>(kDirectTilesPerCta) * gd) c->grid_gd[m] = gd;
     }
-    // the fused round (gasloc_outer_round, gasloc_run) for the same small stores:
-    // both separate kernels are bound by their ramp and tail there
+    // the fused round (gasloc_fused_round) for the same small stores
     for (int m = 0; m < 6; ++m) {
         c->grid_r[m] = 0;
         if (!fusable) continue;
@@ -846,6 +849,7 @@ int enqueue_local_steps(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     a.table = c->table_d;
     a.state = c->state_d;
     a.ticket = c->ticket + 1;   // slot 0: the gossip and consensus-error reductions
+    a.work = c->work;
     a.lr_sched = c->lr_sched_d;
     a.lr_steps = c->lr_steps;
     a.lr_after = c->lr_after;
@@ -934,12 +938,12 @@ int enqueue_gossip(gasloc_ctx *c, cudaStream_t s) {
     return GASLOC_OK;
 }
 
-// Enqueues one whole round: H local steps, then the gossip round.  Where the
-// fused round kernel serves the store and every worker takes the round's last
-// step from the same iterate (all from x, or all from y), the first H - 1
-// steps are AdamW launches and the last step runs fused with the gossip
-// round; otherwise the round is enqueued as the two calls would enqueue it.
-// The results are the same either way, bit for bit.
+// Enqueues one whole round for gasloc_fused_round: H local steps, then the
+// gossip round.  Where the fused round kernel serves the store and every
+// worker takes the round's last step from the same iterate (all from x, or
+// all from y), the first H - 1 steps are AdamW launches and the last step
+// runs fused with the gossip round; otherwise the round is enqueued as the
+// two calls would enqueue it.  The results are the same either way.
 int enqueue_round(gasloc_ctx *c, int32_t H, cudaStream_t s) {
     const gasloc_hparams &hp = c->hp;
     int32_t Hu = H;   // the workers' common step count (-1: they differ)
@@ -1042,8 +1046,8 @@ int gasloc_gossip_round(gasloc_ctx *c) {
     return enqueue_gossip(c, c->stream);
 }
 
-int gasloc_outer_round(gasloc_ctx *c, int32_t H) {
-    NvtxRange r("gasloc_outer_round");
+int gasloc_fused_round(gasloc_ctx *c, int32_t H) {
+    NvtxRange r("gasloc_fused_round");
     int rc = check_started(c);
     if (rc) return rc;
     rc = check_H(c, H);
@@ -1087,7 +1091,8 @@ int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) 
         const bool ce0 = c->ce_valid;
         e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
         if (e != cudaSuccess) return cuda_fail(e, "begin capture");
-        rc = enqueue_round(c, H, c->cap_stream);
+        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, c->cap_stream);
+        if (!rc) rc = enqueue_gossip(c, c->cap_stream);
         cudaGraph_t g = nullptr;
         const cudaError_t e2 = cudaStreamEndCapture(c->cap_stream, &g);
         c->graph_launches = c->launches - launches0;

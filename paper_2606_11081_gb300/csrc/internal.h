@@ -121,6 +121,7 @@ struct AdamwArgs {
     float beta1, beta2, omb1, omb2, eps, sigma;
     int32_t n_workers;                    // rows of every per-worker array
     int32_t staged;                       // fp32: the staged kernel (small replica stores)
+    unsigned long long *work;             // staged kernels: [0] units claimed, [1] producers done (return to 0)
     int32_t *err;                         // device error word (checked build)
 };
 

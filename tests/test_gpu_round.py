@@ -1,4 +1,4 @@
-"""gasloc_outer_round: one whole round of Algorithm 1 (H local steps, then the
+"""gasloc_fused_round: one whole round of Algorithm 1 (H local steps, then the
 gossip round).  For at most 4 workers with fp32 storage and a small store,
 where every worker takes the round's last step from the same iterate, that
 step runs fused with the gossip round in one kernel.  Every step acts on each
@@ -78,7 +78,7 @@ def test_outer_round_equals_the_two_calls(case, mode):
     R = 4
     with _ctx(N, P, topo, 31, hp, numels, Hi_a) as a, _ctx(N, P, topo, 31, hp, numels, Hi_a) as b:
         for r in range(R):
-            a.outer_round(H)
+            a.fused_round(H)
             b.local_steps(H)
             b.gossip_round()
             assert a.consensus_error() == pytest.approx(b.consensus_error(), rel=1e-12, abs=1e-300), r
@@ -91,7 +91,7 @@ def test_outer_round_equals_the_two_calls(case, mode):
         # the rounds go on from the fused state exactly as from the other
         a.local_steps(1)
         a.gossip_round()
-        b.outer_round(1)
+        b.fused_round(1)
         np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
 
 
@@ -101,7 +101,7 @@ def test_outer_round_matches_the_oracle(mode):
     ctx, st = make_pair(N, P, "matching", seed=44, hp=_outer(mode))
     with ctx:
         for _ in range(R):
-            ctx.outer_round(2)
+            ctx.fused_round(2)
             st.local_steps(2)
             st.gossip_round()
             assert_ce(ctx.consensus_error(), st)
@@ -115,7 +115,7 @@ def test_outer_round_in_the_middle_of_a_round():
     with _ctx(4, 3000, "ring", 5, hp) as a, _ctx(4, 3000, "ring", 5, hp) as b:
         for _ in range(2):
             a.local_steps(1)
-            a.outer_round(1)
+            a.fused_round(1)
             b.local_steps(2)
             b.gossip_round()
         for w in ("x", "y", "m", "v", "b"):
@@ -134,7 +134,7 @@ def test_outer_round_on_parameter_ranges():
     try:
         for r in range(3):
             for c in [whole] + parts:
-                c.outer_round(2)
+                c.fused_round(2)
             assert sum(p.consensus_error() for p in parts) == pytest.approx(whole.consensus_error(), rel=1e-12)
         for w in ("x", "y", "m", "v", "b"):
             np.testing.assert_array_equal(np.concatenate([p.read_all(w) for p in parts], axis=1), whole.read_all(w))
@@ -158,7 +158,7 @@ def test_outer_round_ring_full_size():
     st = oracle.get("f32").state(oracle_problem(w.n_workers, P, w.topology, w.seed, full), kidx.astype(np.int64))
     with _ctx(w.n_workers, P, w.topology, w.seed, hp) as a, _ctx(w.n_workers, P, w.topology, w.seed, hp) as b:
         for _ in range(3):
-            a.outer_round(w.H)
+            a.fused_round(w.H)
             b.local_steps(w.H)
             b.gossip_round()
             st.local_steps(w.H)
