@@ -70,20 +70,39 @@ def peak_hbm():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-KERNEL_SOURCE = {"adamw": "adamw.cu", "gossip": "gossip.cu", "ce": "ce.cu", "average": "setup.cu"}
+KERNEL_SOURCE = {"adamw": "adamw.cu", "gossip": "gossip.cu", "ce": "ce.cu", "average": "setup.cu",
+                 "round": "round.cu"}
+CSRC = os.path.join(ROOT, "paper_2606_11081_gb300", "csrc")
+
+
+def source_digest(name: str) -> str:
+    """sha256 over a kernel source file and the local headers it includes,
+    transitively (each file once, in name order): the code a profile of its
+    kernels was taken from."""
+    seen, todo = set(), [name]
+    while todo:
+        f = todo.pop()
+        if f in seen or not os.path.exists(os.path.join(CSRC, f)):
+            continue
+        seen.add(f)
+        text = open(os.path.join(CSRC, f)).read()
+        todo.extend(re.findall(r'^#include "([^"]+)"', text, re.M))
+    h = hashlib.sha256()
+    for f in sorted(seen):
+        h.update(f.encode() + b"\0" + open(os.path.join(CSRC, f), "rb").read())
+    return h.hexdigest()
 
 
 def kernel_traffic(kernel: str, workload: str):
     """DRAM bytes per launch from the committed ncu summary, if the kernel's
-    source file is unchanged since the capture (else None)."""
+    source (its file and the headers it includes) is unchanged since the
+    capture (else None)."""
     prof = os.path.join(ROOT, "profiles", "%s_%s.md" % (kernel, workload))
-    src = os.path.join(ROOT, "paper_2606_11081_gb300", "csrc", KERNEL_SOURCE[kernel])
     try:
         text = open(prof).read()
         m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
         h = re.search(r"source_sha256:\s*([0-9a-f]+)", text)
-        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()
-        if m and h and h.group(1) == cur:
+        if m and h and h.group(1) == source_digest(KERNEL_SOURCE[kernel]):
             return float(m.group(1))
     except Exception:
         pass
@@ -543,6 +562,10 @@ def main():
 
     # the same rounds replayed from a CUDA graph (gasloc_run)
     graph_ms = measure_graph(ctx, torch, stream, K, H)
+    # the labelled fused-round variant, where its kernel serves the store
+    fused = None
+    if N <= 4 and es == 4 and world == 1:
+        fused = measure_fused(ctx, torch, stream, K, H, w, steps, es, adamw_bytes + gossip_bytes, peak)
     # the network average (Algorithm 1's output), timed on its own
     avg_ms = measure_average(g, ctx, torch, stream, P, 5)
     avg_bytes = es * N * P + 4 * P
@@ -621,6 +644,7 @@ def main():
                       "note": "the same rounds through gasloc_run (one captured round replayed), "
                               "timed after the main measurement; this GPU's parameters (its range when "
                               "the replicas are split over GPUs)"},
+            "fused_round": fused,
             "e2e": e2e, "cpu_baseline": cpu, "gpu_launches": launches, "clocks": clk,
             "consensus_error": ce,
         }

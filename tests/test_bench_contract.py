@@ -58,3 +58,31 @@ def test_main_arm_line():
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     assert d["cpu_baseline"]["cores"] >= 1
+
+
+def test_profile_digest_follows_included_headers(tmp_path, monkeypatch):
+    """A profile's traffic counts only while the code it was taken from is
+    unchanged: the kernel file and every local header it includes, however
+    deep, but nothing else."""
+    sys.path.insert(0, ROOT)
+    import bench
+    (tmp_path / "k.cu").write_text('#include "a.cuh"\n#include <cstdio>\nint k;\n')
+    (tmp_path / "a.cuh").write_text('#pragma once\n#include "b.cuh"\n')
+    (tmp_path / "b.cuh").write_text('int b = 1;\n')
+    (tmp_path / "c.cuh").write_text('int c = 1;\n')
+    monkeypatch.setattr(bench, "CSRC", str(tmp_path))
+    d0 = bench.source_digest("k.cu")
+    (tmp_path / "c.cuh").write_text('int c = 2;\n')     # not included
+    assert bench.source_digest("k.cu") == d0
+    (tmp_path / "b.cuh").write_text('int b = 2;\n')     # included through a.cuh
+    d1 = bench.source_digest("k.cu")
+    assert d1 != d0
+    (tmp_path / "k.cu").write_text('#include "a.cuh"\n#include <cstdio>\nint k2;\n')
+    assert bench.source_digest("k.cu") != d1
+
+
+def test_every_profiled_kernel_source_exists():
+    sys.path.insert(0, ROOT)
+    import bench
+    for f in bench.KERNEL_SOURCE.values():
+        assert os.path.exists(os.path.join(bench.CSRC, f)), f
