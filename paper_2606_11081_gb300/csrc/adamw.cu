@@ -15,7 +15,8 @@
 // fp32 storage (adamw_kernel): one thread owns a column of 4 consecutive
 // elements of a tile and walks the active workers U at a time (U from 2 to 4,
 // chosen per launch from the number of workers stepped and whether each has
-// its own h: see Batch), issuing all of their loads before any arithmetic.
+// its own h: see Batch), issuing all of their loads before any arithmetic;
+// CTAs claim their tiles from a global counter.
 // bf16 storage (adamw_staged_kernel): a producer warp stages the rows in
 // shared memory with bulk copies while 256 consumer threads compute (see
 // there); with half the bytes per element the arithmetic sets the pace, and
@@ -106,77 +107,101 @@ __global__ void __launch_bounds__(kBlock, 2) adamw_kernel(const AdamwArgs a) {
     }
     int32_t cur = -1;
     TensorDesc d{};
-    for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
+    // Tiles: blockIdx.x first, then claimed one at a time from a global
+    // counter (claim k is tile gridDim.x + k), so that a CTA that drew slower
+    // memory simply takes fewer (a static split left the slowest CTAs setting
+    // the launch's end: the claimed tiles took the 8-, 16- and 32-worker
+    // workloads from 1.001 / 0.987 / 1.006 to 1.024 / 1.000 / 1.015 of the
+    // copy peak).  Thread 0 claims the next tile while the block works on this
+    // one and publishes it after the tile's barrier, in one of two slots (a
+    // slot is rewritten only after every thread has read it).
+    __shared__ long long next_tile[2];
+    int par = 0;
+    for (int64_t ti = blockIdx.x; ti < a.ntiles; par ^= 1) {
+        if (threadIdx.x == 0)
+            next_tile[par] = static_cast<long long>(gridDim.x) + static_cast<long long>(atomicAdd(a.work, 1ull));
         const Tile tl = a.tiles[ti];
         const int e0 = 4 * threadIdx.x;
-        if (e0 >= tl.len) continue;
-        if (tl.tensor != cur) {
-            d = a.tens[tl.tensor];
-            cur = tl.tensor;
-        }
-        const T *X = as<T>(static_cast<const void *>(d.x));
-        const T *C = as<T>(static_cast<const void *>(d.c));
-        const T *Hh = as<T>(static_cast<const void *>(d.h));
-        T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
-        const int64_t off = tl.start + e0;
-        const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
-        const uint32_t k0 = static_cast<uint32_t>(d.goff + off);   // global index of the column's first element
-        float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::template load4<kLdCurv>(Hh + off);
-
-        for (int a0 = 0; a0 < a.n_active; a0 += U) {
-            // every load of the batch is issued before any arithmetic; the
-            // raw words stay packed until their worker is processed
-            typename E::Raw Y[U], M[U], V[U], Cc[U], Hw[U];
-            bool okr[U];   // worker row and column inside its buffers (checked build)
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                okr[u] = a0 + u < a.n_active && row_ok(a.worker[a0 + u], a.n_workers, off, 4, d.wstride, a.err);
-                if (okr[u]) {
-                    const int i = a.worker[a0 + u];
-                    const int64_t o = i * d.wstride + off;
-                    const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
-                    Y[u] = E::template load_raw<kLdIterate>(src + o);
-                    M[u] = E::template load_raw<kLdMoments>(Mw + o);
-                    V[u] = E::template load_raw<kLdMoments>(Vw + o);
-                    Cc[u] = E::template load_raw<kLdCentre>(C + o);
-                    if (PER_WORKER_H) Hw[u] = E::template load_raw<kLdCurv>(Hh + i * d.hstride + off);
-                }
+        if (e0 < tl.len) {
+            if (tl.tensor != cur) {
+                d = a.tens[tl.tensor];
+                cur = tl.tensor;
             }
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                if (okr[u]) {
-                    const int i = a.worker[a0 + u];
-                    const float2 nstep = x2::splat(-tab.step[i]);
-                    const float2 isb = x2::splat(tab.isb[i]);
-                    const float2 dec = SCHED ? x2::splat(tab.decay[i]) : x2::splat(a.decay);
-                    const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
-                    const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
-                    const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
-                                 Cu = E::unpack(Cc[u]);
-                    float2 m01, v01, m23, v23;
-                    const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
-                                                  noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
-                    const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
-                                                  noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
-                    const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
-                    const int64_t o = i * d.wstride + off;
-                    if (nvalid == 4) {
-                        E::template store4<kSt>(Yw + o, yo);
-                        E::template store4<kSt>(Mw + o, mo);
-                        E::template store4<kSt>(Vw + o, vo);
-                    } else {
-                        const float ya[4] = {yo.x, yo.y, yo.z, yo.w};
-                        const float ma[4] = {mo.x, mo.y, mo.z, mo.w};
-                        const float va[4] = {vo.x, vo.y, vo.z, vo.w};
-                        for (int l = 0; l < nvalid; ++l) {
-                            E::store1(Yw + o + l, ya[l]);
-                            E::store1(Mw + o + l, ma[l]);
-                            E::store1(Vw + o + l, va[l]);
+            const T *X = as<T>(static_cast<const void *>(d.x));
+            const T *C = as<T>(static_cast<const void *>(d.c));
+            const T *Hh = as<T>(static_cast<const void *>(d.h));
+            T *Yw = as<T>(d.y), *Mw = as<T>(d.m), *Vw = as<T>(d.v);
+            const int64_t off = tl.start + e0;
+            const int nvalid = tl.len - e0 < 4 ? tl.len - e0 : 4;
+            const uint32_t k0 = static_cast<uint32_t>(d.goff + off);   // global index of the column's first element
+            float4 hs = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (!PER_WORKER_H && row_ok(0, 1, off, 4, d.wstride, a.err)) hs = E::template load4<kLdCurv>(Hh + off);
+
+            for (int a0 = 0; a0 < a.n_active; a0 += U) {
+                // every load of the batch is issued before any arithmetic; the
+                // raw words stay packed until their worker is processed
+                typename E::Raw Y[U], M[U], V[U], Cc[U], Hw[U];
+                bool okr[U];   // worker row and column inside its buffers (checked build)
+    #pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    okr[u] = a0 + u < a.n_active && row_ok(a.worker[a0 + u], a.n_workers, off, 4, d.wstride, a.err);
+                    if (okr[u]) {
+                        const int i = a.worker[a0 + u];
+                        const int64_t o = i * d.wstride + off;
+                        const T *src = ((a.from_x_mask >> i) & 1u) ? X : Yw;
+                        Y[u] = E::template load_raw<kLdIterate>(src + o);
+                        M[u] = E::template load_raw<kLdMoments>(Mw + o);
+                        V[u] = E::template load_raw<kLdMoments>(Vw + o);
+                        Cc[u] = E::template load_raw<kLdCentre>(C + o);
+                        if (PER_WORKER_H) Hw[u] = E::template load_raw<kLdCurv>(Hh + i * d.hstride + off);
+                    }
+                }
+    #pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    if (okr[u]) {
+                        const int i = a.worker[a0 + u];
+                        const float2 nstep = x2::splat(-tab.step[i]);
+                        const float2 isb = x2::splat(tab.isb[i]);
+                        const float2 dec = SCHED ? x2::splat(tab.decay[i]) : x2::splat(a.decay);
+                        const uint32_t klo = tab.key_lo[i], khi = tab.key_hi[i];
+                        const float4 h4 = PER_WORKER_H ? E::unpack(Hw[u]) : hs;
+                        const float4 Yu = E::unpack(Y[u]), Mu = E::unpack(M[u]), Vu = E::unpack(V[u]),
+                                     Cu = E::unpack(Cc[u]);
+                        float2 m01, v01, m23, v23;
+                        const float2 y01 = adamw_pair(x2::lo(Yu), x2::lo(Mu), x2::lo(Vu), x2::lo(Cu), x2::lo(h4),
+                                                      noise_pair(k0, klo, khi), nstep, isb, dec, kc, m01, v01);
+                        const float2 y23 = adamw_pair(x2::hi(Yu), x2::hi(Mu), x2::hi(Vu), x2::hi(Cu), x2::hi(h4),
+                                                      noise_pair(k0 + 2, klo, khi), nstep, isb, dec, kc, m23, v23);
+                        const float4 yo = x2::join(y01, y23), mo = x2::join(m01, m23), vo = x2::join(v01, v23);
+                        const int64_t o = i * d.wstride + off;
+                        if (nvalid == 4) {
+                            E::template store4<kSt>(Yw + o, yo);
+                            E::template store4<kSt>(Mw + o, mo);
+                            E::template store4<kSt>(Vw + o, vo);
+                        } else {
+                            const float ya[4] = {yo.x, yo.y, yo.z, yo.w};
+                            const float ma[4] = {mo.x, mo.y, mo.z, mo.w};
+                            const float va[4] = {vo.x, vo.y, vo.z, vo.w};
+                            for (int l = 0; l < nvalid; ++l) {
+                                E::store1(Yw + o + l, ya[l]);
+                                E::store1(Mw + o + l, ma[l]);
+                                E::store1(Vw + o + l, va[l]);
+                            }
                         }
                     }
                 }
             }
+        }
+        __syncthreads();
+        ti = next_tile[par];
+    }
+    // every block has made its last claim before it counts itself out; the
+    // last one returns the counter to 0 for the next launch
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(a.work + 1, 1ull) == gridDim.x - 1ull) {
+            atomicExch(a.work, 0ull);
+            atomicExch(a.work + 1, 0ull);
         }
     }
 }
