@@ -1,16 +1,17 @@
 """gasloc_fused_round: one whole round of Algorithm 1 (H local steps, then the
-gossip round).  For at most 4 workers with fp32 storage and a small store,
-where every worker takes the round's last step from the same iterate, that
-step runs fused with the gossip round in one kernel.  Every step acts on each
+gossip round) with the round's last local step fused into the gossip kernel,
+an opt-in variant outside the one-pass-per-local-step byte model.  It serves
+at most 4 workers with fp32 storage and a small store, where every worker
+takes the round's last step from the same iterate.  Every step acts on each
 parameter index on its own, so the fused round must reproduce the two calls
-bit for bit: every array and the step counters; the consensus error is the
+bit for bit: every array and the step counters.  The consensus error is the
 same sum of the same per-element terms, whose fp64 partial sums the fused
 kernel takes over other tiles (512 elements, its own grid), so it agrees to
-the rounding of the sum order (relative 1e-12).  Where the
-fused kernel runs, a round makes exactly one launch fewer than the two calls;
-elsewhere (more workers, bf16, workers with different step counts, H = 0) the
-same launches.  The oracle checks the fused path directly on every outer mode
-and at the 4-worker 1 Mi-parameter size."""
+the rounding of the sum order (relative 1e-12).  Where the fused kernel
+runs, a round makes exactly one launch fewer than the two calls; elsewhere
+(more workers, bf16, workers with different step counts, H = 0) the same
+launches.  The oracle checks the fused path directly on every outer mode and
+at the 4-worker 1 Mi-parameter size."""
 import numpy as np
 import pytest
 import torch
@@ -69,7 +70,7 @@ CASES = [
 
 @pytest.mark.parametrize("mode", MODES)
 @pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
-def test_outer_round_equals_the_two_calls(case, mode):
+def test_fused_round_equals_the_two_calls(case, mode):
     _, N, P, topo, extra, numels, H, Hi, fused = case
     if numels is not None:
         P = sum(numels)
@@ -96,7 +97,7 @@ def test_outer_round_equals_the_two_calls(case, mode):
 
 
 @pytest.mark.parametrize("mode", MODES)
-def test_outer_round_matches_the_oracle(mode):
+def test_fused_round_matches_the_oracle(mode):
     N, P, R = 4, 3 * 512 + 5, 3
     ctx, st = make_pair(N, P, "matching", seed=44, hp=_outer(mode))
     with ctx:
@@ -109,7 +110,7 @@ def test_outer_round_matches_the_oracle(mode):
             np.testing.assert_array_equal(ctx.read_all(w), st.get_all(w).astype(np.float32), err_msg=w)
 
 
-def test_outer_round_in_the_middle_of_a_round():
+def test_fused_round_in_the_middle_of_a_round():
     # every worker already took a step this round: the fused step starts from y
     hp = _outer("nesterov")
     with _ctx(4, 3000, "ring", 5, hp) as a, _ctx(4, 3000, "ring", 5, hp) as b:
@@ -123,7 +124,7 @@ def test_outer_round_in_the_middle_of_a_round():
         assert a.consensus_error() == pytest.approx(b.consensus_error(), rel=1e-12)
 
 
-def test_outer_round_on_parameter_ranges():
+def test_fused_round_on_parameter_ranges():
     # range contexts (odd cuts: the noise keys follow the global index) add up
     # to the whole context, all of them running fused rounds
     N, P, cuts = 4, 6001, [1, 2501, 4097]
@@ -143,7 +144,7 @@ def test_outer_round_on_parameter_ranges():
             c.close()
 
 
-def test_outer_round_ring_full_size():
+def test_fused_round_ring_full_size():
     """The 4-worker ring on 1 Mi parameters, one local step per round, in the
     launch configuration the benchmark times: fused rounds equal the two calls
     on every element, and the oracle on sampled elements (the tiles' edges and
