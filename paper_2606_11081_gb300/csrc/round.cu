@@ -19,6 +19,11 @@
 // Small stores only: at a few tiles per CTA both separate kernels are bound by
 // their ramp and tail rather than by HBM, and one kernel pays those once.
 //
+// It is an opt-in variant (gasloc_fused_round).  The separate kernels make one
+// HBM pass per local step, the last step's iterate written for the gossip
+// kernel to read back, as where a trainer's gradient arrives between steps;
+// that is the byte model gasloc_run and the benchmark's rounds keep.
+//
 // The step's per-worker scalars come from the step table; the last CTA to
 // have read them (atomic ticket, nothing waits) advances every worker's step
 // counters and writes their next step's scalars while the others work.  The
