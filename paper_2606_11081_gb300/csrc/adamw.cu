@@ -268,6 +268,11 @@ __device__ __forceinline__ void mbar_release(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ptx::smem_addr(bar)) : "memory");
 }
 
+// Barrier of the staged kernel's consumer warps only (the producer does not take part).
+__device__ __forceinline__ void staged_consumer_sync() {
+    asm volatile("barrier.sync 1, %0;" ::"r"(kStagedConsumers) : "memory");
+}
+
 template <bool PER_WORKER_H, bool SCHED, typename T = bf16>
 __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::kMinBlocks)
     adamw_staged_kernel(const AdamwArgs a) {
@@ -282,11 +287,8 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
     uint64_t *empty = full + kStages;
     UnitDesc *descs = reinterpret_cast<UnitDesc *>(smem + SS::kDescOffset);
     __shared__ StepTable tab;
-    __shared__ int last_copy;
     __shared__ int abort_flag;
 
-    for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += blockDim.x)
-        reinterpret_cast<uint32_t *>(&tab)[q] = reinterpret_cast<const uint32_t *>(a.table)[q];
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&full[s], 1);
@@ -295,17 +297,7 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
         ptx::fence_mbar_init();
         abort_flag = 0;
     }
-    __syncthreads();
-    // the last CTA to have copied the scalars advances the counters and
-    // writes the next step's scalars (as in adamw_kernel)
-    if (threadIdx.x == 0) last_copy = atomicAdd(a.ticket, 1u) == gridDim.x - 1u;
-    __syncthreads();
-    if (last_copy && threadIdx.x < 32) {
-        const int i = threadIdx.x;
-        if (i < a.n_workers && ((a.active_mask >> i) & 1u))
-            advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd, a.seed);
-        if (i == 0) *a.ticket = 0u;
-    }
+    __syncthreads();   // the producer starts its copies at once; the consumers first copy the step's scalars
 
     // units of this CTA: its tiles (grid stride) x the groups of G active workers
     // units: the tiles x the groups of G active workers (unit u: tile
@@ -426,6 +418,24 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
     }
 
     // ------------------------------------------------------------ consumers ---
+    for (int q = threadIdx.x; q < static_cast<int>(sizeof(StepTable) / 4); q += kStagedConsumers)
+        reinterpret_cast<uint32_t *>(&tab)[q] = reinterpret_cast<const uint32_t *>(a.table)[q];
+    staged_consumer_sync();
+    // the last CTA to have copied the scalars advances the counters and
+    // writes the next step's scalars (as in adamw_kernel); only warp 0 waits
+    // for the ticket, the other warps go on to the first unit
+    if (threadIdx.x < 32) {
+        unsigned t = 0;
+        if (lane == 0) t = atomicAdd(a.ticket, 1u);
+        t = __shfl_sync(0xffffffffu, t, 0);
+        if (t == gridDim.x - 1u) {
+            const int i = lane;
+            if (i < a.n_workers && ((a.active_mask >> i) & 1u))
+                advance_step(a.state, a.table, i, a.beta1d, a.beta2d, a.lr_sched, a.lr_steps, a.lr_after, a.wd,
+                             a.seed);
+            if (i == 0) *a.ticket = 0u;
+        }
+    }
     const Consts kc{x2::splat(a.beta1), x2::splat(a.beta2), x2::splat(a.omb1), x2::splat(a.omb2),
                     x2::splat(a.eps), x2::splat(a.sigma)};
     const int e0 = 4 * threadIdx.x;

@@ -597,11 +597,11 @@ template <int MODE>
 __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const GossipArgs a) {
     using R = ModeRows<MODE>;
     using E = Elem<float>;
-    __shared__ Topo tp;
+    __shared__ DenseRows dr;
     __shared__ double red[kDirectThreads / 32];
     __shared__ int last;
     const int n = a.n_workers;
-    copy_topo_rows(a.topo, tp, n, blockDim.x);
+    dense_rows(a.topo, dr, n, a.err);
     __syncthreads();
     const int64_t round = __ldcg(&a.state->round);
     const OuterK ok2{x2::splat(-a.eta_out), x2::splat(a.mu), x2::splat(a.alpha), x2::splat(a.oma),
@@ -639,7 +639,7 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
             rows[1][j] = E::load4<Cache::kL2>(k1 + o);
             if (R::kHasB) rows[R::kRows - 1][j] = E::load4<Cache::kL2>(B + o);
         }
-        column_update<MODE, 4>(rows, tp, n, ok2, round == 0, static_cast<float *>(d.x), static_cast<float *>(d.b),
+        column_update<MODE, 4>(rows, dr, n, ok2, round == 0, static_cast<float *>(d.x), static_cast<float *>(d.b),
                                d.wstride, off, tl.len - e0 < 4 ? tl.len - e0 : 4, inv_n, ce_acc, a.err);
     }
     // one partial per CTA; the last CTA adds them in CTA order, stores the

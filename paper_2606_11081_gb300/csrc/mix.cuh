@@ -106,25 +106,55 @@ struct Col<4> {
     static __device__ __forceinline__ void store(float *p, float4 v) { __stcg(reinterpret_cast<float4 *>(p), v); }
 };
 
-// The first n rows of the round's neighbour table into shared memory, by
-// threads 0..nthreads-1 (the caller synchronises them).
-__device__ __forceinline__ void copy_topo_rows(const Topo *src, Topo &tp, int n, int nthreads) {
-    for (int q = threadIdx.x; q < n * kMaxWorkers; q += nthreads) {
-        const int i = q / kMaxWorkers, c = q % kMaxWorkers;
-        tp.nbr[i][c] = src->nbr[i][c];
-        tp.w[i][c] = src->w[i][c];
+// The round's neighbour table for n <= kColumnWorkers workers in dense form:
+// bit j of mask[i] is set iff j is in N_i (i itself included), with weight
+// w[i][j] (0 elsewhere).  The table lists N_i once each, in ascending order,
+// so mixing over j = 0..n-1 where the bit is set takes the terms of the list
+// in its order: the same sums.  A thread holding every worker's rows in
+// registers then indexes them statically, where following the list would
+// select each neighbour's row out of the n with a chain of selects.
+struct DenseRows {
+    float w[kColumnWorkers][kColumnWorkers];
+    uint32_t mask[kColumnWorkers];
+};
+
+// Row i built by thread i < n from the table in global memory (the caller
+// synchronises before use).  The first kColumnWorkers entries of a row are
+// read at once; entries past the degree are not used.
+__device__ __forceinline__ void dense_rows(const Topo *src, DenseRows &dr, int n, int32_t *err) {
+    const int i = threadIdx.x;
+    if (i >= n || i >= kColumnWorkers) return;
+    int32_t nb[kColumnWorkers];
+    float wq[kColumnWorkers];
+    const int dg = src->deg[i];
+#pragma unroll
+    for (int q = 0; q < kColumnWorkers; ++q) {
+        nb[q] = src->nbr[i][q];
+        wq[q] = src->w[i][q];
+        dr.w[i][q] = 0.f;
     }
-    if (threadIdx.x < n) tp.deg[threadIdx.x] = src->deg[threadIdx.x];
+    uint32_t m = 0;
+    if (span_ok(dg, dg + 1, kColumnWorkers, err)) {
+#pragma unroll
+        for (int q = 0; q < kColumnWorkers; ++q) {
+            if (q > dg) break;
+            const int j = nb[q];
+            if (!span_ok(j, j + 1, n, err)) continue;
+            m |= 1u << j;
+            dr.w[i][j] = wq[q];
+        }
+    }
+    dr.mask[i] = m;
 }
 
 // One column of V elements for every worker (n <= kColumnWorkers) from the
 // rows held in registers (rows[kind][worker], kinds as ModeRows): the mixing
-// over the round's neighbour lists, the outer update, the stores of x and b
+// over the round's neighbours (dense form), the outer update, the stores of x and b
 // at X / B + worker * wstride + off (nvalid <= V elements), and the column's
 // consensus-error terms added to ce_acc element by element.
 template <int MODE, int V>
 __device__ __forceinline__ void column_update(const typename Col<V>::T (&rows)[ModeRows<MODE>::kRows][kColumnWorkers],
-                                              const Topo &tp, int n, const OuterK &ok2, bool first_round, float *X,
+                                              const DenseRows &dr, int n, const OuterK &ok2, bool first_round, float *X,
                                               float *B, int64_t wstride, int64_t off, int nvalid, float inv_n,
                                               double &ce_acc, int32_t *err) {
     using R = ModeRows<MODE>;
@@ -140,24 +170,16 @@ __device__ __forceinline__ void column_update(const typename Col<V>::T (&rows)[M
         float2 acc[NP];
 #pragma unroll
         for (int p = 0; p < NP; ++p) acc[p] = x2::splat(0.f);
-        int dg = tp.deg[i];
-        if (!span_ok(dg, dg + 1, kMaxWorkers, err)) dg = -1;
-        for (int q = 0; q <= dg; ++q) {
-            const int j = tp.nbr[i][q];
-            if (!span_ok(j, j + 1, n, err)) continue;
-            const float2 w = x2::splat(tp.w[i][q]);
-            T sj = rows[0][0], xj = rows[R::kRows > 1 ? 1 : 0][0];
+        const uint32_t mi = dr.mask[i];
 #pragma unroll
-            for (int jj = 1; jj < kColumnWorkers; ++jj)   // register select, no dynamic index
-                if (jj == j) {
-                    sj = rows[0][jj];
-                    if (MODE == kOutEq2) xj = rows[1][jj];
-                }
+        for (int j = 0; j < kColumnWorkers; ++j) {   // ascending j, as the neighbour list
+            if (!((mi >> j) & 1u)) continue;
+            const float2 w = x2::splat(dr.w[i][j]);
 #pragma unroll
             for (int p = 0; p < NP; ++p) {
-                float2 s = C::pair(sj, p);
+                float2 s = C::pair(rows[0][j], p);
                 if (MODE == kOutEq2) {   // z_j = x_j + eta (y_j - x_j)
-                    const float2 xp = C::pair(xj, p);
+                    const float2 xp = C::pair(rows[1][j], p);
                     s = x2::fma(ok2.eta, x2::sub(s, xp), xp);
                 }
                 acc[p] = x2::fma(w, s, acc[p]);

@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const Round
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + RR::kBarOffset);
     uint64_t *empty = full + kStages;
     TileDesc *descs = reinterpret_cast<TileDesc *>(smem + RR::kDescOffset);
-    __shared__ Topo tp;
+    __shared__ DenseRows dr;
     __shared__ float s_nstep[kColumnWorkers], s_isb[kColumnWorkers], s_dec[kColumnWorkers];
     __shared__ uint32_t s_klo[kColumnWorkers], s_khi[kColumnWorkers];
     __shared__ double red[kThreads / 32];
@@ -200,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const Round
         }
     } else {
         // ------------------------------------------------------------ consumers ---
-        copy_topo_rows(a.topo, tp, n, kConsumers);
+        dense_rows(a.topo, dr, n, a.err);
         if (threadIdx.x < n) {   // this step's scalars of worker i
             const int i = threadIdx.x;
             s_nstep[i] = -a.table->step[i];
@@ -286,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const Round
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);   // every row of the stage is read
             if (active)
-                column_update<MODE, kV>(rows, tp, n, ok2, round == 0, u.x, u.b, u.wstride, off, nvalid, inv_n,
+                column_update<MODE, kV>(rows, dr, n, ok2, round == 0, u.x, u.b, u.wstride, off, nvalid, inv_n,
                                         ce_acc, a.err);
         }
         if (abort_flag) ce_acc = __longlong_as_double(0x7ff8000000000000ll);
