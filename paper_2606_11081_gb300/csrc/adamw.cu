@@ -317,6 +317,10 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
         int64_t issued = 0;
         bool aborted = false;
         unsigned long long next = 0;   // the unit claimed for the next stage (lane 0's claim, broadcast)
+        // tensor 0's descriptor read at once, beside the first tile's (a flat
+        // store has no other)
+        int32_t cur = 0;
+        TensorDesc d = a.tens[0];
         if (SS::kDynamic) {
             if (lane == 0) next = atomicAdd(a.work, 1ull);
             next = __shfl_sync(0xffffffffu, next, 0);
@@ -355,7 +359,10 @@ __global__ void __launch_bounds__(kStagedThreads, StagedShape<T, PER_WORKER_H>::
             const int64_t ti = static_cast<int64_t>(unit / ngroups);
             const int a0 = static_cast<int>(unit % ngroups) * G;
             const Tile tl = a.tiles[ti];
-            const TensorDesc &d = a.tens[tl.tensor];
+            if (tl.tensor != cur) {
+                d = a.tens[tl.tensor];
+                cur = tl.tensor;
+            }
             const int nw = a.n_active - a0 < G ? a.n_active - a0 : G;
             const int lenr = (tl.len + kVec - 1) / kVec * kVec;   // whole 16-byte pieces (the row padding is allocated)
             const uint32_t bytes = static_cast<uint32_t>(lenr) * sizeof(T);

@@ -610,8 +610,10 @@ __global__ void __launch_bounds__(kDirectThreads, 2) gossip_direct_kernel(const 
     const uint32_t fresh = a.fresh_mask;
     double ce_acc = 0.0;
     const int e0 = 4 * threadIdx.x;
-    int32_t cur = -1;
-    TensorDesc d{};
+    // tensor 0's descriptor read at once, beside the first tile's (a flat
+    // store has no other)
+    int32_t cur = 0;
+    TensorDesc d = a.tens[0];
     for (int64_t ti = blockIdx.x; ti < a.ntiles; ti += gridDim.x) {
         const Tile tl = a.tiles[ti];
         if (e0 >= tl.len) continue;

@@ -129,6 +129,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const Round
         const int ncopies = nrows + (PER_WORKER_H ? 0 : 1);
         int64_t issued = 0;
         bool aborted = false;
+        // tensor 0's descriptor read at once, beside the first tile's (a flat
+        // store has no other)
+        int32_t cur = 0;
+        TensorDesc d = a.tens[0];
         for (int64_t it = 0; it < my_n; ++it) {
             const int s = static_cast<int>(it % kStages);
             if (it >= kStages) {
@@ -144,7 +148,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) round_kernel(const Round
                 break;
             }
             const Tile tl = a.tiles[blockIdx.x + it * gridDim.x];
-            const TensorDesc &d = a.tens[tl.tensor];
+            if (tl.tensor != cur) {
+                d = a.tens[tl.tensor];
+                cur = tl.tensor;
+            }
             const int lenr = (tl.len + 3) & ~3;   // whole 16-byte pieces (the row padding is allocated)
             const uint32_t bytes = static_cast<uint32_t>(lenr) * sizeof(float);
             if (lane == 0) {

@@ -154,11 +154,15 @@ def test_bf16_host_transfer_over_staging_chunks():
 
 @pytest.mark.parametrize("storage", ["f32", "bf16"])
 @pytest.mark.parametrize("N,topo,kw", [(8, "ring", {}), (8, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
-                                       (6, "2peer", {"weights": "lazy"})])
+                                       (6, "2peer", {"weights": "lazy"}), (4, "ring", {}),
+                                       (4, "exp", {"weights": "metropolis", "edge_prob": 0.5}),
+                                       (4, "2peer", {"weights": "lazy"})])
 def test_nonfinite_replica_reaches_neighbours_only(storage, N, topo, kw):
     # A diverged replica (inf in some elements of worker j) is mixed only by
     # the workers whose neighbourhood holds j, as in the oracle's neighbour
-    # lists; the dense bf16 mixing at n <= 8 must not carry it elsewhere.
+    # lists; the dense mixing forms (bf16 at n <= 8, and the fp32 kernel that
+    # holds a column of every worker in registers at n <= 4) must not carry
+    # it elsewhere.
     P = 2 * 1024 + 5
     hp = dict(kw, storage=storage, outer="nesterov")
     ctx, st = make_pair(N, P, topo, seed=900 + N, hp=hp)
