@@ -32,9 +32,10 @@
 // Consensus error: per element e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
 // S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x; fp32 per
 // element (the thread owning the column, or for G > 1 one thread per column
-// after the tile's barrier), each element's term widened to fp64 on its own,
-// one partial per CTA, the last CTA (atomic ticket, nothing waits) adds the
-// partials in CTA order.
+// after the tile's barrier), each element's term widened to fp64 on its own
+// (the direct kernel below: a column's four terms as their exact sum,
+// ce_sum.cuh), one partial per CTA, the last CTA (atomic ticket, nothing
+// waits) adds the partials in CTA order.
 //
 // Waiting: every mbarrier wait is bounded (2 s).  A consumer that times out
 // records kDevWaitTimeout and the CTA stops computing but keeps arriving on

@@ -9,11 +9,14 @@
 //   Nesterov: D = x - acc; b = fma(mu, b, D); x = fma(-eta_out, fma(mu, b, D), x)
 //   (SGD, SGDM, Eq. 2, DAdam, Local-DAdam: see outer_pair)
 // and the consensus-error term e = S2 - (S1/n) S1 with S1 = sum_i (x_i - s),
-// S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x, in fp32,
-// widened to fp64 on its own.
+// S2 = sum_i (x_i - s)^2 over ascending i, s = worker 0's new x, in fp32.
+// In the whole-column update a 4-element column's terms enter the thread's
+// fp64 sum as their exact sum, a 2-element column's one at a time
+// (ce_sum.cuh); elsewhere each term is widened and added on its own.
 #pragma once
 #include <cstdint>
 
+#include "ce_sum.cuh"
 #include "check.cuh"
 #include "f32x2.cuh"
 #include "internal.h"
@@ -151,7 +154,7 @@ __device__ __forceinline__ void dense_rows(const Topo *src, DenseRows &dr, int n
 // rows held in registers (rows[kind][worker], kinds as ModeRows): the mixing
 // over the round's neighbours (dense form), the outer update, the stores of x and b
 // at X / B + worker * wstride + off (nvalid <= V elements), and the column's
-// consensus-error terms added to ce_acc element by element.
+// consensus-error terms added to ce_acc (ce_sum.cuh).
 template <int MODE, int V>
 __device__ __forceinline__ void column_update(const typename Col<V>::T (&rows)[ModeRows<MODE>::kRows][kColumnWorkers],
                                               const DenseRows &dr, int n, const OuterK &ok2, bool first_round, float *X,
@@ -222,13 +225,14 @@ __device__ __forceinline__ void column_update(const typename Col<V>::T (&rows)[M
             }
         }
     }
+    float e[V];   // the column's terms (0 past the tile's end)
 #pragma unroll
-    for (int l = 0; l < V; ++l) {   // each element's term enters the fp64 sum on its own
-        if (l >= nvalid) continue;
+    for (int l = 0; l < V; ++l) {
         const float a = (l & 1) ? s1[l >> 1].y : s1[l >> 1].x;
         const float q = (l & 1) ? s2[l >> 1].y : s2[l >> 1].x;
-        ce_acc += static_cast<double>(__fmaf_rn(-__fmul_rn(a, inv_n), a, q));
+        e[l] = l < nvalid ? __fmaf_rn(-__fmul_rn(a, inv_n), a, q) : 0.f;
     }
+    ce_add_group<V>(e, ce_acc);
 }
 
 // ---------------------------------------------------------------------------
