@@ -234,7 +234,7 @@ def test_consensus_error_closed_form_and_paths():
         assert ctx.consensus_error_now() == pytest.approx(fused, rel=1e-12)
 
 
-@pytest.mark.parametrize("N", [8, 32])
+@pytest.mark.parametrize("N", [4, 8, 32])
 def test_consensus_error_near_consensus_far_from_zero(N):
     # Replicas a thousand times further from zero than from each other:
     # x_ik = a_k + 1e-3 (i - (N-1)/2) with a_k in [1000, 2000).  A one-pass
@@ -269,6 +269,52 @@ def test_consensus_error_near_consensus_far_from_zero(N):
         assert ref == pytest.approx(P * 1e-6 * (N * N - 1) / 12, rel=0.05)
         for got in (now, fused):
             assert got == pytest.approx(exact, rel=tol), (got, exact, tol)
+
+
+@pytest.mark.parametrize("N", [3, 4])
+def test_consensus_error_column_sums_over_wide_magnitudes(N):
+    # The kernel that holds a column of every worker in registers (at most 4
+    # workers, fp32) adds a column's four terms as their exact sum when they
+    # lie within 2^26 of the column's largest, and adds the others (smaller,
+    # subnormal or zero) one at a time.  Element scales spread over 10^-25 ..
+    # 10^10 put every case into most columns: the largest terms near 10^20,
+    # terms many binades below them, subnormal terms and exact zeros.  The
+    # standalone reduction adds every term on its own, so the two differ only
+    # in the order of their fp64 additions; both are within the shifted
+    # form's bound of the exact value.
+    P = 5 * 1024 + 7
+    hp = dict(outer="sgd", outer_lr=0.0)        # the gossip round leaves x as it is
+    ctx, st = make_pair(N, P, "ring", seed=40 + N, hp=hp)
+    rng = np.random.default_rng(N)
+    scale = 10.0 ** rng.uniform(-25.0, 10.0, P)
+    scale[rng.random(P) < 0.1] = 0.0            # some columns hold equal replicas: terms of exactly 0
+    x = np.stack([(scale * ((i - (N - 1) / 2) + 0.3 * rng.standard_normal(P))).astype(np.float32)
+                  for i in range(N)])
+    xd = x.astype(np.float64)
+    exact = ((xd - xd.mean(0)) ** 2).sum() / N
+    with ctx:
+        for i in range(N):
+            ctx.write("x", i, x[i])
+            st.set("x", i, xd[i])
+        now = ctx.consensus_error_now()                 # every term added on its own
+        ctx.gossip_round()                              # column sums, in the register-column kernel
+        np.testing.assert_array_equal(ctx.read_all("x"), x)
+        fused = ctx.consensus_error()
+        st.gossip_round()
+        assert st.consensus_error() == pytest.approx(exact, rel=1e-12)
+        assert fused == pytest.approx(now, rel=1e-12)
+        tol = ce_bound(xd)
+        for got in (now, fused):
+            assert got == pytest.approx(exact, rel=tol), (got, exact, tol)
+        # a non-finite replica value makes the round's value non-finite in
+        # both reductions (the whole column is then added term by term)
+        bad = ctx.read("x", 1)
+        bad[1030] = np.inf
+        ctx.write("x", 1, bad)
+        ctx.gossip_round()
+        fused = ctx.consensus_error()
+        assert not np.isfinite(fused)
+        assert not np.isfinite(ctx.consensus_error_now())
 
 
 @pytest.mark.parametrize("storage", ["f32", "bf16"])
