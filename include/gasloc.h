@@ -236,9 +236,10 @@ int gasloc_fused_round(gasloc_ctx *ctx, int32_t H);
 /* Runs `rounds` complete outer rounds -- H local steps (H > 0, or
  * GASLOC_PER_WORKER_STEPS for each worker's H_i, or 0) followed by a gossip
  * round -- exactly as that many gasloc_local_steps + gasloc_gossip_round
- * calls would, but replayed from a CUDA graph of one round that is captured
- * on the first call and reused until the hyperparameters, H or the H_i
- * change.  Every per-step scalar is derived on the device from device-resident
+ * calls would, but replayed from CUDA graphs: one of 8 consecutive rounds
+ * while at least 8 are left, one of a single round for the rest.  Each is
+ * captured when first needed and reused until the hyperparameters, H or the
+ * H_i change.  Every per-step scalar is derived on the device from device-resident
  * step counters, so the replayed rounds need no host work.  Must start at a
  * round boundary (ESTATE otherwise).  If ce_trace_host is not NULL it
  * receives the consensus error of each round (rounds <= 4096) and the call

@@ -47,6 +47,8 @@ constexpr int64_t kPadFloats = 64;
 constexpr int kTileA = 1024;          // init / adamw / ce / average tiles (4 x 256 threads)
 constexpr int kMaxLocalSteps = 1024;
 constexpr int kCeRing = 4096;
+// Rounds per replay of gasloc_run's longer graph (a single-round graph takes the rest).
+constexpr int32_t kGraphBlock = 8;
 constexpr int64_t kMaxScheduleSteps = int64_t(1) << 24;
 constexpr int kDirectTilesPerCta = 8;   // the direct gossip variant up to this many 1024-element tiles per CTA
 constexpr int kStagedTilesPerCta = 8;   // fp32 stores take the staged AdamW up to this many tiles per CTA
@@ -152,6 +154,10 @@ struct gasloc_ctx {
     int32_t graph_H = 0;
     uint64_t graph_gen = 0, gen = 1; // configuration generation the graph was built for
     int64_t graph_launches = 0;      // kernels per replayed round
+    cudaGraphExec_t graph_blk = nullptr;   // kGraphBlock consecutive rounds, for longer runs
+    int32_t graph_blk_H = 0;
+    uint64_t graph_blk_gen = 0;
+    int64_t graph_blk_launches = 0;  // kernels per replay of the block
     int32_t *err_d = nullptr;
     void *pinned = nullptr;   // [ce double][err int32][Topo]
     std::vector<std::pair<void *, size_t>> allocs;
@@ -201,6 +207,8 @@ struct gasloc_ctx {
         if (started || !allocs.empty()) cudaStreamSynchronize(stream);
         if (graph) cudaGraphExecDestroy(graph);
         graph = nullptr;
+        if (graph_blk) cudaGraphExecDestroy(graph_blk);
+        graph_blk = nullptr;
         if (cap_stream) cudaStreamDestroy(cap_stream);
         cap_stream = nullptr;
         for (auto &pr : allocs) {
@@ -1025,6 +1033,60 @@ int check_H(const gasloc_ctx *c, int32_t H) {
     return GASLOC_OK;
 }
 
+// Captures nr consecutive rounds (H local steps, then gossip) into an
+// executable graph.  The step table is refreshed and a static neighbour
+// table built outside the graph, so a replay holds AdamW, the round's table
+// where it is drawn each round, and gossip.  Every kernel reads its round
+// and step counters from device memory, so consecutive rounds in one graph
+// are the rounds the calls would run.  The host mirrors are restored after
+// the capture; the caller advances them once per replayed round.
+int capture_rounds(gasloc_ctx *c, int32_t H, int32_t nr, cudaGraphExec_t *out, int64_t *launches_out) {
+    if (*out) cudaGraphExecDestroy(*out);
+    *out = nullptr;
+    if (!c->cap_stream && cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
+        cudaGetLastError();
+        return fail(GASLOC_ECUDA, "creating the capture stream failed");
+    }
+    int rc = refresh_step_table(c, c->stream);
+    if (rc) return rc;
+    if (c->topo_static && !c->topo_ready) {
+        rc = build_topology(c, c->round, nullptr, c->topo_d, c->stream);
+        if (rc) return rc;
+        c->topo_ready = true;
+    }
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    const std::vector<int64_t> nsteps0 = c->nsteps;
+    const int64_t round0 = c->round, launches0 = c->launches;
+    const bool ce0 = c->ce_valid;
+    e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) return cuda_fail(e, "begin capture");
+    for (int32_t r = 0; r < nr && !rc; ++r) {
+        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, c->cap_stream);
+        if (!rc) rc = enqueue_gossip(c, c->cap_stream);
+    }
+    cudaGraph_t g = nullptr;
+    const cudaError_t e2 = cudaStreamEndCapture(c->cap_stream, &g);
+    *launches_out = c->launches - launches0;
+    c->nsteps = nsteps0;
+    c->round = round0;
+    c->launches = launches0;
+    c->ce_valid = ce0;
+    c->fresh_mask = 0;
+    if (rc) {
+        if (g) cudaGraphDestroy(g);
+        return rc;
+    }
+    if (e2 != cudaSuccess) return cuda_fail(e2, "end capture");
+    e = cudaGraphInstantiate(out, g, 0);
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) {
+        *out = nullptr;
+        return cuda_fail(e, "graph instantiate");
+    }
+    return GASLOC_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -1067,60 +1129,27 @@ int gasloc_run(gasloc_ctx *c, int32_t rounds, int32_t H, double *ce_trace_host) 
     if (rounds == 0) return GASLOC_OK;
     const int64_t r0 = c->round;
     if (!c->graph || c->graph_gen != c->gen || c->graph_H != H) {
-        if (c->graph) cudaGraphExecDestroy(c->graph);
-        c->graph = nullptr;
-        if (!c->cap_stream && cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess) {
-            cudaGetLastError();
-            return fail(GASLOC_ECUDA, "creating the capture stream failed");
-        }
-        // the step table is refreshed and a static neighbour table built
-        // outside the graph (the replayed round holds AdamW and gossip only)
-        rc = refresh_step_table(c, c->stream);
+        rc = capture_rounds(c, H, 1, &c->graph, &c->graph_launches);
         if (rc) return rc;
-        if (c->topo_static && !c->topo_ready) {
-            rc = build_topology(c, c->round, nullptr, c->topo_d, c->stream);
-            if (rc) return rc;
-            c->topo_ready = true;
-        }
-        cudaError_t e = cudaStreamSynchronize(c->stream);
-        if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
-        // capture one round; the host mirrors are restored afterwards and
-        // advanced once per replay
-        const std::vector<int64_t> nsteps0 = c->nsteps;
-        const int64_t round0 = c->round, launches0 = c->launches;
-        const bool ce0 = c->ce_valid;
-        e = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
-        if (e != cudaSuccess) return cuda_fail(e, "begin capture");
-        rc = H == 0 ? GASLOC_OK : enqueue_local_steps(c, H, c->cap_stream);
-        if (!rc) rc = enqueue_gossip(c, c->cap_stream);
-        cudaGraph_t g = nullptr;
-        const cudaError_t e2 = cudaStreamEndCapture(c->cap_stream, &g);
-        c->graph_launches = c->launches - launches0;
-        c->nsteps = nsteps0;
-        c->round = round0;
-        c->launches = launches0;
-        c->ce_valid = ce0;
-        c->fresh_mask = 0;
-        if (rc) {
-            if (g) cudaGraphDestroy(g);
-            return rc;
-        }
-        if (e2 != cudaSuccess) return cuda_fail(e2, "end capture");
-        e = cudaGraphInstantiate(&c->graph, g, 0);
-        cudaGraphDestroy(g);
-        if (e != cudaSuccess) {
-            c->graph = nullptr;
-            return cuda_fail(e, "graph instantiate");
-        }
         c->graph_gen = c->gen;
         c->graph_H = H;
     }
-    for (int32_t r = 0; r < rounds; ++r) {
-        const cudaError_t e = cudaGraphLaunch(c->graph, c->stream);
+    if (rounds >= kGraphBlock && (!c->graph_blk || c->graph_blk_gen != c->gen || c->graph_blk_H != H)) {
+        rc = capture_rounds(c, H, kGraphBlock, &c->graph_blk, &c->graph_blk_launches);
+        if (rc) return rc;
+        c->graph_blk_gen = c->gen;
+        c->graph_blk_H = H;
+    }
+    // blocks of kGraphBlock rounds while that many are left, then single rounds
+    for (int32_t r = 0; r < rounds;) {
+        const bool blk = rounds - r >= kGraphBlock;
+        const cudaError_t e = cudaGraphLaunch(blk ? c->graph_blk : c->graph, c->stream);
         if (e != cudaSuccess) return cuda_fail(e, "graph launch");
-        for (int32_t i = 0; i < c->n; ++i) c->nsteps[i] += H < 0 ? c->Hi[i] : H;
-        c->round += 1;
-        c->launches += c->graph_launches;
+        const int32_t nr = blk ? kGraphBlock : 1;
+        for (int32_t i = 0; i < c->n; ++i) c->nsteps[i] += static_cast<int64_t>(nr) * (H < 0 ? c->Hi[i] : H);
+        c->round += nr;
+        c->launches += blk ? c->graph_blk_launches : c->graph_launches;
+        r += nr;
     }
     c->ce_valid = true;
     if (ce_trace_host) {

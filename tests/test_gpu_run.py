@@ -1,7 +1,9 @@
-"""gasloc_run: rounds replayed from a CUDA graph must be exactly the rounds
-the call-by-call API produces (and the oracle's), including random per-round
-graphs (the round number is read on the device), per-worker step counts, a
-hyperparameter change (a new graph is captured) and the consensus-error trace."""
+"""gasloc_run: rounds replayed from CUDA graphs (one of 8 consecutive rounds
+while that many are left, one of a single round for the rest) must be
+exactly the rounds the call-by-call API produces (and the oracle's),
+including random per-round graphs (the round number is read on the device),
+per-worker step counts, a hyperparameter change (new graphs are captured)
+and the consensus-error trace."""
 import numpy as np
 import pytest
 
@@ -34,7 +36,8 @@ CASES = [
 
 @pytest.mark.parametrize("N,topo,kw,H,Hi", CASES)
 def test_run_matches_stepwise_and_oracle(N, topo, kw, H, Hi):
-    P, R = 3 * 1024 + 7, 6
+    # 19 rounds: two replays of the 8-round graph, then three single rounds
+    P, R = 3 * 1024 + 7, 19
     hp = dict(kw, lr=2e-3)
     a, st = make_pair(N, P, topo, seed=42, hp=hp, Hi=Hi)
     b, _ = make_pair(N, P, topo, seed=42, hp=hp, Hi=Hi)
@@ -67,15 +70,15 @@ def test_hparam_change_recaptures():
     a, _ = make_pair(8, P, "exp", seed=7, hp=dict(lr=1e-3))
     b, _ = make_pair(8, P, "exp", seed=7, hp=dict(lr=1e-3))
     with a, b:
-        a.run(3, 1)
-        for _ in range(3):
+        a.run(10, 1)          # both graphs captured: 8 rounds, then 1 + 1
+        for _ in range(10):
             b.local_steps(1)
             b.gossip_round()
         hp2 = g.make_hparams(**dict(wl.COMMON_HP, lr=4e-3, outer="sgdm", outer_momentum=0.5))
         a.set_hparams(hp2)
         b.set_hparams(hp2)
-        a.run(4, 2)
-        for _ in range(4):
+        a.run(12, 2)          # both captured again for the new settings and H
+        for _ in range(12):
             b.local_steps(2)
             b.gossip_round()
         np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
