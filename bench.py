@@ -641,7 +641,8 @@ def main():
                                   "frac_of_nominal_8tbs":
                                       (adamw_bytes + gossip_bytes) / (ms / K / 1e3) / 1e9 / NOMINAL_HBM_GBS}},
             "graph": {"ms_per_step": graph_ms, "value": units / (graph_ms * K / 1e3),
-                      "note": "the same rounds through gasloc_run (one captured round replayed), "
+                      "note": "the same rounds through gasloc_run (graphs of 8 captured rounds replayed, single "
+                              "rounds for the rest), "
                               "timed after the main measurement; this GPU's parameters (its range when "
                               "the replicas are split over GPUs)"},
             "fused_round": fused,
