@@ -65,6 +65,32 @@ def test_run_matches_stepwise_and_oracle(N, topo, kw, H, Hi):
         np.testing.assert_array_equal(a.read_all("x"), b.read_all("x"))
 
 
+def test_long_run_matches_stepwise_and_oracle():
+    # 75 rounds: nine replays of the 8-round graph, then three single rounds;
+    # random per-round graphs and per-worker step counts make every round
+    # differ, and the trace holds every round's value
+    N, P, R, Hi = 6, 2 * 1024 + 9, 75, [1, 3, 2, 1, 2, 3]
+    hp = dict(weights="metropolis", edge_prob=0.5, per_worker_h=True, lr=2e-3)
+    a, st = make_pair(N, P, "exp", seed=17, hp=hp, Hi=Hi)
+    b, _ = make_pair(N, P, "exp", seed=17, hp=hp, Hi=Hi)
+    with a, b:
+        trace = a.run(R, g.PER_WORKER_STEPS, trace=True)
+        ces = []
+        for _ in range(R):
+            b.local_steps(g.PER_WORKER_STEPS)
+            b.gossip_round()
+            ces.append(b.consensus_error())
+            st.local_steps(0, np.array(Hi, np.int32))
+            st.gossip_round()
+        np.testing.assert_array_equal(trace, np.array(ces))
+        assert a.round == b.round == R
+        for i in range(N):
+            assert a.steps_taken(i) == b.steps_taken(i) == st.steps_taken(i)
+        for w in ("x", "b", "m", "v", "y"):
+            np.testing.assert_array_equal(a.read_all(w), b.read_all(w), err_msg=w)
+        np.testing.assert_array_equal(a.read_all("x"), st.get_all("x").astype(np.float32))
+
+
 def test_hparam_change_recaptures():
     P = 5000
     a, _ = make_pair(8, P, "exp", seed=7, hp=dict(lr=1e-3))
