@@ -663,8 +663,9 @@ def main():
 
 
 def measure_graph(ctx, torch, stream, K, H):
-    """Mean round time (ms) of K rounds run by gasloc_run from its CUDA graph."""
-    ctx.run(1, H)   # capture (and one round)
+    """Mean round time (ms) of K rounds run by gasloc_run from its CUDA graphs
+    (of 8 rounds and of one, both captured before the timed region)."""
+    ctx.run(9 if K >= 8 else 1, H)   # captures (and 9 or 1 rounds)
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
